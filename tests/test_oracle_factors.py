@@ -1,0 +1,126 @@
+"""Pins of the factor generator (Sec. III, Eq. 1) against mathematics and LAPACK.
+
+Each test fixes a property that a plausible mistake would break:
+* prune(): brute-force ranking and the tie rule (wrong key, wrong order);
+* keep = 1 (no pruning): the residual scheme is Eckart-Young deflation, so
+  sigma_n equal the singular values of W and K = R steps rebuild W exactly
+  (a residual formed with the wrong sign or never updated fails);
+* any keep: ||R^(n+1)||_F^2 = ||R^(n)||_F^2 - sigma_n^2 ||v'_n||^2 exactly,
+  because u^T R = sigma v^T; pruning u, or subtracting the unpruned term,
+  or a transposed residual, breaks the identity.
+"""
+import numpy as np
+import pytest
+
+from oracle import factors as F
+from workloads import draw_weight, nz_from_keep
+
+
+def _brute_prune(v, nz):
+    pairs = sorted(((-abs(float(x)), i) for i, x in enumerate(v)))
+    kept = sorted(i for _, i in pairs[:nz])
+    return kept
+
+
+@pytest.mark.parametrize("C,nz", [(7, 1), (7, 3), (7, 7), (128, 64), (300, 31)])
+def test_prune_matches_brute_force(C, nz):
+    rng = np.random.default_rng(C * 131 + nz)
+    for _ in range(5):
+        v = rng.standard_normal(C)
+        idx, val = F.prune(v, nz)
+        assert list(idx) == _brute_prune(v, nz)
+        assert np.array_equal(val, v[idx])
+        assert idx.dtype == np.int32 and np.all(np.diff(idx) > 0)
+        dropped = np.setdiff1d(np.arange(C), idx)
+        if dropped.size:
+            assert np.abs(v[idx]).min() >= np.abs(v[dropped]).max()
+
+
+def test_prune_ties_prefer_lower_index():
+    v = np.array([0.5, -2.0, 2.0, 0.5, -0.5, 1.0])
+    # |v| ranking: 2.0 (idx 1), 2.0 (idx 2), 1.0 (idx 5), 0.5 (idx 0), 0.5 (3), 0.5 (4)
+    assert list(F.prune(v, 2)[0]) == [1, 2]
+    assert list(F.prune(v, 4)[0]) == [0, 1, 2, 5]
+    assert list(F.prune(v, 5)[0]) == [0, 1, 2, 3, 5]
+
+
+def test_prune_rejects_bad_nz():
+    with pytest.raises(ValueError):
+        F.prune(np.ones(4), 0)
+    with pytest.raises(ValueError):
+        F.prune(np.ones(4), 5)
+
+
+def test_nz_from_keep_values():
+    # NZ = max(1, floor(keep*C + 1/2)) for the five workloads' (keep, C)
+    assert nz_from_keep(0.5, 128) == 64
+    assert nz_from_keep(0.25, 1536) == 384
+    assert nz_from_keep(0.5, 1536) == 768
+    assert nz_from_keep(0.5, 3072) == 1536
+    assert nz_from_keep(0.1, 3072) == 307
+    assert nz_from_keep(0.3, 6144) == 1843
+    assert nz_from_keep(0.3, 4096) == 1229
+    assert nz_from_keep(1e-9, 100) == 1
+
+
+def test_top_triplet_sign_and_norms():
+    W = draw_weight(6, 11, 5)
+    s, u, v = F.top_triplet(W)
+    assert abs(np.linalg.norm(u) - 1) < 1e-12 and abs(np.linalg.norm(v) - 1) < 1e-12
+    assert np.isclose(s, np.linalg.svd(W, compute_uv=False)[0], rtol=1e-13)
+    assert v[np.argmax(np.abs(v))] > 0
+    assert np.allclose(W.T @ u, s * v, atol=1e-12)   # u^T W = sigma v^T
+    assert np.allclose(W @ v, s * u, atol=1e-12)
+
+
+@pytest.mark.parametrize("H,C", [(8, 16), (64, 128)])
+def test_unpruned_residual_scheme_is_svd_deflation(H, C):
+    W = draw_weight(H, C, 17 + H)
+    f = F.decompose_gate(W, H, C)                   # keep = 1, full rank
+    s_ref = np.linalg.svd(W, compute_uv=False)
+    assert np.allclose(f["sigma"], s_ref, rtol=1e-10, atol=1e-12)
+    assert np.abs(F.reconstruct(f, H, C) - W).max() < 1e-12
+    # each rank-1 term is the LAPACK SVD term of the same index (up to sign)
+    U, _, Vt = np.linalg.svd(W, full_matrices=False)
+    for n in range(0, H, max(1, H // 8)):
+        v_full = np.zeros(C)
+        v_full[f["idx"][n]] = f["val"][n]
+        assert np.allclose(np.outer(f["u"][n], v_full), np.outer(U[:, n], Vt[n]), atol=1e-8)
+
+
+@pytest.mark.parametrize("keep", [0.5, 0.25, 0.1, 0.02])
+def test_frobenius_decrease_law(keep):
+    H, C = 32, 96
+    W = draw_weight(H, C, 23)
+    nz = nz_from_keep(keep, C)
+    K = 40
+    f = F.decompose_gate(W, K, nz, return_residual_norms=True)
+    fro2 = f["resid_fro2"]
+    assert np.isclose(fro2[0], np.sum(W * W), rtol=1e-14)
+    for n in range(K):
+        vn2 = float(np.sum(f["val"][n] ** 2))
+        pred = fro2[n] - f["sigma"][n] ** 2 * vn2
+        assert abs(fro2[n + 1] - pred) <= 1e-10 * fro2[0]
+        assert fro2[n + 1] <= fro2[n] + 1e-12 * fro2[0]
+        assert np.count_nonzero(f["u"][n]) == H       # u is dense: not pruned
+        assert len(f["idx"][n]) == nz
+
+
+def test_masks_are_top_magnitudes_of_residual_triplet():
+    H, C = 16, 40
+    W = draw_weight(H, C, 31)
+    nz = 9
+    f = F.decompose_gate(W, 6, nz)
+    # recompute step n's unpruned v from the residual and check the mask
+    Wt = np.zeros_like(W)
+    for n in range(6):
+        _, _, v = F.top_triplet(W - Wt)
+        assert list(f["idx"][n]) == _brute_prune(v, nz)
+        Wt = F.reconstruct(f, n + 1, C)
+
+
+def test_rank1_keep1_is_top_svd_term():
+    W = draw_weight(12, 30, 3)
+    f = F.decompose_gate(W, 1, 30)
+    U, s, Vt = np.linalg.svd(W, full_matrices=False)
+    assert np.allclose(F.reconstruct(f, 1, 30), s[0] * np.outer(U[:, 0], Vt[0]), atol=1e-13)
