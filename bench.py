@@ -1,0 +1,375 @@
+#!/usr/bin/env python3
+"""Benchmark of progressive approximate-LSTM inference on GB300.
+
+Workload (batch-1 latency workload): one LSTM layer, D=1024 (ReLU-distributed
+CNN-feature-like inputs), H=512, T=20 timesteps, one stream per GPU, fp32
+factors, keep 25% of each v (NZ=384 of C=1536), refinement depth K=256 with
+intermediate outputs at depths 16 and 64 emitted in the same run.  One step
+is one call of the library over the whole sequence: the hoisted input
+projection, the persistent recurrence kernel (coefficients, sums over u,
+cell update, intermediate outputs) -- every step of the path.
+
+Metric: timesteps*streams per second (whole job over all GPUs) and the p50
+per-timestep latency; a sweep over K = 16, 64, 256 is reported beside it.
+Factor sets and inputs are seeded synthetic draws with the structure of the
+method's factors (the timed cost does not depend on the values).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank drives its own GPU with its own stream (weak
+scaling, no data-path collective); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+if HERE not in sys.path:
+    sys.path.insert(0, HERE)
+
+from workloads import WORKLOADS, nz_from_keep, synthetic_layer_factors, workload_inputs  # noqa: E402
+
+METRIC = "approx-LSTM timesteps·streams/sec vs rank K; p50 per-step latency at batch 1"
+UNIT = "timesteps*streams/s"
+WL = WORKLOADS["c2"]
+KEEP = 0.25
+K_MAIN = 256
+CKPTS = (16, 64)
+K_SWEEP = (16, 64, 256)
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _config(n_gpus: int) -> dict:
+    C = WL.C()
+    return {
+        "workload": (f"{WL.name}: 1-layer LSTM D={WL.D} H={WL.H} T={WL.T}, {WL.B} stream per GPU, fp32 factors, "
+                     f"keep {KEEP} -> NZ={nz_from_keep(KEEP, C)} of C={C}, K={K_MAIN}, "
+                     f"intermediate outputs at K={','.join(map(str, CKPTS))}"),
+        "streams_per_gpu": WL.B, "timesteps": WL.T, "K": K_MAIN, "checkpoints": list(CKPTS),
+        "l2": "flushed between timed steps (256 MiB device write outside the step's events)",
+        "parallelism": f"replicas x{n_gpus} (independent streams, no collective)",
+    }
+
+
+def _dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# --------------------------------------------------------------------------
+# host-side helpers (also used by the CPU tests)
+# --------------------------------------------------------------------------
+
+def algorithmic_bytes_per_timestep(H: int, C: int, nz: int, K: int, s: int = 4) -> int:
+    """Factor bytes one timestep of one stream must read: 4 gates x K terms x
+    (NZ values + a 1-bit column mask + u + sigma)."""
+    return 4 * K * (nz * s + (C + 7) // 8 + H * s + s)
+
+
+def recurrence_bytes_per_timestep(H: int, nz_h: float, K: int, s: int = 4) -> float:
+    """Factor bytes of the recurrent part alone (h columns of v, mask, u, sigma)."""
+    return 4 * K * (nz_h * s + (H + 7) // 8 + H * s + s)
+
+
+def aggregate(values_ms, world_size: int, units_per_rank: int):
+    """Whole-job throughput from per-rank step times: units of all ranks over the slowest rank."""
+    t = max(values_ms)
+    return units_per_rank * world_size / (t / 1e3), t
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"bench_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200", "-i", str(self.gpu)], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return None
+        sm, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# reference arm: the fp64 oracle on the host cores
+# --------------------------------------------------------------------------
+
+def _oracle_sample(reps_budget_s: float, K: int, checkpoints=CKPTS):
+    """Time the oracle (as it stands) on the benchmark workload; returns (s per run, runs)."""
+    import oracle
+    layers = [synthetic_layer_factors(WL, 0, K, KEEP)]
+    x = workload_inputs(WL).astype(np.float32).astype(np.float64)
+    runs, t0 = 0, time.perf_counter()
+    while True:
+        oracle.run_lstm(layers, x, K, checkpoints=checkpoints)
+        runs += 1
+        el = time.perf_counter() - t0
+        if el >= reps_budget_s:
+            return el / runs, runs
+
+
+def cpu_baseline(budget_s: float = 12.0) -> dict:
+    """Oracle throughput on the host, single-threaded, in a child process."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = (f"import sys; sys.path.insert(0, {HERE!r}); import bench; "
+            f"s, n = bench._oracle_sample({budget_s}, {K_MAIN}); print(s, n)")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": "failed: " + r.stderr[-200:]}
+    s_per_run, runs = map(float, r.stdout.split())
+    return {"value": WL.T * WL.B / s_per_run, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": (f"{int(runs)} full runs of the benchmark workload (T={WL.T}, B={WL.B}, K={K_MAIN}, "
+                       f"checkpoints {list(CKPTS)}) in {s_per_run * runs:.1f} s, fp64 NumPy, 1 thread")}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist_env()
+    if rank != 0:
+        return
+    import oracle
+    layers = [synthetic_layer_factors(WL, 0, K_MAIN, KEEP)]
+    x = workload_inputs(WL).astype(np.float32).astype(np.float64)
+    for _ in range(args.warmup):
+        oracle.run_lstm(layers, x, K_MAIN, checkpoints=CKPTS)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.run_lstm(layers, x, K_MAIN, checkpoints=CKPTS)
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * sum(times) / len(times)
+    value = WL.T * WL.B / (ms / 1e3)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": _config(1),
+        "p50_us_per_timestep": 1e3 * statistics.median(times) / WL.T * 1e3,
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{args.steps} full runs of the benchmark workload, fp64 NumPy, one thread"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, OPT_TIMING, Q_CLUSTER, Q_LAST_PATH, Q_LAUNCHES
+
+    ws, rank, local = _dist_env()
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist_mod
+        dist = dist_mod
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if ws > 1 else 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+
+    H, D, T, B = WL.H, WL.D, WL.T, WL.B
+    C = WL.C()
+    nz = nz_from_keep(KEEP, C)
+    factors = synthetic_layer_factors(WL, 0, K_MAIN, KEEP)
+    nz_h = float(np.mean([np.count_nonzero(f["idx"] >= D) / f["idx"].shape[0] for f in factors]))
+    m = LSTMApprox(1, [D], H, K_MAIN, B, "fp32", stream=stream)
+    m.set_layer(0, factors)
+    x_host = workload_inputs(WL).astype(np.float32)
+    x = torch.from_numpy(x_host).to(dev)
+    out_h = torch.empty((T, B, H), device=dev)
+    out_c = torch.empty((1, B, H), device=dev)
+    ck_h = torch.empty((len(CKPTS), T, B, H), device=dev)
+    ck_c = torch.empty((len(CKPTS), T, B, H), device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def step(K=K_MAIN, cps=CKPTS):
+        m.run(x, K, out_h, out_c=out_c, checkpoints=list(cps), ckpt_h=ck_h if cps else None,
+              ckpt_c=ck_c if cps else None)
+
+    def timed_loop(nsteps, fn):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nsteps)]
+        for i in range(nsteps):
+            flush.fill_(float(i))
+            evs[i][0].record(stream)
+            fn()
+            evs[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        return [a.elapsed_time(b) for a, b in evs]
+
+    for _ in range(args.warmup):
+        step()
+    m.sync()
+
+    # ---- main timed region -------------------------------------------------
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    launches0 = m.query(Q_LAUNCHES)
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        step_ms = timed_loop(args.steps, step)
+    m.sync()
+    launches = m.query(Q_LAUNCHES) - launches0
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    ms_mean = sum(step_ms) / len(step_ms)
+    p50_ms = statistics.median(step_ms)
+    path = m.query(Q_LAST_PATH)
+    cluster = m.query(Q_CLUSTER)
+
+    # ---- per-phase device times (CUDA events on the library's stream) ------
+    m.set_option(OPT_TIMING, 1)
+    ph = []
+    for i in range(max(10, min(args.steps, 50))):
+        flush.fill_(float(i))
+        step()
+        ph.append(m.phase_times())
+    m.set_option(OPT_TIMING, 0)
+    xproj_ms = statistics.mean(p[0] for p in ph)
+    rec_ms = statistics.mean(p[1] for p in ph)
+
+    # ---- K sweep (separate runs, no intermediate outputs) ------------------
+    sweep = []
+    for K in K_SWEEP:
+        for _ in range(3):
+            step(K, ())
+        t = timed_loop(max(10, min(args.steps, 50)), lambda K=K: step(K, ()))
+        med = statistics.median(t)
+        sweep.append({"K": K, "value": T * B / (statistics.mean(t) / 1e3), "unit": UNIT,
+                      "p50_us_per_timestep": 1e3 * med / T,
+                      "effective_factor_gbs": algorithmic_bytes_per_timestep(H, C, nz, K) * T / (med / 1e3) / 1e9})
+
+    # ---- end to end through the host-buffer entry point ---------------------
+    xh = torch.from_numpy(x_host).pin_memory()
+    oh = torch.empty((T, B, H), dtype=torch.float32).pin_memory()
+    kh = torch.empty((len(CKPTS), T, B, H), dtype=torch.float32).pin_memory()
+    xh_np, oh_np, kh_np = xh.numpy(), oh.numpy(), kh.numpy()
+    for _ in range(3):
+        m.run_host(xh_np, K_MAIN, oh_np, checkpoints=list(CKPTS), ckpt_h=kh_np)
+    e2e_t = []
+    for i in range(args.steps):
+        flush.fill_(float(i))
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        m.run_host(xh_np, K_MAIN, oh_np, checkpoints=list(CKPTS), ckpt_h=kh_np)
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_ms = 1e3 * sum(e2e_t) / len(e2e_t)
+
+    # ---- aggregate over ranks ----------------------------------------------
+    vals = torch.tensor([ms_mean, e2e_ms], dtype=torch.float64, device=dev)
+    if dist:
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+    ms_max, e2e_max = float(vals[0]), float(vals[1])
+    value = T * B * ws / (ms_max / 1e3)
+    e2e_value = T * B * ws / (e2e_max / 1e3)
+
+    if rank == 0:
+        peaks = {}
+        try:
+            peaks = json.load(open(os.path.join(HERE, "MEASURED_PEAKS.json")))
+        except (OSError, ValueError):
+            pass
+        hbm_peak = peaks.get("hbm_gbs")
+        peak_note = "measured (MEASURED_PEAKS.json hbm_gbs)" if hbm_peak else "fallback 6800 GB/s"
+        hbm_peak = hbm_peak or 6800.0
+        rec_bytes = recurrence_bytes_per_timestep(H, nz_h, K_MAIN) * T
+        achieved = rec_bytes / (rec_ms / 1e3) / 1e9
+        path_bytes = algorithmic_bytes_per_timestep(H, C, nz, K_MAIN) * T
+        clocks = clk.summary()
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": _config(ws),
+            "p50_us_per_timestep": 1e3 * p50_ms / T,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(x_host.nbytes),
+                    "d2h_bytes_per_step": int(oh.numel() * 4 + kh.numel() * 4)},
+            "roofline": {"kernel": "persistent recurrence kernel", "bound": "hbm", "achieved": achieved,
+                         "peak": hbm_peak, "peak_source": peak_note, "unit": "GB/s", "frac": achieved / hbm_peak,
+                         "traffic": None,
+                         "algorithmic_bytes_per_launch": rec_bytes, "launch_ms": rec_ms},
+            "path_effective_gbs": path_bytes / (ms_max / 1e3) / 1e9,
+            "phase_ms": {"input_projection": xproj_ms, "recurrence": rec_ms},
+            "recurrence_path": {1: "simt", 2: "persistent", 3: "tensor"}.get(path, str(path)),
+            "cluster_ctas": cluster,
+            "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
+        }
+        if ws == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

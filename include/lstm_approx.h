@@ -1,0 +1,197 @@
+/*
+ * lstm_approx.h -- progressive approximate-LSTM inference on sm_103a (GB300).
+ *
+ * The method (arXiv 1905.00689, Sec. III, Eq. 1): each LSTM gate's augmented
+ * matrix W = [Wx Wh] (R x C, R = hidden size H, C = D + H) is replaced by a
+ * sum of K pruned rank-1 terms sigma^(n) u^(n) prune(v^(n), NZ)^T taken from
+ * the residual of the previous terms.  One timestep of one stream computes,
+ * per gate g and with x~ = [x_t ; h_{t-1}] (Sec. III):
+ *
+ *     t_g[n] = prune(v_g^(n))^T x~                    (dot products, 2 NZ ops)
+ *     y_g    = sum_{n<=K} sigma_g^(n) u_g^(n) t_g[n]    (2R + 1 ops per n)
+ *
+ * followed by the gate nonlinearities and the cell update of Sec. II
+ * (i, f, o: logistic sigmoid; cell gate: tanh; c_t = f c_{t-1} + i g;
+ * h_t = o tanh(c_t)).  Prefix sums over n <= k_j give the intermediate
+ * ("progressive", Sec. I and Fig. 1b) outputs for a refinement depth k_j.
+ *
+ * Gate order everywhere in this interface: 0 = input (i), 1 = forget (f),
+ * 2 = cell candidate (g), 3 = output (o).
+ *
+ * Conventions for every entry point:
+ *   - returns an lstm_approx_status; nothing aborts, throws or prints;
+ *   - arguments are checked before anything is launched; a call that
+ *     returns LSTM_APPROX_EINVAL or LSTM_APPROX_ESTATE changes no state;
+ *   - the text of the last error of a handle is lstm_approx_last_error();
+ *   - there is no CPU fallback: without a usable sm_103a device every call
+ *     that needs one returns LSTM_APPROX_ECUDA.
+ */
+#ifndef LSTM_APPROX_H
+#define LSTM_APPROX_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct lstm_approx lstm_approx_t; /* opaque; owned by the library */
+
+enum lstm_approx_status {
+  LSTM_APPROX_OK = 0,
+  LSTM_APPROX_EINVAL = 1,   /* invalid argument (size, pointer, range) */
+  LSTM_APPROX_ENOMEM = 2,   /* device or host allocation failed */
+  LSTM_APPROX_ECUDA = 3,    /* CUDA error, or no usable sm_103a device */
+  LSTM_APPROX_ETIMEOUT = 4, /* a bounded in-kernel wait ran out */
+  LSTM_APPROX_ESTATE = 5    /* factors not set, or K above the depth set */
+};
+
+/* Storage/operand type of the factors u, v.  sigma, bias, the state and all
+ * accumulation are fp32 in both.  BF16 is the tensor-core path. */
+enum lstm_approx_dtype { LSTM_APPROX_FP32 = 0, LSTM_APPROX_BF16 = 1 };
+
+/*
+ * Create a handle for an L-layer stack (layer l >= 1 consumes layer l-1's
+ * h_t as its input, so input_dims[l] must equal `hidden` for l >= 1).
+ *
+ *   out         receives the handle (set to NULL on failure)
+ *   num_layers  L >= 1
+ *   input_dims  host array [L]; input_dims[0] = D >= 1
+ *   hidden      H = R >= 1 (Sec. III: W is R x C, C = D + H)
+ *   max_rank    largest refinement depth K (N_steps, Sec. III) ever set
+ *   max_batch   largest number of independent streams B passed to run
+ *   dtype       enum lstm_approx_dtype
+ *   cuda_stream cudaStream_t every launch and copy of this handle goes to;
+ *               NULL = the legacy default stream.  Not owned.
+ *
+ * Allocates the device factor storage and per-stream state.  Errors:
+ * EINVAL (sizes), ECUDA (no sm_103a device), ENOMEM.
+ */
+int lstm_approx_create(lstm_approx_t **out, int num_layers, const int *input_dims, int hidden,
+                       int max_rank, int max_batch, int dtype, void *cuda_stream);
+
+/*
+ * Set the first K refinement terms of one gate (Eq. 1): for n < K,
+ * sigma[n] u[n][:] prune(v[n])^T, where prune(v[n]) has the nz entries
+ * v_val[n][m] at columns v_idx[n][m] of the augmented input x~ = [x; h]
+ * (columns 0..D-1 multiply x_t, columns D..D+H-1 multiply h_{t-1}).
+ *
+ *   layer, gate  0 <= layer < L, 0 <= gate < 4 (i, f, g, o)
+ *   K            1 <= K <= max_rank; later runs may use any depth <= K
+ *   nz           1 <= nz <= C (the paper's NZ; may differ between gates)
+ *   sigma        host [K] (fp64)
+ *   u            host [K][H] row-major (fp64); u is not pruned
+ *   v_idx        host [K][nz]; each row strictly increasing, in [0, C)
+ *   v_val        host [K][nz] (fp64)
+ *   bias         host [H] added to the gate pre-activation, or NULL = 0
+ *                (the paper writes no bias; it is exact, not approximated)
+ *
+ * The library copies the arrays (the caller keeps ownership), rounds sigma
+ * and bias to fp32 and u, v to the handle's dtype (fp64 -> fp32 -> bf16,
+ * each round-to-nearest-even), packs them and uploads them with one
+ * synchronous copy.  Errors: EINVAL (ranges, unsorted or out-of-range
+ * indices), ECUDA.
+ */
+int lstm_approx_set_factors(lstm_approx_t *h, int layer, int gate, int K, int nz, const double *sigma,
+                            const double *u, const int32_t *v_idx, const double *v_val,
+                            const double *bias);
+
+/*
+ * Run the stack over a sequence: T timesteps of B independent streams at
+ * refinement depth K, asynchronously on the handle's stream.
+ *
+ * All tensors are caller-owned DEVICE pointers, fp32, row-major:
+ *   x        [T][B][D]          input sequence of layer 0
+ *   h0, c0   [L][B][H] or NULL  initial state (NULL = zeros)
+ *   out_h    [T][B][H]          top layer's h_t at depth K
+ *   out_c    [L][B][H] or NULL  each layer's final c_T (for resuming)
+ *   checkpoints host [J], strictly increasing, each in [1, K], J <= 8
+ *            (may be NULL when J = 0)
+ *   ckpt_h, ckpt_c [J][T][B][H] or NULL: the top layer's h_t, c_t when its
+ *            refinement sums stop at depth k_j.  h_{t-1} and c_{t-1} always
+ *            come from the full-depth chain, so one run yields every depth
+ *            without recomputing shared prefixes (computation cut short as
+ *            the time budget is hit, Sec. VI-B.1).
+ *
+ * 1 <= T, 1 <= B <= max_batch, 1 <= K <= the depth set for every gate.
+ * Errors: EINVAL, ESTATE (a gate's factors missing or shallower than K),
+ * ENOMEM (growing the T-dependent scratch), ECUDA (launch failure).
+ * Kernel-side failures (a bounded wait that ran out) are reported by the
+ * next lstm_approx_sync().  The first run at a new largest T*B may allocate
+ * scratch (synchronising the stream).
+ */
+int lstm_approx_run(lstm_approx_t *h, const float *x, int T, int B, int K, const float *h0,
+                    const float *c0, float *out_h, float *out_c, const int *checkpoints, int J,
+                    float *ckpt_h, float *ckpt_c);
+
+/*
+ * lstm_approx_run with every tensor a HOST pointer (same shapes and
+ * meaning).  Copies the inputs to device staging buffers owned by the
+ * handle, runs, copies the outputs back and waits for the stream.  Host
+ * buffers in page-locked memory copy fastest.  Returns what
+ * lstm_approx_run or lstm_approx_sync would.
+ */
+int lstm_approx_run_host(lstm_approx_t *h, const float *x, int T, int B, int K, const float *h0,
+                         const float *c0, float *out_h, float *out_c, const int *checkpoints, int J,
+                         float *ckpt_h, float *ckpt_c);
+
+/*
+ * Wait for the handle's stream and report kernel-side status: OK, or
+ * ETIMEOUT when a bounded in-kernel wait ran out since the last sync (the
+ * outputs of that run are then invalid; the status word is cleared), or
+ * ECUDA.
+ */
+int lstm_approx_sync(lstm_approx_t *h);
+
+/*
+ * Read back the pruning mask of term k (0 <= k < K set) of (layer, gate)
+ * from the device-resident packed representation.  idx_out: host [C]
+ * (capacity C = D_layer + H); *nz_out receives the count.  The indices are
+ * ascending and must equal the v_idx row passed to set_factors bit for bit.
+ */
+int lstm_approx_get_mask(lstm_approx_t *h, int layer, int gate, int k, int32_t *idx_out, int *nz_out);
+
+/* Text of the handle's last error ("" if none).  Static text for NULL. */
+const char *lstm_approx_last_error(const lstm_approx_t *h);
+
+/* Free the handle and everything it owns (waits for its stream).  NULL-safe. */
+void lstm_approx_destroy(lstm_approx_t *h);
+
+/* ---- introspection and tuning (tests, benchmarks) ---------------------- */
+
+enum lstm_approx_query_key {
+  LSTM_APPROX_Q_LAUNCHES = 0,    /* kernels launched by this handle so far */
+  LSTM_APPROX_Q_LAST_PATH = 1,   /* recurrence path of the last run (enum below) */
+  LSTM_APPROX_Q_CLUSTER = 2,     /* CTAs per cluster of the last persistent run */
+  LSTM_APPROX_Q_DEVICE_BYTES = 3 /* device bytes currently held by the handle */
+};
+enum lstm_approx_path {
+  LSTM_APPROX_PATH_NONE = 0,
+  LSTM_APPROX_PATH_SIMT = 1,       /* per-timestep CUDA-core kernels */
+  LSTM_APPROX_PATH_PERSISTENT = 2, /* one persistent cluster launch over all T (fp32) */
+  LSTM_APPROX_PATH_TENSOR = 3      /* tcgen05/TMEM GEMMs with fused epilogues (bf16) */
+};
+int lstm_approx_query(const lstm_approx_t *h, int key, long long *value);
+
+enum lstm_approx_option_key {
+  LSTM_APPROX_OPT_FORCE_PATH = 0,   /* 0 = automatic, else an lstm_approx_path */
+  LSTM_APPROX_OPT_CLUSTER = 1,      /* 0 = automatic, else 1, 2, 4, 8 or 16 */
+  LSTM_APPROX_OPT_TIMING = 2,       /* 1 = record CUDA events around each phase */
+  LSTM_APPROX_OPT_WAIT_LIMIT = 3,   /* bounded-wait limit in polls (default 2^26) */
+  LSTM_APPROX_OPT_TEST_STALL = 4    /* 1 = next persistent run waits on a signal
+                                       nobody sends (exercises ETIMEOUT) */
+};
+int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
+
+/*
+ * Device milliseconds of the last run's phases, from CUDA events recorded
+ * on the handle's stream when LSTM_APPROX_OPT_TIMING is 1 (waits for the
+ * stream).  ms_out[0] = input projection (hoisted over all T), ms_out[1] =
+ * recurrence (all layers, all T), ms_out[2] = whole run.
+ */
+int lstm_approx_phase_times(lstm_approx_t *h, float *ms_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LSTM_APPROX_H */

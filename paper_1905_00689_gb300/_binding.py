@@ -1,0 +1,188 @@
+"""ctypes binding of liblstm_approx.so (argument marshalling only).
+
+Every entry point of include/lstm_approx.h is exposed under its own name;
+:class:`LSTMApprox` wraps a handle for callers holding torch tensors (device
+memory and the current stream come from PyTorch; every step of the
+recurrence runs in the library's kernels).  There is no fallback: if the
+library is missing or cannot run, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "liblstm_approx.so")
+
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, ESTATE = range(6)
+FP32, BF16 = 0, 1
+Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES = range(4)
+PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
+OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL = range(5)
+STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ETIMEOUT: "ETIMEOUT",
+                ESTATE: "ESTATE"}
+
+EXPORTS = (
+    "lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_run_host",
+    "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
+    "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times",
+)
+
+_lib = None
+
+
+class LSTMApproxError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {message}")
+        self.code = code
+
+
+def load(path: str = LIB_PATH):
+    """Load the library (once).  Raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build() "
+                           "or python -m paper_1905_00689_gb300.build")
+    lib = ctypes.CDLL(path)
+    P, I, LL = ctypes.c_void_p, ctypes.c_int, ctypes.c_longlong
+    lib.lstm_approx_create.argtypes = [ctypes.POINTER(P), I, ctypes.POINTER(I), I, I, I, I, P]
+    lib.lstm_approx_set_factors.argtypes = [P, I, I, I, I, P, P, P, P, P]
+    run_args = [P, P, I, I, I, P, P, P, P, P, I, P, P]
+    lib.lstm_approx_run.argtypes = run_args
+    lib.lstm_approx_run_host.argtypes = run_args
+    lib.lstm_approx_sync.argtypes = [P]
+    lib.lstm_approx_get_mask.argtypes = [P, I, I, I, P, ctypes.POINTER(I)]
+    lib.lstm_approx_last_error.argtypes = [P]
+    lib.lstm_approx_last_error.restype = ctypes.c_char_p
+    lib.lstm_approx_destroy.argtypes = [P]
+    lib.lstm_approx_destroy.restype = None
+    lib.lstm_approx_query.argtypes = [P, I, ctypes.POINTER(LL)]
+    lib.lstm_approx_set_option.argtypes = [P, I, LL]
+    lib.lstm_approx_phase_times.argtypes = [P, ctypes.POINTER(ctypes.c_float)]
+    for name in EXPORTS:
+        if name not in ("lstm_approx_last_error", "lstm_approx_destroy"):
+            getattr(lib, name).restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def _ptr(t) -> Optional[int]:
+    """Device address of a torch tensor (None passes NULL)."""
+    if t is None:
+        return None
+    if not t.is_contiguous() or t.dtype.itemsize != 4:
+        raise ValueError("tensors must be contiguous fp32")
+    return t.data_ptr()
+
+
+def _np_ptr(a) -> Optional[int]:
+    if a is None:
+        return None
+    return a.ctypes.data
+
+
+class LSTMApprox:
+    """One handle of the library.
+
+    `stream` is a torch.cuda.Stream (default: torch's current stream on the
+    current device); tensors passed to :meth:`run` must live on that device.
+    """
+
+    def __init__(self, num_layers: int, input_dims: Sequence[int], hidden: int, max_rank: int,
+                 max_batch: int, dtype: str = "fp32", stream=None):
+        import torch
+        self.lib = load()
+        self.L, self.H = num_layers, hidden
+        self.input_dims = list(input_dims)
+        self.dtype = dtype
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        self.stream = stream
+        dims = (ctypes.c_int * num_layers)(*self.input_dims)
+        h = ctypes.c_void_p()
+        rc = self.lib.lstm_approx_create(ctypes.byref(h), num_layers, dims, hidden, max_rank, max_batch,
+                                         BF16 if dtype == "bf16" else FP32,
+                                         ctypes.c_void_p(stream.cuda_stream))
+        if rc != OK:
+            raise LSTMApproxError(rc, "lstm_approx_create failed")
+        self.h = h
+
+    # -- helpers ---------------------------------------------------------
+    def _check(self, rc: int):
+        if rc != OK:
+            msg = self.lib.lstm_approx_last_error(self.h).decode()
+            raise LSTMApproxError(rc, msg)
+
+    def close(self):
+        if getattr(self, "h", None):
+            self.lib.lstm_approx_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # -- entry points ----------------------------------------------------
+    def set_factors(self, layer: int, gate: int, sigma, u, idx, val, bias=None):
+        sigma = np.ascontiguousarray(sigma, dtype=np.float64)
+        u = np.ascontiguousarray(u, dtype=np.float64)
+        idx = np.ascontiguousarray(idx, dtype=np.int32)
+        val = np.ascontiguousarray(val, dtype=np.float64)
+        K, nz = idx.shape
+        b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float64)
+        self._check(self.lib.lstm_approx_set_factors(self.h, layer, gate, K, nz, _np_ptr(sigma), _np_ptr(u),
+                                                     _np_ptr(idx), _np_ptr(val), _np_ptr(b)))
+
+    def set_layer(self, layer: int, gates):
+        """gates: four dicts with sigma, u, idx, val (and optional bias)."""
+        for g, f in enumerate(gates):
+            self.set_factors(layer, g, f["sigma"], f["u"], f["idx"], f["val"], f.get("bias"))
+
+    def run(self, x, K: int, out_h, h0=None, c0=None, out_c=None, checkpoints=(), ckpt_h=None, ckpt_c=None):
+        """Device run; x [T][B][D] fp32 CUDA tensor, out_h [T][B][H]."""
+        T, B = x.shape[0], x.shape[1]
+        cps = (ctypes.c_int * max(1, len(checkpoints)))(*checkpoints)
+        self._check(self.lib.lstm_approx_run(self.h, _ptr(x), T, B, K, _ptr(h0), _ptr(c0), _ptr(out_h),
+                                             _ptr(out_c), cps, len(checkpoints), _ptr(ckpt_h), _ptr(ckpt_c)))
+
+    def run_host(self, x: np.ndarray, K: int, out_h: np.ndarray, h0=None, c0=None, out_c=None,
+                 checkpoints=(), ckpt_h=None, ckpt_c=None):
+        """Host-buffer run (float32 numpy arrays, C order); synchronous."""
+        for a in (x, out_h, h0, c0, out_c, ckpt_h, ckpt_c):
+            if a is not None and (a.dtype != np.float32 or not a.flags["C_CONTIGUOUS"]):
+                raise ValueError("host buffers must be C-contiguous float32")
+        T, B = x.shape[0], x.shape[1]
+        cps = (ctypes.c_int * max(1, len(checkpoints)))(*checkpoints)
+        self._check(self.lib.lstm_approx_run_host(self.h, _np_ptr(x), T, B, K, _np_ptr(h0), _np_ptr(c0),
+                                                  _np_ptr(out_h), _np_ptr(out_c), cps, len(checkpoints),
+                                                  _np_ptr(ckpt_h), _np_ptr(ckpt_c)))
+
+    def sync(self):
+        self._check(self.lib.lstm_approx_sync(self.h))
+
+    def get_mask(self, layer: int, gate: int, k: int) -> np.ndarray:
+        C = self.input_dims[layer] + self.H
+        out = np.zeros(C, dtype=np.int32)
+        n = ctypes.c_int(0)
+        self._check(self.lib.lstm_approx_get_mask(self.h, layer, gate, k, _np_ptr(out), ctypes.byref(n)))
+        return out[: n.value].copy()
+
+    def query(self, key: int) -> int:
+        v = ctypes.c_longlong(0)
+        self._check(self.lib.lstm_approx_query(self.h, key, ctypes.byref(v)))
+        return v.value
+
+    def set_option(self, key: int, value: int):
+        self._check(self.lib.lstm_approx_set_option(self.h, key, value))
+
+    def phase_times(self):
+        ms = (ctypes.c_float * 3)()
+        self._check(self.lib.lstm_approx_phase_times(self.h, ms))
+        return list(ms)

@@ -1,0 +1,155 @@
+// Internal declarations shared by the C-ABI implementation and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "../../include/lstm_approx.h"
+
+namespace lstm_approx_impl {
+
+constexpr int kMaxCheckpoints = 8;
+
+struct Checkpoints {
+  int n;
+  int k[kMaxCheckpoints];
+};
+
+// Device factor storage of one layer.  Row (g, k) of the packed matrices is
+// storage row g * Ks + k ("gate-major"), rows k >= K_set are zero.
+//   Vx   [4*Ks][ldx]  masked-dense pruned v over the x columns (ldx >= D)
+//   Vh   [4*Ks][ldh]  masked-dense pruned v over the h columns (ldh >= H)
+//   U    fp32: [4][Ks][H] (u_k[j] at (g*Ks + k)*H + j)
+//        bf16: [4][H][Ks] (u_k[j] at (g*H + j)*Ks + k, K-major for the MMA)
+//   sigma [4][Ks] fp32, bias [4][H] fp32
+//   mask [4*Ks][mask_words] bit c set <=> column c of x~ is kept
+struct LayerStore {
+  int D = 0, C = 0, ldx = 0;
+  void* Vx = nullptr;
+  void* Vh = nullptr;
+  void* U = nullptr;
+  float* sigma = nullptr;
+  float* bias = nullptr;
+  uint32_t* mask = nullptr;
+  int mask_words = 0;
+  int Kset[4] = {0, 0, 0, 0};
+  int nz[4] = {0, 0, 0, 0};
+};
+
+struct Timing {
+  bool on = false;
+  std::vector<cudaEvent_t> ev;  // pairs (start, stop) per phase launch
+  std::vector<int> phase;       // 0 = input projection, 1 = recurrence
+  cudaEvent_t run0 = nullptr, run1 = nullptr;
+};
+
+}  // namespace lstm_approx_impl
+
+struct lstm_approx {
+  int L = 0, H = 0, ldh = 0, Kmax = 0, Ks = 0, max_batch = 0, dtype = 0;
+  cudaStream_t stream = nullptr;
+  int device = 0, sm_count = 0;
+  std::vector<lstm_approx_impl::LayerStore> layers;
+
+  // state and scratch
+  float* h_state = nullptr;   // [L][max_batch][H]
+  float* c_state = nullptr;   // [L][max_batch][H]
+  size_t cap_TB = 0;          // capacity (T*B) of the T-dependent scratch
+  float* Px = nullptr;        // [T*B][4*Ks] hoisted input projection
+  float* seq = nullptr;       // [T*B][H] output sequence of a lower layer
+  void* tau = nullptr;        // [max_batch][4*Ks] refinement coefficients
+  int* err = nullptr;         // device status word (0 = ok)
+
+  // staging for lstm_approx_run_host
+  size_t stage_bytes = 0;
+  char* stage = nullptr;
+
+  // options and counters
+  int opt_force_path = 0, opt_cluster = 0;
+  long long opt_wait_limit_us = 2000000;
+  int opt_test_stall = 0;
+  long long launches = 0;
+  int last_path = 0, last_cluster = 0;
+  long long device_bytes = 0;
+  lstm_approx_impl::Timing timing;
+  std::string last_error;
+};
+
+namespace lstm_approx_impl {
+
+// ---- generic CUDA-core kernels (any size, both factor types) -------------
+
+// out[n][srow(r)] = sum_c A[srow(r)][c] * Bm[n][c] for run rows r < 4K, where
+// srow(r) = (r / K) * Ks + r % K.  mode 0 stores the sum; mode 1 stores
+// sigma[srow] * (sum + P[n][srow]).
+cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks, const float* Bm, int ldb,
+                             int N, int Kdim, float* out, int ldo, int mode, const float* sigma,
+                             const float* P, int ldp, cudaStream_t s);
+
+// One timestep of the refinement sums over u (a3), the intermediate outputs
+// (a6) and the cell update (a4) for B streams.
+struct CellArgs {
+  const void* U;
+  bool u_bf16;
+  long long gs, ks, js;  // element strides of U over (gate, k, unit)
+  int K, Ks, H, B;
+  const float* tau;      // [B][ldt], coefficient of (g, k) at g*Ks + k
+  int ldt;
+  const float* bias;     // [4][H]
+  float* c_state;        // [B][H], read then overwritten
+  float* h_state;        // [B][H], overwritten
+  float* out_h;          // [B][H] or null
+  Checkpoints ck;
+  float* ckpt_h;         // element (j, b, unit) at j*ck_stride + b*H + unit, or null
+  float* ckpt_c;
+  long long ck_stride;
+};
+cudaError_t launch_cell_step(const CellArgs& a, cudaStream_t s);
+
+// ---- persistent cluster kernel (fp32 factors, small batch) ---------------
+
+struct PersistentPlan {
+  int CS = 0;        // CTAs per cluster
+  int RA = 0;        // coefficient rows per CTA (multiple of 4)
+  int UB = 0;        // hidden units per CTA (multiple of 4)
+  int upl = 0;       // units per lane (1 or 2)
+  int kpw = 0;       // refinement terms per warp segment
+  int nseg = 0;      // segments (<= warps)
+  int seg_start[17] = {0};
+  int ck_seg[kMaxCheckpoints] = {0};
+  size_t smem = 0;
+  int pxc = 0;       // timesteps of P staged in shared memory at once
+};
+
+// Chooses a plan; returns false (with a reason) if the shape does not fit.
+bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, int sm_count,
+                     PersistentPlan* plan, std::string* why);
+
+struct PersistentArgs {
+  const float* Vh;     // [4*Ks][ldh]
+  const float* U;      // [4][Ks][H]
+  const float* sigma;  // [4][Ks]
+  const float* bias;   // [4][H]
+  const float* P;      // [T][B][4*Ks]
+  const float* h0;     // [B][H] or null
+  const float* c0;     // [B][H] or null
+  float* out_h;        // [T][B][H]
+  float* c_last;       // [B][H] or null
+  float* ckpt_h;       // [J][T][B][H] or null
+  float* ckpt_c;
+  int* err;
+  int H, K, Ks, ldh, T, B;
+  Checkpoints ck;
+  long long wait_limit_ns;
+  int test_stall;
+};
+cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s);
+
+// ---- error codes written to the device status word -----------------------
+constexpr int kErrWaitTimeoutA = 1;
+constexpr int kErrWaitTimeoutB = 2;
+
+}  // namespace lstm_approx_impl

@@ -1,0 +1,596 @@
+// C-ABI of the approximate-LSTM library: handle, factor packing, dispatch.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+
+using namespace lstm_approx_impl;
+
+namespace {
+
+int fail(lstm_approx_t* h, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (h) h->last_error = buf;
+  return code;
+}
+
+int cuda_fail(lstm_approx_t* h, cudaError_t e, const char* what) {
+  return fail(h, e == cudaErrorMemoryAllocation ? LSTM_APPROX_ENOMEM : LSTM_APPROX_ECUDA, "%s: %s", what,
+              cudaGetErrorString(e));
+}
+
+#define LA_CUDA(h, call, what)                      \
+  do {                                              \
+    cudaError_t e_ = (call);                        \
+    if (e_ != cudaSuccess) return cuda_fail(h, e_, what); \
+  } while (0)
+
+inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
+
+// fp64 -> fp32 -> bf16, both steps round-to-nearest-even.
+inline uint16_t to_bf16_bits(double x) {
+  const float f = static_cast<float>(x);
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7F800000u) == 0x7F800000u) return static_cast<uint16_t>(u >> 16);  // inf / nan
+  const uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7FFFu + lsb;
+  return static_cast<uint16_t>(u >> 16);
+}
+
+size_t elem_size(int dtype) { return dtype == LSTM_APPROX_BF16 ? 2 : 4; }
+
+int dmalloc(lstm_approx_t* h, void** p, size_t bytes, const char* what) {
+  *p = nullptr;
+  if (bytes == 0) return LSTM_APPROX_OK;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    *p = nullptr;
+    return cuda_fail(h, e, what);
+  }
+  e = cudaMemset(*p, 0, bytes);
+  if (e != cudaSuccess) return cuda_fail(h, e, what);
+  h->device_bytes += static_cast<long long>(bytes);
+  return LSTM_APPROX_OK;
+}
+
+void dfree(lstm_approx_t* h, void* p, size_t bytes) {
+  if (p) {
+    cudaFree(p);
+    h->device_bytes -= static_cast<long long>(bytes);
+  }
+}
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+size_t layer_bytes_vx(const lstm_approx_t* h, const LayerStore& s) {
+  return 4ull * h->Ks * s.ldx * elem_size(h->dtype);
+}
+size_t layer_bytes_vh(const lstm_approx_t* h) { return 4ull * h->Ks * h->ldh * elem_size(h->dtype); }
+size_t layer_bytes_u(const lstm_approx_t* h) { return 4ull * h->Ks * h->H * elem_size(h->dtype); }
+
+void free_scratch(lstm_approx_t* h) {
+  dfree(h, h->Px, h->cap_TB * 4ull * h->Ks * sizeof(float));
+  dfree(h, h->seq, h->cap_TB * (size_t)h->H * sizeof(float));
+  h->Px = nullptr;
+  h->seq = nullptr;
+  h->cap_TB = 0;
+}
+
+int ensure_scratch(lstm_approx_t* h, size_t TB) {
+  if (TB <= h->cap_TB) return LSTM_APPROX_OK;
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "synchronising before growing scratch");
+  free_scratch(h);
+  int rc = dmalloc(h, reinterpret_cast<void**>(&h->Px), TB * 4ull * h->Ks * sizeof(float), "scratch P");
+  if (rc) return rc;
+  if (h->L > 1) {
+    rc = dmalloc(h, reinterpret_cast<void**>(&h->seq), TB * (size_t)h->H * sizeof(float), "scratch seq");
+    if (rc) return rc;
+  }
+  h->cap_TB = TB;
+  return LSTM_APPROX_OK;
+}
+
+int validate_run(lstm_approx_t* h, const float* x, int T, int B, int K, float* out_h, const int* checkpoints,
+                 int J, Checkpoints* ck) {
+  if (!x || !out_h) return fail(h, LSTM_APPROX_EINVAL, "x and out_h must not be NULL");
+  if (T < 1) return fail(h, LSTM_APPROX_EINVAL, "T=%d must be >= 1", T);
+  if (B < 1 || B > h->max_batch) return fail(h, LSTM_APPROX_EINVAL, "B=%d outside [1, %d]", B, h->max_batch);
+  if (K < 1 || K > h->Kmax) return fail(h, LSTM_APPROX_EINVAL, "K=%d outside [1, %d]", K, h->Kmax);
+  if (J < 0 || J > kMaxCheckpoints) return fail(h, LSTM_APPROX_EINVAL, "J=%d outside [0, %d]", J, kMaxCheckpoints);
+  if (J > 0 && !checkpoints) return fail(h, LSTM_APPROX_EINVAL, "checkpoints is NULL with J=%d", J);
+  ck->n = J;
+  for (int j = 0; j < J; ++j) {
+    const int k = checkpoints[j];
+    if (k < 1 || k > K) return fail(h, LSTM_APPROX_EINVAL, "checkpoint %d = %d outside [1, K=%d]", j, k, K);
+    if (j > 0 && k <= checkpoints[j - 1])
+      return fail(h, LSTM_APPROX_EINVAL, "checkpoints must be strictly increasing");
+    ck->k[j] = k;
+  }
+  for (int j = J; j < kMaxCheckpoints; ++j) ck->k[j] = 0;
+  for (int l = 0; l < h->L; ++l)
+    for (int g = 0; g < 4; ++g)
+      if (h->layers[l].Kset[g] < K)
+        return fail(h, LSTM_APPROX_ESTATE, "layer %d gate %d has %d terms set, run asks K=%d", l, g,
+                    h->layers[l].Kset[g], K);
+  return LSTM_APPROX_OK;
+}
+
+struct PhaseTimer {
+  lstm_approx_t* h;
+  int phase;
+  cudaEvent_t e1 = nullptr;
+  PhaseTimer(lstm_approx_t* hh, int ph) : h(hh), phase(ph) {
+    if (!h->timing.on) return;
+    cudaEvent_t e0;
+    cudaEventCreate(&e0);
+    cudaEventCreate(&e1);
+    cudaEventRecord(e0, h->stream);
+    h->timing.ev.push_back(e0);
+    h->timing.ev.push_back(e1);
+    h->timing.phase.push_back(phase);
+  }
+  ~PhaseTimer() {
+    if (e1) cudaEventRecord(e1, h->stream);
+  }
+};
+
+void clear_timing(lstm_approx_t* h) {
+  for (cudaEvent_t e : h->timing.ev) cudaEventDestroy(e);
+  h->timing.ev.clear();
+  h->timing.phase.clear();
+}
+
+int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const float* h0, const float* c0,
+               float* out_h, float* out_c, const Checkpoints& ck, float* ckpt_h, float* ckpt_c) {
+  const int H = h->H;
+  const bool bf16 = h->dtype == LSTM_APPROX_BF16;
+  int rc = ensure_scratch(h, static_cast<size_t>(T) * B);
+  if (rc) return rc;
+  if (h->timing.on) {
+    clear_timing(h);
+    if (!h->timing.run0) {
+      cudaEventCreate(&h->timing.run0);
+      cudaEventCreate(&h->timing.run1);
+    }
+    cudaEventRecord(h->timing.run0, h->stream);
+  }
+  const long long ldp = 4LL * h->Ks;
+  for (int l = 0; l < h->L; ++l) {
+    const LayerStore& s = h->layers[l];
+    const bool top = l == h->L - 1;
+    const float* in = l == 0 ? x : h->seq;
+    float* out = top ? out_h : h->seq;
+    const Checkpoints none = {0, {0}};
+    const Checkpoints& lck = top ? ck : none;
+    // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
+    {
+      PhaseTimer pt(h, 0);
+      LA_CUDA(h,
+              launch_rows_gemm(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, 0, nullptr,
+                               nullptr, 0, h->stream),
+              "input projection launch");
+      h->launches += 1;
+    }
+    const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
+    const float* l_c0 = c0 ? c0 + (size_t)l * B * H : nullptr;
+    float* l_cout = out_c ? out_c + (size_t)l * B * H : nullptr;
+
+    // recurrence path
+    int path = h->opt_force_path;
+    PersistentPlan plan;
+    std::string why;
+    if (path == 0) {
+      path = LSTM_APPROX_PATH_SIMT;
+      if (!bf16 && B <= 64 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+        path = LSTM_APPROX_PATH_PERSISTENT;
+    } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
+      if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
+      if (!plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+        return fail(h, LSTM_APPROX_EINVAL, "persistent path unavailable: %s", why.c_str());
+    } else if (path == LSTM_APPROX_PATH_TENSOR) {
+      return fail(h, LSTM_APPROX_EINVAL, "tensor path not available for this shape");
+    }
+    PhaseTimer pt(h, 1);
+    if (path == LSTM_APPROX_PATH_PERSISTENT) {
+      PersistentArgs a{};
+      a.Vh = static_cast<const float*>(s.Vh);
+      a.U = static_cast<const float*>(s.U);
+      a.sigma = s.sigma;
+      a.bias = s.bias;
+      a.P = h->Px;
+      a.h0 = l_h0;
+      a.c0 = l_c0;
+      a.out_h = out;
+      a.c_last = l_cout;
+      a.ckpt_h = top ? ckpt_h : nullptr;
+      a.ckpt_c = top ? ckpt_c : nullptr;
+      a.err = h->err;
+      a.H = H;
+      a.K = K;
+      a.Ks = h->Ks;
+      a.ldh = h->ldh;
+      a.T = T;
+      a.B = B;
+      a.ck = lck;
+      a.wait_limit_ns = h->opt_wait_limit_us * 1000LL;
+      a.test_stall = h->opt_test_stall;
+      h->opt_test_stall = 0;
+      LA_CUDA(h, launch_persistent(plan, a, h->stream), "persistent kernel launch");
+      h->launches += 1;
+      h->last_cluster = plan.CS;
+    } else {
+      float* hs = h->h_state + (size_t)l * h->max_batch * H;
+      float* cs = h->c_state + (size_t)l * h->max_batch * H;
+      const size_t sb = (size_t)B * H * sizeof(float);
+      if (l_h0) LA_CUDA(h, cudaMemcpyAsync(hs, l_h0, sb, cudaMemcpyDeviceToDevice, h->stream), "h0 copy");
+      else LA_CUDA(h, cudaMemsetAsync(hs, 0, sb, h->stream), "h0 clear");
+      if (l_c0) LA_CUDA(h, cudaMemcpyAsync(cs, l_c0, sb, cudaMemcpyDeviceToDevice, h->stream), "c0 copy");
+      else LA_CUDA(h, cudaMemsetAsync(cs, 0, sb, h->stream), "c0 clear");
+      float* tau = static_cast<float*>(h->tau);
+      for (int t = 0; t < T; ++t) {
+        // (a2) tau' = sigma * (P_t + prune(v)[D:]^T h_{t-1})
+        LA_CUDA(h,
+                launch_rows_gemm(s.Vh, bf16, h->ldh, K, h->Ks, hs, H, B, H, tau, (int)ldp, 1, s.sigma,
+                                 h->Px + (size_t)t * B * ldp, (int)ldp, h->stream),
+                "recurrent projection launch");
+        // (a3, a4, a6) sums over u, intermediate outputs, cell update
+        CellArgs ca{};
+        ca.U = s.U;
+        ca.u_bf16 = bf16;
+        if (bf16) {
+          ca.gs = (long long)H * h->Ks;
+          ca.ks = 1;
+          ca.js = h->Ks;
+        } else {
+          ca.gs = (long long)h->Ks * H;
+          ca.ks = H;
+          ca.js = 1;
+        }
+        ca.K = K;
+        ca.Ks = h->Ks;
+        ca.H = H;
+        ca.B = B;
+        ca.tau = tau;
+        ca.ldt = (int)ldp;
+        ca.bias = s.bias;
+        ca.c_state = cs;
+        ca.h_state = hs;
+        ca.out_h = out + (size_t)t * B * H;
+        ca.ck = lck;
+        ca.ckpt_h = (top && ckpt_h) ? ckpt_h + (size_t)t * B * H : nullptr;
+        ca.ckpt_c = (top && ckpt_c) ? ckpt_c + (size_t)t * B * H : nullptr;
+        ca.ck_stride = (long long)T * B * H;
+        LA_CUDA(h, launch_cell_step(ca, h->stream), "cell step launch");
+        h->launches += 2;
+      }
+      if (l_cout) LA_CUDA(h, cudaMemcpyAsync(l_cout, cs, sb, cudaMemcpyDeviceToDevice, h->stream), "c copy");
+    }
+    h->last_path = path;
+  }
+  if (h->timing.on) cudaEventRecord(h->timing.run1, h->stream);
+  return LSTM_APPROX_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dims, int hidden, int max_rank,
+                       int max_batch, int dtype, void* cuda_stream) {
+  if (!out) return LSTM_APPROX_EINVAL;
+  *out = nullptr;
+  if (num_layers < 1 || num_layers > 64 || !input_dims || hidden < 1 || max_rank < 1 || max_batch < 1 ||
+      (dtype != LSTM_APPROX_FP32 && dtype != LSTM_APPROX_BF16))
+    return LSTM_APPROX_EINVAL;
+  if (input_dims[0] < 1) return LSTM_APPROX_EINVAL;
+  for (int l = 1; l < num_layers; ++l)
+    if (input_dims[l] != hidden) return LSTM_APPROX_EINVAL;
+  if (hidden > (1 << 20) || input_dims[0] > (1 << 22) || max_rank > (1 << 16) || max_batch > (1 << 20))
+    return LSTM_APPROX_EINVAL;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return LSTM_APPROX_ECUDA;
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return LSTM_APPROX_ECUDA;
+  if (prop.major != 10 || prop.minor != 3) return LSTM_APPROX_ECUDA;
+
+  lstm_approx_t* h = new (std::nothrow) lstm_approx;
+  if (!h) return LSTM_APPROX_ENOMEM;
+  h->L = num_layers;
+  h->H = hidden;
+  h->ldh = round_up(hidden, 8);
+  h->Kmax = max_rank;
+  h->Ks = dtype == LSTM_APPROX_BF16 ? round_up(max_rank, 128) : round_up(max_rank, 4);
+  h->max_batch = max_batch;
+  h->dtype = dtype;
+  h->stream = static_cast<cudaStream_t>(cuda_stream);
+  h->device = dev;
+  h->sm_count = prop.multiProcessorCount;
+  h->layers.resize(num_layers);
+  int rc = LSTM_APPROX_OK;
+  for (int l = 0; l < num_layers && !rc; ++l) {
+    LayerStore& s = h->layers[l];
+    s.D = input_dims[l];
+    s.C = s.D + hidden;
+    s.ldx = round_up(s.D, 8);
+    s.mask_words = (s.C + 31) / 32;
+    if (!rc) rc = dmalloc(h, &s.Vx, layer_bytes_vx(h, s), "factor storage");
+    if (!rc) rc = dmalloc(h, &s.Vh, layer_bytes_vh(h), "factor storage");
+    if (!rc) rc = dmalloc(h, &s.U, layer_bytes_u(h), "factor storage");
+    if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.sigma), 4ull * h->Ks * 4, "factor storage");
+    if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.bias), 4ull * hidden * 4, "factor storage");
+    if (!rc)
+      rc = dmalloc(h, reinterpret_cast<void**>(&s.mask), 4ull * h->Ks * s.mask_words * 4, "factor storage");
+  }
+  const size_t state = (size_t)num_layers * max_batch * hidden * sizeof(float);
+  if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->h_state), state, "state");
+  if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->c_state), state, "state");
+  if (!rc) rc = dmalloc(h, &h->tau, (size_t)max_batch * 4 * h->Ks * sizeof(float), "scratch tau");
+  if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->err), sizeof(int), "status word");
+  if (rc) {
+    lstm_approx_destroy(h);
+    return rc;
+  }
+  *out = h;
+  return LSTM_APPROX_OK;
+}
+
+int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz, const double* sigma,
+                            const double* u, const int32_t* v_idx, const double* v_val, const double* bias) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  if (layer < 0 || layer >= h->L) return fail(h, LSTM_APPROX_EINVAL, "layer %d outside [0, %d)", layer, h->L);
+  if (gate < 0 || gate > 3) return fail(h, LSTM_APPROX_EINVAL, "gate %d outside [0, 4)", gate);
+  LayerStore& s = h->layers[layer];
+  if (K < 1 || K > h->Kmax) return fail(h, LSTM_APPROX_EINVAL, "K=%d outside [1, %d]", K, h->Kmax);
+  if (nz < 1 || nz > s.C) return fail(h, LSTM_APPROX_EINVAL, "nz=%d outside [1, C=%d]", nz, s.C);
+  if (!sigma || !u || !v_idx || !v_val) return fail(h, LSTM_APPROX_EINVAL, "factor pointer is NULL");
+  for (int k = 0; k < K; ++k)
+    for (int m = 0; m < nz; ++m) {
+      const int32_t c = v_idx[(size_t)k * nz + m];
+      if (c < 0 || c >= s.C) return fail(h, LSTM_APPROX_EINVAL, "v_idx[%d][%d]=%d outside [0, %d)", k, m, c, s.C);
+      if (m > 0 && c <= v_idx[(size_t)k * nz + m - 1])
+        return fail(h, LSTM_APPROX_EINVAL, "v_idx row %d not strictly increasing", k);
+    }
+  DeviceGuard dg(h->device);
+  const int H = h->H, D = s.D, Ks = h->Ks;
+  const bool bf16 = h->dtype == LSTM_APPROX_BF16;
+  const size_t es = elem_size(h->dtype);
+  std::vector<unsigned char> vx((size_t)K * s.ldx * es, 0), vh((size_t)K * h->ldh * es, 0),
+      uu((size_t)K * H * es, 0);
+  std::vector<uint32_t> mask((size_t)K * s.mask_words, 0);
+  std::vector<float> sg(K), bs(H, 0.f);
+  auto put = [&](std::vector<unsigned char>& buf, size_t i, double v) {
+    if (bf16) {
+      const uint16_t b = to_bf16_bits(v);
+      std::memcpy(buf.data() + 2 * i, &b, 2);
+    } else {
+      const float f = static_cast<float>(v);
+      std::memcpy(buf.data() + 4 * i, &f, 4);
+    }
+  };
+  for (int k = 0; k < K; ++k) {
+    sg[k] = static_cast<float>(sigma[k]);
+    for (int m = 0; m < nz; ++m) {
+      const int c = v_idx[(size_t)k * nz + m];
+      const double v = v_val[(size_t)k * nz + m];
+      if (c < D) put(vx, (size_t)k * s.ldx + c, v);
+      else put(vh, (size_t)k * h->ldh + (c - D), v);
+      mask[(size_t)k * s.mask_words + c / 32] |= 1u << (c % 32);
+    }
+    for (int j = 0; j < H; ++j) {
+      // fp32: [K][H] rows; bf16: [H][K] (copied into [H][Ks] below)
+      if (bf16) put(uu, (size_t)j * K + k, u[(size_t)k * H + j]);
+      else put(uu, (size_t)k * H + j, u[(size_t)k * H + j]);
+    }
+  }
+  if (bias)
+    for (int j = 0; j < H; ++j) bs[j] = static_cast<float>(bias[j]);
+  const size_t row0 = (size_t)gate * Ks;
+  char* Vx = static_cast<char*>(s.Vx);
+  char* Vh = static_cast<char*>(s.Vh);
+  char* U = static_cast<char*>(s.U);
+  LA_CUDA(h, cudaMemcpy(Vx + row0 * s.ldx * es, vx.data(), vx.size(), cudaMemcpyHostToDevice), "factor upload");
+  LA_CUDA(h, cudaMemcpy(Vh + row0 * h->ldh * es, vh.data(), vh.size(), cudaMemcpyHostToDevice), "factor upload");
+  if (bf16)
+    LA_CUDA(h,
+            cudaMemcpy2D(U + (size_t)gate * H * Ks * es, Ks * es, uu.data(), K * es, K * es, H,
+                         cudaMemcpyHostToDevice),
+            "factor upload");
+  else
+    LA_CUDA(h, cudaMemcpy(U + row0 * H * es, uu.data(), uu.size(), cudaMemcpyHostToDevice), "factor upload");
+  LA_CUDA(h, cudaMemcpy(s.sigma + row0, sg.data(), K * sizeof(float), cudaMemcpyHostToDevice), "factor upload");
+  LA_CUDA(h, cudaMemcpy(s.bias + (size_t)gate * H, bs.data(), H * sizeof(float), cudaMemcpyHostToDevice),
+          "factor upload");
+  LA_CUDA(h,
+          cudaMemcpy(s.mask + row0 * s.mask_words, mask.data(), mask.size() * sizeof(uint32_t),
+                     cudaMemcpyHostToDevice),
+          "factor upload");
+  s.Kset[gate] = K;
+  s.nz[gate] = nz;
+  return LSTM_APPROX_OK;
+}
+
+int lstm_approx_run(lstm_approx_t* h, const float* x, int T, int B, int K, const float* h0, const float* c0,
+                    float* out_h, float* out_c, const int* checkpoints, int J, float* ckpt_h, float* ckpt_c) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  Checkpoints ck;
+  int rc = validate_run(h, x, T, B, K, out_h, checkpoints, J, &ck);
+  if (rc) return rc;
+  DeviceGuard dg(h->device);
+  return run_device(h, x, T, B, K, h0, c0, out_h, out_c, ck, ckpt_h, ckpt_c);
+}
+
+int lstm_approx_run_host(lstm_approx_t* h, const float* x, int T, int B, int K, const float* h0, const float* c0,
+                         float* out_h, float* out_c, const int* checkpoints, int J, float* ckpt_h, float* ckpt_c) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  Checkpoints ck;
+  int rc = validate_run(h, x, T, B, K, out_h, checkpoints, J, &ck);
+  if (rc) return rc;
+  DeviceGuard dg(h->device);
+  const size_t H = h->H, L = h->L, D = h->layers[0].D;
+  const size_t nx = (size_t)T * B * D, ns = L * B * H, no = (size_t)T * B * H, nk = (size_t)J * T * B * H;
+  const size_t off_x = 0, off_h0 = off_x + nx, off_c0 = off_h0 + ns, off_oh = off_c0 + ns, off_oc = off_oh + no,
+               off_kh = off_oc + ns, off_kc = off_kh + nk, total = (off_kc + nk) * sizeof(float);
+  if (total > h->stage_bytes) {
+    LA_CUDA(h, cudaStreamSynchronize(h->stream), "synchronising before growing staging");
+    dfree(h, h->stage, h->stage_bytes);
+    h->stage = nullptr;
+    h->stage_bytes = 0;
+    rc = dmalloc(h, reinterpret_cast<void**>(&h->stage), total, "host-call staging");
+    if (rc) return rc;
+    h->stage_bytes = total;
+  }
+  float* st = reinterpret_cast<float*>(h->stage);
+  LA_CUDA(h, cudaMemcpyAsync(st + off_x, x, nx * 4, cudaMemcpyHostToDevice, h->stream), "input copy");
+  if (h0) LA_CUDA(h, cudaMemcpyAsync(st + off_h0, h0, ns * 4, cudaMemcpyHostToDevice, h->stream), "h0 copy");
+  if (c0) LA_CUDA(h, cudaMemcpyAsync(st + off_c0, c0, ns * 4, cudaMemcpyHostToDevice, h->stream), "c0 copy");
+  rc = run_device(h, st + off_x, T, B, K, h0 ? st + off_h0 : nullptr, c0 ? st + off_c0 : nullptr, st + off_oh,
+                  out_c ? st + off_oc : nullptr, ck, ckpt_h ? st + off_kh : nullptr, ckpt_c ? st + off_kc : nullptr);
+  if (rc) return rc;
+  LA_CUDA(h, cudaMemcpyAsync(out_h, st + off_oh, no * 4, cudaMemcpyDeviceToHost, h->stream), "output copy");
+  if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, st + off_oc, ns * 4, cudaMemcpyDeviceToHost, h->stream), "c copy");
+  if (ckpt_h && nk)
+    LA_CUDA(h, cudaMemcpyAsync(ckpt_h, st + off_kh, nk * 4, cudaMemcpyDeviceToHost, h->stream), "ckpt copy");
+  if (ckpt_c && nk)
+    LA_CUDA(h, cudaMemcpyAsync(ckpt_c, st + off_kc, nk * 4, cudaMemcpyDeviceToHost, h->stream), "ckpt copy");
+  return lstm_approx_sync(h);
+}
+
+int lstm_approx_sync(lstm_approx_t* h) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  DeviceGuard dg(h->device);
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
+  int code = 0;
+  LA_CUDA(h, cudaMemcpy(&code, h->err, sizeof(int), cudaMemcpyDeviceToHost), "status read");
+  if (code != 0) {
+    LA_CUDA(h, cudaMemset(h->err, 0, sizeof(int)), "status clear");
+    return fail(h, LSTM_APPROX_ETIMEOUT, "a bounded in-kernel wait ran out (code %d); outputs are invalid", code);
+  }
+  return LSTM_APPROX_OK;
+}
+
+int lstm_approx_get_mask(lstm_approx_t* h, int layer, int gate, int k, int32_t* idx_out, int* nz_out) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  if (layer < 0 || layer >= h->L || gate < 0 || gate > 3 || !idx_out || !nz_out)
+    return fail(h, LSTM_APPROX_EINVAL, "bad layer/gate/pointer");
+  const LayerStore& s = h->layers[layer];
+  if (k < 0 || k >= s.Kset[gate]) return fail(h, LSTM_APPROX_EINVAL, "term %d not set", k);
+  DeviceGuard dg(h->device);
+  std::vector<uint32_t> words(s.mask_words);
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
+  LA_CUDA(h,
+          cudaMemcpy(words.data(), s.mask + ((size_t)gate * h->Ks + k) * s.mask_words,
+                     s.mask_words * sizeof(uint32_t), cudaMemcpyDeviceToHost),
+          "mask read");
+  int n = 0;
+  for (int c = 0; c < s.C; ++c)
+    if (words[c / 32] >> (c % 32) & 1u) idx_out[n++] = c;
+  *nz_out = n;
+  return LSTM_APPROX_OK;
+}
+
+const char* lstm_approx_last_error(const lstm_approx_t* h) {
+  if (!h) return "invalid handle (NULL)";
+  return h->last_error.c_str();
+}
+
+void lstm_approx_destroy(lstm_approx_t* h) {
+  if (!h) return;
+  DeviceGuard dg(h->device);
+  cudaStreamSynchronize(h->stream);
+  clear_timing(h);
+  if (h->timing.run0) cudaEventDestroy(h->timing.run0);
+  if (h->timing.run1) cudaEventDestroy(h->timing.run1);
+  for (LayerStore& s : h->layers) {
+    cudaFree(s.Vx);
+    cudaFree(s.Vh);
+    cudaFree(s.U);
+    cudaFree(s.sigma);
+    cudaFree(s.bias);
+    cudaFree(s.mask);
+  }
+  cudaFree(h->h_state);
+  cudaFree(h->c_state);
+  cudaFree(h->Px);
+  cudaFree(h->seq);
+  cudaFree(h->tau);
+  cudaFree(h->err);
+  cudaFree(h->stage);
+  delete h;
+}
+
+int lstm_approx_query(const lstm_approx_t* h, int key, long long* value) {
+  if (!h || !value) return LSTM_APPROX_EINVAL;
+  switch (key) {
+    case LSTM_APPROX_Q_LAUNCHES: *value = h->launches; return LSTM_APPROX_OK;
+    case LSTM_APPROX_Q_LAST_PATH: *value = h->last_path; return LSTM_APPROX_OK;
+    case LSTM_APPROX_Q_CLUSTER: *value = h->last_cluster; return LSTM_APPROX_OK;
+    case LSTM_APPROX_Q_DEVICE_BYTES: *value = h->device_bytes; return LSTM_APPROX_OK;
+    default: return LSTM_APPROX_EINVAL;
+  }
+}
+
+int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  switch (key) {
+    case LSTM_APPROX_OPT_FORCE_PATH:
+      if (value < 0 || value > 3) return fail(h, LSTM_APPROX_EINVAL, "bad path %lld", value);
+      h->opt_force_path = (int)value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_CLUSTER:
+      if (value != 0 && value != 1 && value != 2 && value != 4 && value != 8 && value != 16)
+        return fail(h, LSTM_APPROX_EINVAL, "bad cluster size %lld", value);
+      h->opt_cluster = (int)value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_TIMING:
+      h->timing.on = value != 0;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_WAIT_LIMIT:
+      if (value < 1) return fail(h, LSTM_APPROX_EINVAL, "wait limit must be >= 1 us");
+      h->opt_wait_limit_us = value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_TEST_STALL:
+      h->opt_test_stall = value != 0;
+      return LSTM_APPROX_OK;
+    default: return fail(h, LSTM_APPROX_EINVAL, "unknown option %d", key);
+  }
+}
+
+int lstm_approx_phase_times(lstm_approx_t* h, float* ms_out) {
+  if (!h || !ms_out) return LSTM_APPROX_EINVAL;
+  if (!h->timing.on || !h->timing.run0) return fail(h, LSTM_APPROX_ESTATE, "timing was not enabled for the last run");
+  DeviceGuard dg(h->device);
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
+  ms_out[0] = ms_out[1] = ms_out[2] = 0.f;
+  for (size_t i = 0; i + 1 < h->timing.ev.size(); i += 2) {
+    float ms = 0.f;
+    LA_CUDA(h, cudaEventElapsedTime(&ms, h->timing.ev[i], h->timing.ev[i + 1]), "event time");
+    ms_out[h->timing.phase[i / 2]] += ms;
+  }
+  LA_CUDA(h, cudaEventElapsedTime(&ms_out[2], h->timing.run0, h->timing.run1), "event time");
+  return LSTM_APPROX_OK;
+}
+
+}  // extern "C"

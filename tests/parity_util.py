@@ -1,0 +1,95 @@
+"""Helpers shared by the GPU parity tests (test infrastructure)."""
+from __future__ import annotations
+
+import functools
+
+import numpy as np
+
+import oracle
+from workloads import (WORKLOADS, draw_weights, nz_from_keep, rounded_factors, synthetic_layer_factors,
+                       workload_inputs)
+
+FP32_TOL = 1e-4   # max relative error, fp32 factors
+BF16_TOL = 2e-2   # max relative error, bf16 factors / fp32 accumulate
+
+
+def max_rel_err(got, ref) -> float:
+    """max_i |got_i - ref_i| / max(|ref_i|, 1e-2 * max_j |ref_j|)."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    if ref.size == 0:
+        return 0.0
+    floor = 1e-2 * max(np.abs(ref).max(), 1e-30)
+    return float((np.abs(got - ref) / np.maximum(np.abs(ref), floor)).max())
+
+
+@functools.lru_cache(maxsize=None)
+def decomposed_layer(wname: str, layer: int, K: int, keep: float):
+    """Oracle residual decomposition of the workload's seeded gate matrices."""
+    w = WORKLOADS[wname]
+    nz = nz_from_keep(keep, w.C(layer))
+    return tuple(oracle.decompose_layer(draw_weights(w, layer), K, nz))
+
+
+@functools.lru_cache(maxsize=None)
+def synthetic_layer(wname: str, layer: int, K: int, keep: float):
+    return tuple(synthetic_layer_factors(WORKLOADS[wname], layer, K, keep))
+
+
+def run_gpu(layers, x, K, dtype="fp32", h0=None, c0=None, checkpoints=(), force_path=0, cluster=0,
+            max_rank=None, max_batch=None, want_c=True):
+    """Set factors, run through the C-ABI, return numpy outputs and the handle."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, OPT_CLUSTER, OPT_FORCE_PATH
+    dev = torch.device("cuda:0")
+    T, B, D = x.shape
+    L = len(layers)
+    H = layers[0][0]["u"].shape[1]
+    mr = max_rank or max(len(g["sigma"]) for lay in layers for g in lay)
+    m = LSTMApprox(L, [D] + [H] * (L - 1), H, mr, max_batch or B, dtype)
+    for l, gates in enumerate(layers):
+        m.set_layer(l, gates)
+    if force_path:
+        m.set_option(OPT_FORCE_PATH, force_path)
+    if cluster:
+        m.set_option(OPT_CLUSTER, cluster)
+    xt = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(dev)
+    out_h = torch.full((T, B, H), float("nan"), device=dev)
+    out_c = torch.full((L, B, H), float("nan"), device=dev) if want_c else None
+    J = len(checkpoints)
+    ck_h = torch.full((J, T, B, H), float("nan"), device=dev) if J else None
+    ck_c = torch.full((J, T, B, H), float("nan"), device=dev) if J else None
+    th0 = None if h0 is None else torch.from_numpy(np.ascontiguousarray(h0, dtype=np.float32)).to(dev)
+    tc0 = None if c0 is None else torch.from_numpy(np.ascontiguousarray(c0, dtype=np.float32)).to(dev)
+    m.run(xt, K, out_h, h0=th0, c0=tc0, out_c=out_c, checkpoints=list(checkpoints), ckpt_h=ck_h, ckpt_c=ck_c)
+    m.sync()
+    res = {"h": out_h.double().cpu().numpy()}
+    if want_c:
+        res["c_last"] = out_c.double().cpu().numpy()
+    if J:
+        res["ckpt_h"] = ck_h.double().cpu().numpy()
+        res["ckpt_c"] = ck_c.double().cpu().numpy()
+    return res, m
+
+
+def oracle_run(layers, x, K, dtype="fp32", **kw):
+    """Oracle on the factors as the library stores them (rounded to dtype)."""
+    rl = [rounded_factors(g, dtype) for g in layers]
+    xr = np.asarray(x, dtype=np.float32).astype(np.float64)
+    return oracle.run_lstm(rl, xr, K, **kw)
+
+
+def assert_parity(got, ref, tol, keys=("h", "c_last", "ckpt_h", "ckpt_c")):
+    errs = {}
+    for k in keys:
+        if k in got and k in ref:
+            assert np.all(np.isfinite(got[k])), f"{k}: non-finite output"
+            errs[k] = max_rel_err(got[k], ref[k])
+    bad = {k: v for k, v in errs.items() if v > tol}
+    assert not bad, f"max relative error above {tol}: {errs}"
+    return errs
+
+
+__all__ = ["FP32_TOL", "BF16_TOL", "max_rel_err", "decomposed_layer", "synthetic_layer", "run_gpu",
+           "oracle_run", "assert_parity", "workload_inputs", "WORKLOADS"]

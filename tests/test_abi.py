@@ -1,0 +1,83 @@
+"""The C-ABI library loads and exports every entry point its header declares.
+
+Runs without a GPU: no call here launches or computes anything.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for f in os.listdir(inc):
+        if f.endswith(".h"):
+            text = open(os.path.join(inc, f)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(lstm_approx_\w+)\s*\(", text))
+    return names
+
+
+@pytest.fixture(scope="module")
+def built_lib():
+    from paper_1905_00689_gb300 import build as b
+    b.build()
+    from paper_1905_00689_gb300 import _binding
+    return _binding.load()
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_destroy",
+              "lstm_approx_get_mask", "lstm_approx_last_error"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(built_lib):
+    for n in sorted(_declared()):
+        assert hasattr(built_lib, n), f"{n} declared in include/ but not exported"
+
+
+def test_binding_covers_every_declared_symbol():
+    from paper_1905_00689_gb300 import _binding
+    assert set(_binding.EXPORTS) == _declared()
+
+
+def test_invalid_arguments_rejected_before_any_device_work(built_lib):
+    h = ctypes.c_void_p()
+    dims = (ctypes.c_int * 2)(16, 99)
+    # layer 1's input must equal the hidden size
+    assert built_lib.lstm_approx_create(ctypes.byref(h), 2, dims, 8, 4, 1, 0, None) == 1
+    assert built_lib.lstm_approx_create(ctypes.byref(h), 0, dims, 8, 4, 1, 0, None) == 1
+    assert built_lib.lstm_approx_create(ctypes.byref(h), 1, dims, 8, 4, 1, 7, None) == 1
+    assert built_lib.lstm_approx_create(None, 1, dims, 8, 4, 1, 0, None) == 1
+    assert h.value is None
+    # NULL handles are rejected, destroy is NULL-safe
+    assert built_lib.lstm_approx_run(None, None, 1, 1, 1, None, None, None, None, None, 0, None, None) == 1
+    assert built_lib.lstm_approx_sync(None) == 1
+    built_lib.lstm_approx_destroy(None)
+    assert built_lib.lstm_approx_last_error(None) == b"invalid handle (NULL)"
+
+
+def test_no_cpu_fallback_without_a_device(built_lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a CUDA device is present")
+    h = ctypes.c_void_p()
+    dims = (ctypes.c_int * 1)(16)
+    assert built_lib.lstm_approx_create(ctypes.byref(h), 1, dims, 8, 4, 1, 0, None) == 3  # ECUDA
+    assert h.value is None
+
+
+def test_product_path_does_not_import_the_oracle():
+    pkg = os.path.join(ROOT, "paper_1905_00689_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(from|import)\s+oracle", text, flags=re.M), f
+                assert "oracle/" not in text, f
