@@ -136,6 +136,42 @@ int lstm_approx_run_host(lstm_approx_t *h, const float *x, int T, int B, int K, 
                          float *ckpt_h, float *ckpt_c);
 
 /*
+ * Allocation-free variant of lstm_approx_run for one fp32 layer.  The paper
+ * has no counterpart: this entry point exists for callers that must not
+ * allocate device memory once running -- hard real-time control loops,
+ * where cudaMalloc's unbounded latency (and device synchronisation) is not
+ * acceptable and safety rules often forbid allocation after start-up, and
+ * plug-ins inside a host framework whose own allocator owns all device
+ * memory.  Such callers allocate factors, inputs and outputs up front and
+ * pass them here; no handle is involved and nothing is allocated.
+ *
+ * Factors are caller-owned DEVICE arrays, fp32, in the library's packed
+ * layout (row (g, k) = g*K + k, gate order i, f, g, o):
+ *   Vx [4][K][D]  masked-dense pruned v over the x columns (zeros elsewhere)
+ *   Vh [4][K][H]  masked-dense pruned v over the h columns (16-byte aligned)
+ *   U  [4][K][H]  u_k (16-byte aligned);  sigma [4][K];  bias [4][H] or NULL
+ * x, h0, c0, out_h, out_c, checkpoints, J, ckpt_h, ckpt_c: as for
+ * lstm_approx_run with L = 1 (device pointers, checkpoints on the host).
+ * cuda_stream: cudaStream_t to run on (NULL = legacy default stream).
+ * msg: optional host buffer of msg_len bytes that receives an error text.
+ *
+ * The scratch (the hoisted input projection, a status word, a zero bias)
+ * is a fixed 4 MiB __device__ array inside the library, held by every GPU
+ * that loads it until the process exits; calls needing more than
+ * T*B*4*K + 4*H (rounded up to 64) + 64 <= 1048576 floats are rejected with
+ * EINVAL.  The first call on a device looks up the array's address (do it
+ * before any stream capture).  Every call shares the array and it keeps the
+ * last call's contents, so calls that overlap on the GPU race.  The call is
+ * synchronous: it waits for the stream and returns OK, EINVAL (sizes,
+ * alignment, a shape the persistent kernel cannot hold), ECUDA or ETIMEOUT.
+ */
+int lstm_approx_run_static(const float *Vx, const float *Vh, const float *U, const float *sigma,
+                           const float *bias, int D, int H, int K, const float *x, int T, int B,
+                           const float *h0, const float *c0, float *out_h, float *out_c,
+                           const int *checkpoints, int J, float *ckpt_h, float *ckpt_c,
+                           void *cuda_stream, char *msg, int msg_len);
+
+/*
  * Wait for the handle's stream and report kernel-side status: OK, or
  * ETIMEOUT when a bounded in-kernel wait ran out since the last sync (the
  * outputs of that run are then invalid; the status word is cleared), or

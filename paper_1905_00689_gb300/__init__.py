@@ -7,7 +7,7 @@ Importing the package does not load the library; constructing
 been built.
 """
 from ._binding import (  # noqa: F401
-    BF16, FP32, LSTMApprox, LSTMApproxError, load,
+    BF16, FP32, LSTMApprox, LSTMApproxError, load, run_static,
     PATH_NONE, PATH_PERSISTENT, PATH_SIMT, PATH_TENSOR,
     OPT_CLUSTER, OPT_FORCE_PATH, OPT_TEST_STALL, OPT_TIMING, OPT_WAIT_LIMIT,
     Q_CLUSTER, Q_DEVICE_BYTES, Q_LAST_PATH, Q_LAUNCHES,

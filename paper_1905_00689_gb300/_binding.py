@@ -28,7 +28,7 @@ STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ET
 EXPORTS = (
     "lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_run_host",
     "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
-    "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times",
+    "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times", "lstm_approx_run_static",
 )
 
 _lib = None
@@ -64,6 +64,8 @@ def load(path: str = LIB_PATH):
     lib.lstm_approx_query.argtypes = [P, I, ctypes.POINTER(LL)]
     lib.lstm_approx_set_option.argtypes = [P, I, LL]
     lib.lstm_approx_phase_times.argtypes = [P, ctypes.POINTER(ctypes.c_float)]
+    lib.lstm_approx_run_static.argtypes = [P, P, P, P, P, I, I, I, P, I, I, P, P, P, P, P, I, P, P, P,
+                                           ctypes.c_char_p, I]
     for name in EXPORTS:
         if name not in ("lstm_approx_last_error", "lstm_approx_destroy"):
             getattr(lib, name).restype = ctypes.c_int
@@ -84,6 +86,28 @@ def _np_ptr(a) -> Optional[int]:
     if a is None:
         return None
     return a.ctypes.data
+
+
+def run_static(Vx, Vh, U, sigma, bias, x, K, out_h, h0=None, c0=None, out_c=None, checkpoints=(),
+               ckpt_h=None, ckpt_c=None, stream=None):
+    """lstm_approx_run_static on torch CUDA tensors (no handle, no device allocation).
+
+    Vx [4][K][D], Vh [4][K][H], U [4][K][H], sigma [4][K], bias [4][H] or None:
+    fp32 factors in the library's packed layout.  Synchronous.
+    """
+    import torch
+    lib = load()
+    T, B, D = x.shape
+    H = Vh.shape[-1]
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    cps = (ctypes.c_int * max(1, len(checkpoints)))(*checkpoints)
+    msg = ctypes.create_string_buffer(512)
+    rc = lib.lstm_approx_run_static(_ptr(Vx), _ptr(Vh), _ptr(U), _ptr(sigma), _ptr(bias), D, H, K, _ptr(x), T, B,
+                                    _ptr(h0), _ptr(c0), _ptr(out_h), _ptr(out_c), cps, len(checkpoints),
+                                    _ptr(ckpt_h), _ptr(ckpt_c), ctypes.c_void_p(stream.cuda_stream), msg, 512)
+    if rc != OK:
+        raise LSTMApproxError(rc, msg.value.decode())
 
 
 class LSTMApprox:
