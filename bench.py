@@ -274,7 +274,7 @@ def run_ours(args):
     # ---- per-phase device times (CUDA events on the library's stream) ------
     m.set_option(OPT_TIMING, 1)
     ph = []
-    for i in range(max(10, min(args.steps, 50))):
+    for i in range(3 if args.quick else max(10, min(args.steps, 50))):
         flush.fill_(float(i))
         step()
         ph.append(m.phase_times())
@@ -284,7 +284,7 @@ def run_ours(args):
 
     # ---- K sweep (separate runs, no intermediate outputs) ------------------
     sweep = []
-    for K in K_SWEEP:
+    for K in (() if args.quick else K_SWEEP):
         for _ in range(3):
             step(K, ())
         t = timed_loop(max(10, min(args.steps, 50)), lambda K=K: step(K, ()))
@@ -301,7 +301,7 @@ def run_ours(args):
     for _ in range(3):
         m.run_host(xh_np, K_MAIN, oh_np, checkpoints=list(CKPTS), ckpt_h=kh_np)
     e2e_t = []
-    for i in range(args.steps):
+    for i in range(2 if args.quick else args.steps):
         flush.fill_(float(i))
         torch.cuda.synchronize(dev)
         t0 = time.perf_counter()
@@ -347,7 +347,7 @@ def run_ours(args):
             "cluster_ctas": cluster,
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
         }
-        if ws == 1 and not args.no_cpu_baseline:
+        if ws == 1 and not (args.no_cpu_baseline or args.quick):
             line["cpu_baseline"] = cpu_baseline()
         print(json.dumps(line), flush=True)
     if dist:
@@ -362,6 +362,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--quick", action="store_true",
+                    help="main timed loop only (short side measurements, no K sweep, no CPU baseline)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
