@@ -149,7 +149,8 @@ int lstm_approx_run_host(lstm_approx_t *h, const float *x, int T, int B, int K, 
  * layout (row (g, k) = g*K + k, gate order i, f, g, o):
  *   Vx [4][K][D]  masked-dense pruned v over the x columns (zeros elsewhere)
  *   Vh [4][K][H]  masked-dense pruned v over the h columns (16-byte aligned)
- *   U  [4][K][H]  u_k (16-byte aligned);  sigma [4][K];  bias [4][H] or NULL
+ *   U  [4][H][K]  u_k[j] at (g*H + j)*K + k (16-byte aligned);  sigma [4][K];
+ *                 bias [4][H] or NULL
  * x, h0, c0, out_h, out_c, checkpoints, J, ckpt_h, ckpt_c: as for
  * lstm_approx_run with L = 1 (device pointers, checkpoints on the host).
  * cuda_stream: cudaStream_t to run on (NULL = legacy default stream).

@@ -92,7 +92,7 @@ def run_static(Vx, Vh, U, sigma, bias, x, K, out_h, h0=None, c0=None, out_c=None
                ckpt_h=None, ckpt_c=None, stream=None):
     """lstm_approx_run_static on torch CUDA tensors (no handle, no device allocation).
 
-    Vx [4][K][D], Vh [4][K][H], U [4][K][H], sigma [4][K], bias [4][H] or None:
+    Vx [4][K][D], Vh [4][K][H], U [4][H][K], sigma [4][K], bias [4][H] or None:
     fp32 factors in the library's packed layout.  Synchronous.
     """
     import torch

@@ -22,8 +22,8 @@ struct Checkpoints {
 // storage row g * Ks + k ("gate-major"), rows k >= K_set are zero.
 //   Vx   [4*Ks][ldx]  masked-dense pruned v over the x columns (ldx >= D)
 //   Vh   [4*Ks][ldh]  masked-dense pruned v over the h columns (ldh >= H)
-//   U    fp32: [4][Ks][H] (u_k[j] at (g*Ks + k)*H + j)
-//        bf16: [4][H][Ks] (u_k[j] at (g*H + j)*Ks + k, K-major for the MMA)
+//   U    [4][H][Ks] (u_k[j] at (g*H + j)*Ks + k): K-major, so the terms a
+//        lane or an MMA operand needs are contiguous
 //   sigma [4][Ks] fp32, bias [4][H] fp32
 //   mask [4*Ks][mask_words] bit c set <=> column c of x~ is kept
 struct LayerStore {
@@ -89,6 +89,12 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
                              int N, int Kdim, float* out, int ldo, int mode, const float* sigma,
                              const float* P, int ldp, cudaStream_t s);
 
+// Same product for few columns (N = T*B <= 32): 8-CTA clusters split the
+// D axis and reduce through distributed shared memory (deterministic).
+bool xproj_cluster_fits(int N);
+cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
+                                 int N, int D, float* out, int ldo, cudaStream_t s);
+
 // One timestep of the refinement sums over u (a3), the intermediate outputs
 // (a6) and the cell update (a4) for B streams.
 struct CellArgs {
@@ -114,14 +120,10 @@ cudaError_t launch_cell_step(const CellArgs& a, cudaStream_t s);
 struct PersistentPlan {
   int CS = 0;        // CTAs per cluster
   int RA = 0;        // coefficient rows per CTA (multiple of 4)
-  int UB = 0;        // hidden units per CTA (multiple of 4)
-  int upl = 0;       // units per lane (1 or 2)
-  int kpw = 0;       // refinement terms per warp segment
-  int nseg = 0;      // segments (<= warps)
-  int seg_start[17] = {0};
-  int ck_seg[kMaxCheckpoints] = {0};
-  size_t smem = 0;
-  int pxc = 0;       // timesteps of P staged in shared memory at once
+  int UB = 0;        // hidden units per CTA (16 * upl)
+  int upl = 0;       // hidden units per warp (1, 2 or 4)
+  int kpw = 0;       // refinement terms per lane (1, 2, 4 or 8)
+  size_t smem = 0;   // dynamic shared memory bytes
 };
 
 // Chooses a plan; returns false (with a reason) if the shape does not fit.
@@ -130,7 +132,7 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
 
 struct PersistentArgs {
   const float* Vh;     // [4*Ks][ldh]
-  const float* U;      // [4][Ks][H]
+  const float* U;      // [4][H][Ks]
   const float* sigma;  // [4][Ks]
   const float* bias;   // [4][H]
   const float* P;      // [T][B][4*Ks]

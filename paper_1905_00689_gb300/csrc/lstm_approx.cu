@@ -187,10 +187,14 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
     {
       PhaseTimer pt(h, 0);
-      LA_CUDA(h,
-              launch_rows_gemm(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, 0, nullptr,
-                               nullptr, 0, h->stream),
-              "input projection launch");
+      if (xproj_cluster_fits(T * B))
+        LA_CUDA(h, launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->stream),
+                "input projection launch");
+      else
+        LA_CUDA(h,
+                launch_rows_gemm(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, 0, nullptr,
+                                 nullptr, 0, h->stream),
+                "input projection launch");
       h->launches += 1;
     }
     const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
@@ -203,7 +207,7 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     std::string why;
     if (path == 0) {
       path = LSTM_APPROX_PATH_SIMT;
-      if (!bf16 && B <= 64 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+      if (!bf16 && B <= 8 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
         path = LSTM_APPROX_PATH_PERSISTENT;
     } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
       if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
@@ -259,15 +263,9 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
         CellArgs ca{};
         ca.U = s.U;
         ca.u_bf16 = bf16;
-        if (bf16) {
-          ca.gs = (long long)H * h->Ks;
-          ca.ks = 1;
-          ca.js = h->Ks;
-        } else {
-          ca.gs = (long long)h->Ks * H;
-          ca.ks = H;
-          ca.js = 1;
-        }
+        ca.gs = (long long)H * h->Ks;  // U is [4][H][Ks] for both factor types
+        ca.ks = 1;
+        ca.js = h->Ks;
         ca.K = K;
         ca.Ks = h->Ks;
         ca.H = H;
@@ -399,11 +397,7 @@ int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz
       else put(vh, (size_t)k * h->ldh + (c - D), v);
       mask[(size_t)k * s.mask_words + c / 32] |= 1u << (c % 32);
     }
-    for (int j = 0; j < H; ++j) {
-      // fp32: [K][H] rows; bf16: [H][K] (copied into [H][Ks] below)
-      if (bf16) put(uu, (size_t)j * K + k, u[(size_t)k * H + j]);
-      else put(uu, (size_t)k * H + j, u[(size_t)k * H + j]);
-    }
+    for (int j = 0; j < H; ++j) put(uu, (size_t)j * K + k, u[(size_t)k * H + j]);  // [H][K], into [H][Ks] below
   }
   if (bias)
     for (int j = 0; j < H; ++j) bs[j] = static_cast<float>(bias[j]);
@@ -413,13 +407,9 @@ int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz
   char* U = static_cast<char*>(s.U);
   LA_CUDA(h, cudaMemcpy(Vx + row0 * s.ldx * es, vx.data(), vx.size(), cudaMemcpyHostToDevice), "factor upload");
   LA_CUDA(h, cudaMemcpy(Vh + row0 * h->ldh * es, vh.data(), vh.size(), cudaMemcpyHostToDevice), "factor upload");
-  if (bf16)
-    LA_CUDA(h,
-            cudaMemcpy2D(U + (size_t)gate * H * Ks * es, Ks * es, uu.data(), K * es, K * es, H,
-                         cudaMemcpyHostToDevice),
-            "factor upload");
-  else
-    LA_CUDA(h, cudaMemcpy(U + row0 * H * es, uu.data(), uu.size(), cudaMemcpyHostToDevice), "factor upload");
+  LA_CUDA(h,
+          cudaMemcpy2D(U + (size_t)gate * H * Ks * es, Ks * es, uu.data(), K * es, K * es, H, cudaMemcpyHostToDevice),
+          "factor upload");
   LA_CUDA(h, cudaMemcpy(s.sigma + row0, sg.data(), K * sizeof(float), cudaMemcpyHostToDevice), "factor upload");
   LA_CUDA(h, cudaMemcpy(s.bias + (size_t)gate * H, bs.data(), H * sizeof(float), cudaMemcpyHostToDevice),
           "factor upload");

@@ -51,14 +51,16 @@ __device__ __forceinline__ void mbar_arrive(uint32_t mb) {
 
 // One poll of an mbarrier phase (acquire at cluster scope, so data written
 // by st.async from other CTAs of the cluster is visible once it returns 1).
+// The suspend-time hint (ns) lets a waiting warp sleep in hardware instead
+// of spinning, so it does not take issue slots from warps still working.
 __device__ __forceinline__ uint32_t mbar_try_wait_cluster(uint32_t mb, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(mb), "r"(parity)
+      : "r"(mb), "r"(parity), "r"(20000u)
       : "memory");
   return ok;
 }
@@ -85,7 +87,7 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t mb, uint32_t parity, 
   const uint64_t t0 = global_timer_ns();
   for (uint32_t i = 1;; ++i) {
     if (kCluster ? mbar_try_wait_cluster(mb, parity) : mbar_try_wait_cta(mb, parity)) return true;
-    if ((i & 255u) == 0u) {
+    if ((i & 15u) == 0u) {
       if (*err != 0) return false;
       if (global_timer_ns() - t0 > limit_ns) return false;
     }
@@ -104,13 +106,24 @@ __device__ __forceinline__ void st_async_v4(uint32_t remote_addr, float a, float
       : "memory");
 }
 
+// Bulk copy (TMA engine, no tensor map) of `bytes` from global to this CTA's
+// shared memory, completing `bytes` on the mbarrier at `mb`.  Addresses and
+// size must be multiples of 16 bytes.
+__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t mb) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(mb)
+               : "memory");
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-__device__ __forceinline__ float sigmoid_f(float z) { return 1.0f / (1.0f + expf(-z)); }
+// Logistic function from the hardware exponential and a correctly rounded
+// reciprocal: relative error a few units in the last place of fp32.
+__device__ __forceinline__ float sigmoid_f(float z) { return __frcp_rn(1.0f + __expf(-z)); }
 
 // Gate nonlinearities and cell update (Sec. II): i, f, o sigmoid, g tanh;
 // c = f c_prev + i g; h = o tanh(c).  Pre-activations already include bias.

@@ -20,10 +20,10 @@ pytestmark = pytest.mark.gpu
 
 
 def _pack(gates, D, H, K):
-    """Masked-dense fp32 packing of one layer: Vx [4][K][D], Vh [4][K][H], U [4][K][H], sigma [4][K]."""
+    """Masked-dense fp32 packing of one layer: Vx [4][K][D], Vh [4][K][H], U [4][H][K], sigma [4][K]."""
     Vx = np.zeros((4, K, D), np.float32)
     Vh = np.zeros((4, K, H), np.float32)
-    U = np.zeros((4, K, H), np.float32)
+    U = np.zeros((4, H, K), np.float32)
     S = np.zeros((4, K), np.float32)
     for g, f in enumerate(gates):
         for k in range(K):
@@ -32,7 +32,7 @@ def _pack(gates, D, H, K):
                     Vx[g, k, c] = v
                 else:
                     Vh[g, k, c - D] = v
-        U[g] = f["u"][:K]
+        U[g] = f["u"][:K].T
         S[g] = f["sigma"][:K]
     return Vx, Vh, U, S
 
@@ -67,7 +67,7 @@ def test_static_entry_point_rejects_oversized_scratch(cuda_device):
     dev = torch.device("cuda:0")
     Vx = torch.zeros((4, K, D), device=dev)
     Vh = torch.zeros((4, K, H), device=dev)
-    U = torch.zeros((4, K, H), device=dev)
+    U = torch.zeros((4, H, K), device=dev)
     S = torch.zeros((4, K), device=dev)
     x = torch.zeros((T, B, D), device=dev)
     out_h = torch.zeros((T, B, H), device=dev)
