@@ -18,6 +18,11 @@ struct Checkpoints {
   int k[kMaxCheckpoints];
 };
 
+// Opaque storage of one CUtensorMap (128 bytes, 64-byte aligned).
+struct alignas(64) TcMap {
+  unsigned char bytes[128];
+};
+
 // Device factor storage of one layer.  Row (g, k) of the packed matrices is
 // storage row g * Ks + k ("gate-major"), rows k >= K_set are zero.
 //   Vx   [4*Ks][ldx]  masked-dense pruned v over the x columns (ldx >= D)
@@ -37,6 +42,8 @@ struct LayerStore {
   int mask_words = 0;
   int Kset[4] = {0, 0, 0, 0};
   int nz[4] = {0, 0, 0, 0};
+  bool maps_ready = false;  // tensor maps of Vx, Vh, U (bf16 path), built on first use
+  TcMap map_vx, map_vh, map_u;
 };
 
 struct Timing {
@@ -60,7 +67,10 @@ struct lstm_approx {
   size_t cap_TB = 0;          // capacity (T*B) of the T-dependent scratch
   float* Px = nullptr;        // [T*B][4*Ks] hoisted input projection
   float* seq = nullptr;       // [T*B][H] output sequence of a lower layer
-  void* tau = nullptr;        // [max_batch][4*Ks] refinement coefficients
+  void* tau = nullptr;        // [max_batch][4*Ks] refinement coefficients (fp32, or bf16 on the tensor path)
+  void* x_bf16 = nullptr;     // [T*B][ldx of layer 0] bf16 input (tensor path)
+  void* seq_bf16 = nullptr;   // [T*B][ldh] bf16 sequence between layers (tensor path)
+  void* h_bf16 = nullptr;     // [max_batch][ldh] bf16 h operand (tensor path)
   int* err = nullptr;         // device status word (0 = ok)
 
   // staging for lstm_approx_run_host
@@ -150,8 +160,56 @@ struct PersistentArgs {
 };
 cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s);
 
+// ---- tensor-core path (bf16, tcgen05 / TMEM / TMA) -----------------------
+
+// 2-D K-major bf16 tensor [rows][inner] with `pitch_bytes` between rows, as
+// TMA tiles of 64 inner elements x box_rows rows, 128-byte swizzled.
+bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
+                 uint32_t box_rows);
+int tc_rows_tile_n(int n_cols);  // column tile of launch_tc_rows for n_cols columns
+int tc_gates_tile_n(int B);      // stream tile of launch_tc_gates
+
+struct TcRowsArgs {
+  int Kdim;          // reduction length (D of the layer, or H)
+  int K, Ks;         // refinement depth of the run; gate stride of the packed rows
+  int kt_per_gate;   // 128-row tiles per gate: ceil(K / 128)
+  int N;             // valid columns (T*B for the projection, B for tau')
+  int mode;          // 0: P[n][row] = sum; 1: tau[n][row] = bf16(sigma[row] (sum + P[n][row])), 0 for k >= K
+  float* P;          // [N][ldp]
+  int ldp;
+  const float* sigma;
+  __nv_bfloat16* tau;  // [N][ldt]
+  int ldt;
+  int* err;
+  long long limit_ns;
+};
+cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s);
+
+struct TcGatesArgs {
+  int H, K, Ks, B;
+  int nkb;                  // 64-term chunks: ceil(K / 64)
+  const float* bias;        // [4][H]
+  float* c_state;           // [B][H] fp32, c_{t-1} in, c_t out
+  __nv_bfloat16* h_bf16;    // [B][ldh] h_t out (next step's operand)
+  int ldh;
+  float* out_h;             // [B][H] fp32 h_t (this timestep) or null
+  __nv_bfloat16* seq_bf16;  // [B][ldh] h_t for the next layer (this timestep) or null
+  Checkpoints ck;           // depths, multiples of 16
+  float* ckpt_h;            // element (j, n, unit) at j*ck_stride + n*H + unit (this timestep) or null
+  float* ckpt_c;
+  long long ck_stride;
+  int* err;
+  long long limit_ns;
+};
+cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s);
+
+cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s);
+cudaError_t launch_tc_init_state(const float* h0, const float* c0, int B, int H, __nv_bfloat16* h_bf16, int ldh,
+                                 float* c_state, cudaStream_t s);
+
 // ---- error codes written to the device status word -----------------------
 constexpr int kErrWaitTimeoutA = 1;
 constexpr int kErrWaitTimeoutB = 2;
+constexpr int kErrTcTimeout = 3;
 
 }  // namespace lstm_approx_impl

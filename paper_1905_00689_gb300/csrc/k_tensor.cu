@@ -1,0 +1,459 @@
+// Large-batch tensor-core path (bf16 factors and operands, fp32 accumulate).
+//
+// The two products of one timestep are dense contractions over B streams:
+//   (a2) tau'[n][(g,k)] = sigma_{g,k} (P_t[n][(g,k)] + sum_j Vh[(g,k)][j] h_{t-1}[n][j])
+//   (a3) y_g[n][j]      = sum_k U_g[j][k] tau'[n][(g,k)]
+// and the hoisted input projection (a1) is the first one with x in place of
+// h over all T*B columns (Eq. 1 with the augmentation of Sec. III).
+//
+// tc_rows_kernel computes one 128-row x BN-column tile of the first kind:
+// warp 0 streams K-major tiles of both operands with TMA (128-byte swizzle)
+// through an S-stage mbarrier ring, one thread of warp 1 issues
+// tcgen05.mma (M = 128, N = BN, K = 16 per instruction) into a tensor-memory
+// accumulator, and warps 4..7 read the accumulator back with tcgen05.ld for
+// the epilogue (store P, or form tau' in bf16).
+//
+// tc_gates_kernel computes, for 128 hidden units x NT streams, the four gate
+// sums at once in four tensor-memory accumulators and runs the cell update
+// of Sec. II in the epilogue.  Intermediate depths k_j (multiples of 16) are
+// read from the same accumulators when the MMA stream reaches them: the MMA
+// thread commits, the epilogue warps compute the cell from the partial sums
+// and hand the accumulators back -- no prefix is recomputed.
+//
+// Every mbarrier wait is bounded in wall time; a wait that runs out writes
+// the device status word, the CTA stops issuing work, waits (bounded) for
+// its copies and MMAs in flight, frees its tensor memory and returns.
+#include <cuda.h>
+
+#include <cstring>
+#include <mutex>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace lstm_approx_impl {
+namespace {
+
+using namespace lstm_approx_dev;
+
+constexpr int kTcThreads = 256;
+constexpr int kTileM = 128;
+constexpr int kTileK = 64;  // bf16 elements in one 128-byte swizzled row
+constexpr uint32_t kABytes = kTileM * kTileK * 2;
+
+__device__ __forceinline__ bool wait_cta(uint32_t mb, uint32_t parity, uint64_t limit, const volatile int* err) {
+  return mbar_wait_bounded<false>(mb, parity, limit, err);
+}
+
+// ---------------------------------------------------------------------------
+// tile of tau' / P: rows of the packed factor matrix x columns (streams)
+// ---------------------------------------------------------------------------
+template <int BN, int S>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_rows_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, TcRowsArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  constexpr uint32_t kBBytes = BN * kTileK * 2;
+  constexpr uint32_t kCols = BN < 32 ? 32 : BN;
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t sA = base, sB = base + S * kABytes;
+  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | tmem slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 2));
+  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = blockIdx.x / a.kt_per_gate, kt = blockIdx.x % a.kt_per_gate;
+  const int row0 = g * a.Ks + kt * kTileM;
+  const int col0 = blockIdx.y * BN;
+  const int nkb = (a.Kdim + kTileK - 1) / kTileK;
+  const volatile int* err = a.err;
+  const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(bar0 + 8u * i, 1);
+      mbar_init(bar0 + 8u * (S + i), 1);
+    }
+    mbar_init(accum_bar, 1);
+    mbar_init(drain_bar, 1);
+    fence_mbarrier_init_cluster();
+  }
+  if (warp == 2) {
+    tmem_alloc(smem_u32(tmem_slot), kCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {  // ---- TMA producer ----
+    tma_prefetch_map(&tma);
+    tma_prefetch_map(&tmb);
+    int issued = 0;
+    bool ok = true;
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % S;
+      if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
+      mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
+      tma_load_2d(sA + s * kABytes, &tma, bar0 + 8u * s, kb * kTileK, row0);
+      tma_load_2d(sB + s * kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
+      ++issued;
+    }
+    if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
+    // every issued copy has landed before the CTA may leave
+    for (int s = 0; s < S && s < issued; ++s) {
+      const int last = s + ((issued - 1 - s) / S) * S;
+      wait_cta(bar0 + 8u * s, (last / S) & 1, limit, err);
+    }
+  } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
+    constexpr uint32_t idesc = umma_idesc_bf16(kTileM, BN);
+    bool ok = true;
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % S;
+      if (!(ok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
+      tc_fence_after();
+      const uint64_t da = umma_desc_sw128(sA + s * kABytes);
+      const uint64_t db = umma_desc_sw128(sB + s * kBBytes);
+#pragma unroll
+      for (int kk = 0; kk < kTileK / 16; ++kk)
+        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+      umma_commit(bar0 + 8u * (S + s));  // frees the stage once these MMAs are done
+    }
+    if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
+    umma_commit(accum_bar);
+    umma_commit(drain_bar);
+    wait_cta(drain_bar, 0, limit, err);
+  } else if (warp >= 4) {  // ---- epilogue ----
+    const int q = warp - 4;
+    const bool ok = wait_cta(accum_bar, 0, limit, err);
+    tc_fence_after();
+    const int lrow = 32 * q + lane;
+    const int k = kt * kTileM + lrow;
+    const int row = row0 + lrow;
+    const bool row_ok = k < a.K;
+    const float sig = (a.mode == 1 && row_ok) ? a.sigma[row] : 0.f;
+    const bool write = ok && *err == 0;
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16];
+      tmem_ld16(tmem + ((32u * q) << 16) + c0, v);
+      tmem_wait_ld();
+      if (!write) continue;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int n = col0 + c0 + j;
+        if (n >= a.N) break;
+        if (a.mode == 0) {
+          if (row_ok) a.P[(long long)n * a.ldp + row] = v[j];
+        } else {
+          const float t = row_ok ? sig * (v[j] + a.P[(long long)n * a.ldp + row]) : 0.f;
+          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(t);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kCols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// four gate sums for 128 units x NT streams, cell update in the epilogue
+// ---------------------------------------------------------------------------
+template <int NT, int S>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_gates_kernel(const __grid_constant__ CUtensorMap tmu, const __grid_constant__ CUtensorMap tmt, TcGatesArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  constexpr uint32_t kBBytes = NT * kTileK * 2;
+  constexpr uint32_t kCols = 4 * NT < 32 ? 32 : 4 * NT;
+  static_assert(S >= 4, "a chunk of all four gates must be resident");
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  const uint32_t sA = base, sB = base + S * kABytes;
+  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | ckpt | ckpt_done | slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 4));
+  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
+  const uint32_t ckpt_bar = accum_bar + 16u, ckpt_done = accum_bar + 24u;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j0 = blockIdx.x * kTileM;
+  const int n0 = blockIdx.y * NT;
+  const int nkb = a.nkb;
+  const int J = a.ck.n;
+  const volatile int* err = a.err;
+  const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(bar0 + 8u * i, 1);
+      mbar_init(bar0 + 8u * (S + i), 1);
+    }
+    mbar_init(accum_bar, 1);
+    mbar_init(drain_bar, 1);
+    mbar_init(ckpt_bar, 1);
+    mbar_init(ckpt_done, 4 * 32);
+    fence_mbarrier_init_cluster();
+  }
+  if (warp == 2) {
+    tmem_alloc(smem_u32(tmem_slot), kCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {  // ---- TMA producer: stage i = (chunk i/4, gate i%4) ----
+    tma_prefetch_map(&tmu);
+    tma_prefetch_map(&tmt);
+    const int nst = 4 * nkb;
+    int issued = 0;
+    bool ok = true;
+    for (int i = 0; i < nst; ++i) {
+      const int s = i % S, kb = i >> 2, g = i & 3;
+      if (i >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((i / S) - 1) & 1, limit, err))) break;
+      mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
+      tma_load_2d(sA + s * kABytes, &tmu, bar0 + 8u * s, kb * kTileK, g * a.H + j0);
+      tma_load_2d(sB + s * kBBytes, &tmt, bar0 + 8u * s, g * a.Ks + kb * kTileK, n0);
+      ++issued;
+    }
+    if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
+    for (int s = 0; s < S && s < issued; ++s) {
+      const int last = s + ((issued - 1 - s) / S) * S;
+      wait_cta(bar0 + 8u * s, (last / S) & 1, limit, err);
+    }
+  } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
+    constexpr uint32_t idesc = umma_idesc_bf16(kTileM, NT);
+    bool ok = true;
+    int jj = 0;
+    for (int kb = 0; kb < nkb && ok; ++kb) {
+      uint64_t da[4], db[4];
+      for (int g = 0; g < 4 && ok; ++g) {
+        const int i = 4 * kb + g, s = i % S;
+        ok = wait_cta(bar0 + 8u * s, (i / S) & 1, limit, err);
+        da[g] = umma_desc_sw128(sA + s * kABytes);
+        db[g] = umma_desc_sw128(sB + s * kBBytes);
+      }
+      if (!ok) break;
+      tc_fence_after();
+      // 16-term slices of this chunk, cut where an intermediate depth ends
+      int kk0 = 0;
+      while (kk0 < 4 && ok) {
+        int kk1 = 4;
+        const bool cut_here = jj < J && a.ck.k[jj] <= (kb + 1) * kTileK;
+        if (cut_here) kk1 = (a.ck.k[jj] - kb * kTileK) / 16;
+        for (int g = 0; g < 4; ++g)
+          for (int kk = kk0; kk < kk1; ++kk)
+            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, db[g] + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        if (cut_here) {  // partial sums up to depth k_jj are complete: hand them to the epilogue
+          umma_commit(ckpt_bar);
+          ok = wait_cta(ckpt_done, jj & 1, limit, err);
+          tc_fence_after();
+          ++jj;
+        }
+        kk0 = kk1;
+      }
+      for (int g = 0; g < 4; ++g) umma_commit(bar0 + 8u * (S + (4 * kb + g) % S));
+    }
+    if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
+    while (jj < J) {  // release epilogue warps still waiting for a depth (abort only)
+      umma_commit(ckpt_bar);
+      wait_cta(ckpt_done, jj & 1, limit, err);
+      ++jj;
+    }
+    umma_commit(accum_bar);
+    umma_commit(drain_bar);
+    wait_cta(drain_bar, 0, limit, err);
+  } else if (warp >= 4) {  // ---- epilogue: cell update of Sec. II ----
+    const int q = warp - 4;
+    const int j = j0 + 32 * q + lane;  // hidden unit of this thread
+    const bool unit_ok = j < a.H;
+    float bias[4] = {0.f, 0.f, 0.f, 0.f};
+    if (unit_ok)
+#pragma unroll
+      for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
+    const uint32_t trow = tmem + ((32u * q) << 16);
+    for (int step = 0; step <= J; ++step) {
+      const bool final_sums = step == J;
+      const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)(step & 1), limit, err);
+      tc_fence_after();
+      const bool write = ok && *err == 0 && unit_ok;
+      for (int c0 = 0; c0 < NT; c0 += 16) {
+        float y[4][16];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
+        tmem_wait_ld();
+        if (!write) continue;
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int n = n0 + c0 + c;
+          if (n >= a.B) break;
+          const long long sj = (long long)n * a.H + j;
+          float hh, cc;
+          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], a.c_state[sj],
+                      hh, cc);
+          if (!final_sums) {
+            const long long o = (long long)step * a.ck_stride + sj;
+            if (a.ckpt_h) a.ckpt_h[o] = hh;
+            if (a.ckpt_c) a.ckpt_c[o] = cc;
+          } else {
+            a.c_state[sj] = cc;
+            if (a.out_h) a.out_h[sj] = hh;
+            const __nv_bfloat16 hb = __float2bfloat16_rn(hh);
+            a.h_bf16[(long long)n * a.ldh + j] = hb;
+            if (a.seq_bf16) a.seq_bf16[(long long)n * a.ldh + j] = hb;
+          }
+        }
+      }
+      if (!final_sums) {
+        tc_fence_before();
+        mbar_arrive(ckpt_done);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kCols);
+  }
+}
+
+// x (fp32 [N][D]) -> bf16 [N][ld] with zero columns D..ld-1
+__global__ void to_bf16_kernel(const float* __restrict__ x, int N, int D, __nv_bfloat16* __restrict__ out, int ld) {
+  const long long total = (long long)N * ld;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long n = i / ld;
+    const int d = (int)(i % ld);
+    out[i] = __float2bfloat16_rn(d < D ? x[n * D + d] : 0.f);
+  }
+}
+
+// initial state of the tensor path: h0 -> bf16 operand, c0 -> fp32 state
+__global__ void tc_init_state_kernel(const float* __restrict__ h0, const float* __restrict__ c0, int B, int H,
+                                     __nv_bfloat16* __restrict__ h_bf16, int ldh, float* __restrict__ c_state) {
+  const long long total = (long long)B * ldh;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long n = i / ldh;
+    const int j = (int)(i % ldh);
+    h_bf16[i] = __float2bfloat16_rn((h0 != nullptr && j < H) ? h0[n * H + j] : 0.f);
+    if (j < H) c_state[n * H + j] = c0 != nullptr ? c0[n * H + j] : 0.f;
+  }
+}
+
+// ---- host side -------------------------------------------------------------
+
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encoder() {
+  static EncodeTiled fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiled>(p);
+  });
+  return fn;
+}
+
+template <int BN, int S>
+size_t rows_smem() {
+  return 1024 + S * (kABytes + BN * kTileK * 2) + 8 * (2 * S + 2) + 16;
+}
+template <int NT, int S>
+size_t gates_smem() {
+  return 1024 + S * (kABytes + NT * kTileK * 2) + 8 * (2 * S + 4) + 16;
+}
+
+template <int BN, int S>
+cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
+  auto kern = tc_rows_kernel<BN, S>;
+  static thread_local bool attr = false;
+  const size_t smem = rows_smem<BN, S>();
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid(4 * a.kt_per_gate, (n_cols + BN - 1) / BN);
+  kern<<<grid, kTcThreads, smem, s>>>(*reinterpret_cast<const CUtensorMap*>(A.bytes),
+                                      *reinterpret_cast<const CUtensorMap*>(Bm.bytes), a);
+  return cudaGetLastError();
+}
+
+template <int NT, int S>
+cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s) {
+  auto kern = tc_gates_kernel<NT, S>;
+  static thread_local bool attr = false;
+  const size_t smem = gates_smem<NT, S>();
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  dim3 grid((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT);
+  kern<<<grid, kTcThreads, smem, s>>>(*reinterpret_cast<const CUtensorMap*>(U.bytes),
+                                      *reinterpret_cast<const CUtensorMap*>(Tau.bytes), a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes, uint32_t box_rows) {
+  static_assert(sizeof(CUtensorMap) <= sizeof(m->bytes), "tensor map storage");
+  EncodeTiled enc = encoder();
+  if (!enc) return false;
+  std::memset(m->bytes, 0, sizeof(m->bytes));
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {pitch_bytes};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(reinterpret_cast<CUtensorMap*>(m->bytes), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                         const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int tc_rows_tile_n(int n_cols) { return n_cols >= 256 ? 256 : n_cols > 64 ? 128 : 64; }
+int tc_gates_tile_n(int B) { return B >= 128 ? 128 : 64; }
+
+cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
+  switch (tc_rows_tile_n(n_cols)) {
+    case 256: return launch_rows_t<256, 4>(A, Bm, a, n_cols, s);
+    case 128: return launch_rows_t<128, 6>(A, Bm, a, n_cols, s);
+    default: return launch_rows_t<64, 8>(A, Bm, a, n_cols, s);
+  }
+}
+
+cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s) {
+  if (tc_gates_tile_n(a.B) == 128) return launch_gates_t<128, 6>(U, Tau, a, s);
+  return launch_gates_t<64, 8>(U, Tau, a, s);
+}
+
+cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s) {
+  const long long total = (long long)N * ld;
+  const int blocks = (int)std::min<long long>((total + 255) / 256, 152LL * 16);
+  to_bf16_kernel<<<blocks, 256, 0, s>>>(x, N, D, out, ld);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tc_init_state(const float* h0, const float* c0, int B, int H, __nv_bfloat16* h_bf16, int ldh,
+                                 float* c_state, cudaStream_t s) {
+  const long long total = (long long)B * ldh;
+  const int blocks = (int)std::min<long long>((total + 255) / 256, 152LL * 16);
+  tc_init_state_kernel<<<blocks, 256, 0, s>>>(h0, c0, B, H, h_bf16, ldh, c_state);
+  return cudaGetLastError();
+}
+
+}  // namespace lstm_approx_impl

@@ -90,11 +90,18 @@ size_t layer_bytes_vx(const lstm_approx_t* h, const LayerStore& s) {
 size_t layer_bytes_vh(const lstm_approx_t* h) { return 4ull * h->Ks * h->ldh * elem_size(h->dtype); }
 size_t layer_bytes_u(const lstm_approx_t* h) { return 4ull * h->Ks * h->H * elem_size(h->dtype); }
 
+size_t xbf16_bytes(const lstm_approx_t* h, size_t TB) { return TB * (size_t)h->layers[0].ldx * 2; }
+size_t seqbf16_bytes(const lstm_approx_t* h, size_t TB) { return TB * (size_t)h->ldh * 2; }
+
 void free_scratch(lstm_approx_t* h) {
   dfree(h, h->Px, h->cap_TB * 4ull * h->Ks * sizeof(float));
   dfree(h, h->seq, h->cap_TB * (size_t)h->H * sizeof(float));
+  if (h->x_bf16) dfree(h, h->x_bf16, xbf16_bytes(h, h->cap_TB));
+  if (h->seq_bf16) dfree(h, h->seq_bf16, seqbf16_bytes(h, h->cap_TB));
   h->Px = nullptr;
   h->seq = nullptr;
+  h->x_bf16 = nullptr;
+  h->seq_bf16 = nullptr;
   h->cap_TB = 0;
 }
 
@@ -107,6 +114,14 @@ int ensure_scratch(lstm_approx_t* h, size_t TB) {
   if (h->L > 1) {
     rc = dmalloc(h, reinterpret_cast<void**>(&h->seq), TB * (size_t)h->H * sizeof(float), "scratch seq");
     if (rc) return rc;
+  }
+  if (h->dtype == LSTM_APPROX_BF16) {
+    rc = dmalloc(h, &h->x_bf16, xbf16_bytes(h, TB), "scratch x bf16");
+    if (rc) return rc;
+    if (h->L > 1) {
+      rc = dmalloc(h, &h->seq_bf16, seqbf16_bytes(h, TB), "scratch seq bf16");
+      if (rc) return rc;
+    }
   }
   h->cap_TB = TB;
   return LSTM_APPROX_OK;
@@ -162,6 +177,122 @@ void clear_timing(lstm_approx_t* h) {
   h->timing.phase.clear();
 }
 
+// The tensor path takes bf16 factors; its intermediate depths must fall on
+// the 16-term slices of one MMA instruction.
+bool tensor_path_fits(const lstm_approx_t* h, const Checkpoints& ck) {
+  if (h->dtype != LSTM_APPROX_BF16) return false;
+  for (int j = 0; j < ck.n; ++j)
+    if (ck.k[j] % 16 != 0) return false;
+  return true;
+}
+
+int ensure_factor_maps(lstm_approx_t* h, int l) {
+  LayerStore& s = h->layers[l];
+  if (s.maps_ready) return LSTM_APPROX_OK;
+  const uint64_t rows = 4ull * h->Ks;
+  if (!tc_make_map(&s.map_vx, s.Vx, s.D, rows, (uint64_t)s.ldx * 2, 128) ||
+      !tc_make_map(&s.map_vh, s.Vh, h->H, rows, (uint64_t)h->ldh * 2, 128) ||
+      !tc_make_map(&s.map_u, s.U, h->Ks, 4ull * h->H, (uint64_t)h->Ks * 2, 128))
+    return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for layer %d factors", l);
+  s.maps_ready = true;
+  return LSTM_APPROX_OK;
+}
+
+// One layer on the tensor cores: bf16 input -> (a1) projection -> T x
+// [(a2) tau' tile GEMM, (a3, a4, a6) four-gate GEMM with the cell epilogue].
+int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int K, const float* h0,
+                     const float* c0, float* out_h, float* out_c, const Checkpoints& ck, float* ckpt_h,
+                     float* ckpt_c) {
+  LayerStore& s = h->layers[l];
+  const int H = h->H, D = s.D, TB = T * B;
+  const long long ldp = 4LL * h->Ks;
+  int rc = ensure_factor_maps(h, l);
+  if (rc) return rc;
+  const bool top = l == h->L - 1;
+  const long long limit_ns = h->opt_wait_limit_us * 1000LL;
+  __nv_bfloat16* in_bf16;
+  int ld_in;
+  {
+    PhaseTimer pt(h, 0);
+    if (l == 0) {
+      LA_CUDA(h, launch_to_bf16(x, TB, D, static_cast<__nv_bfloat16*>(h->x_bf16), s.ldx, h->stream),
+              "input conversion launch");
+      in_bf16 = static_cast<__nv_bfloat16*>(h->x_bf16);
+      ld_in = s.ldx;
+      h->launches += 1;
+    } else {
+      in_bf16 = static_cast<__nv_bfloat16*>(h->seq_bf16);
+      ld_in = h->ldh;
+    }
+    TcMap mx;
+    if (!tc_make_map(&mx, in_bf16, D, TB, (uint64_t)ld_in * 2, tc_rows_tile_n(TB)))
+      return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
+    TcRowsArgs ra{};
+    ra.Kdim = D;
+    ra.K = K;
+    ra.Ks = h->Ks;
+    ra.kt_per_gate = (K + 127) / 128;
+    ra.N = TB;
+    ra.mode = 0;
+    ra.P = h->Px;
+    ra.ldp = (int)ldp;
+    ra.err = h->err;
+    ra.limit_ns = limit_ns;
+    LA_CUDA(h, launch_tc_rows(s.map_vx, mx, ra, TB, h->stream), "input projection launch");
+    h->launches += 1;
+  }
+  PhaseTimer pt(h, 1);
+  __nv_bfloat16* hb = static_cast<__nv_bfloat16*>(h->h_bf16);
+  __nv_bfloat16* tau = static_cast<__nv_bfloat16*>(h->tau);
+  float* cs = h->c_state + (size_t)l * h->max_batch * H;
+  LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
+  h->launches += 1;
+  TcMap mh, mt;
+  if (!tc_make_map(&mh, hb, H, B, (uint64_t)h->ldh * 2, tc_rows_tile_n(B)) ||
+      !tc_make_map(&mt, tau, ldp, B, (uint64_t)ldp * 2, tc_gates_tile_n(B)))
+    return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the state");
+  for (int t = 0; t < T; ++t) {
+    TcRowsArgs ra{};
+    ra.Kdim = H;
+    ra.K = K;
+    ra.Ks = h->Ks;
+    ra.kt_per_gate = (K + 127) / 128;
+    ra.N = B;
+    ra.mode = 1;
+    ra.P = h->Px + (size_t)t * B * ldp;
+    ra.ldp = (int)ldp;
+    ra.sigma = s.sigma;
+    ra.tau = tau;
+    ra.ldt = (int)ldp;
+    ra.err = h->err;
+    ra.limit_ns = limit_ns;
+    LA_CUDA(h, launch_tc_rows(s.map_vh, mh, ra, B, h->stream), "recurrent projection launch");
+    TcGatesArgs ga{};
+    ga.H = H;
+    ga.K = K;
+    ga.Ks = h->Ks;
+    ga.B = B;
+    ga.nkb = (K + 63) / 64;
+    ga.bias = s.bias;
+    ga.c_state = cs;
+    ga.h_bf16 = hb;
+    ga.ldh = h->ldh;
+    ga.out_h = out_h ? out_h + (size_t)t * B * H : nullptr;
+    ga.seq_bf16 = top ? nullptr : static_cast<__nv_bfloat16*>(h->seq_bf16) + (size_t)t * B * h->ldh;
+    ga.ck = ck;
+    ga.ckpt_h = ckpt_h ? ckpt_h + (size_t)t * B * H : nullptr;
+    ga.ckpt_c = ckpt_c ? ckpt_c + (size_t)t * B * H : nullptr;
+    ga.ck_stride = (long long)T * B * H;
+    ga.err = h->err;
+    ga.limit_ns = limit_ns;
+    LA_CUDA(h, launch_tc_gates(s.map_u, mt, ga, h->stream), "gate GEMM launch");
+    h->launches += 2;
+  }
+  if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, cs, (size_t)B * H * sizeof(float), cudaMemcpyDeviceToDevice, h->stream),
+                     "c copy");
+  return LSTM_APPROX_OK;
+}
+
 int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const float* h0, const float* c0,
                float* out_h, float* out_c, const Checkpoints& ck, float* ckpt_h, float* ckpt_c) {
   const int H = h->H;
@@ -184,6 +315,35 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     float* out = top ? out_h : h->seq;
     const Checkpoints none = {0, {0}};
     const Checkpoints& lck = top ? ck : none;
+    // recurrence path
+    int path = h->opt_force_path;
+    PersistentPlan plan;
+    std::string why;
+    const bool tensor_ok = bf16 && tensor_path_fits(h, lck);
+    if (path == 0) {
+      path = LSTM_APPROX_PATH_SIMT;
+      if (tensor_ok) path = LSTM_APPROX_PATH_TENSOR;
+      else if (!bf16 && B <= 8 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+        path = LSTM_APPROX_PATH_PERSISTENT;
+    } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
+      if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
+      if (!plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+        return fail(h, LSTM_APPROX_EINVAL, "persistent path unavailable: %s", why.c_str());
+    } else if (path == LSTM_APPROX_PATH_TENSOR) {
+      if (!tensor_ok)
+        return fail(h, LSTM_APPROX_EINVAL,
+                    "tensor path needs bf16 factors and intermediate depths that are multiples of 16");
+    }
+    const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
+    const float* l_c0 = c0 ? c0 + (size_t)l * B * H : nullptr;
+    float* l_cout = out_c ? out_c + (size_t)l * B * H : nullptr;
+    if (path == LSTM_APPROX_PATH_TENSOR) {
+      rc = run_layer_tensor(h, l, x, T, B, K, l_h0, l_c0, top ? out_h : nullptr, l_cout, lck,
+                            top ? ckpt_h : nullptr, top ? ckpt_c : nullptr);
+      if (rc) return rc;
+      h->last_path = path;
+      continue;
+    }
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
     {
       PhaseTimer pt(h, 0);
@@ -196,25 +356,6 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
                                  nullptr, 0, h->stream),
                 "input projection launch");
       h->launches += 1;
-    }
-    const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
-    const float* l_c0 = c0 ? c0 + (size_t)l * B * H : nullptr;
-    float* l_cout = out_c ? out_c + (size_t)l * B * H : nullptr;
-
-    // recurrence path
-    int path = h->opt_force_path;
-    PersistentPlan plan;
-    std::string why;
-    if (path == 0) {
-      path = LSTM_APPROX_PATH_SIMT;
-      if (!bf16 && B <= 8 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
-        path = LSTM_APPROX_PATH_PERSISTENT;
-    } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
-      if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
-      if (!plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
-        return fail(h, LSTM_APPROX_EINVAL, "persistent path unavailable: %s", why.c_str());
-    } else if (path == LSTM_APPROX_PATH_TENSOR) {
-      return fail(h, LSTM_APPROX_EINVAL, "tensor path not available for this shape");
     }
     PhaseTimer pt(h, 1);
     if (path == LSTM_APPROX_PATH_PERSISTENT) {
@@ -347,6 +488,8 @@ int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dim
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->c_state), state, "state");
   if (!rc) rc = dmalloc(h, &h->tau, (size_t)max_batch * 4 * h->Ks * sizeof(float), "scratch tau");
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->err), sizeof(int), "status word");
+  if (!rc && dtype == LSTM_APPROX_BF16)
+    rc = dmalloc(h, &h->h_bf16, (size_t)max_batch * h->ldh * 2, "bf16 state");
   if (rc) {
     lstm_approx_destroy(h);
     return rc;
@@ -528,6 +671,9 @@ void lstm_approx_destroy(lstm_approx_t* h) {
   cudaFree(h->tau);
   cudaFree(h->err);
   cudaFree(h->stage);
+  cudaFree(h->x_bf16);
+  cudaFree(h->seq_bf16);
+  cudaFree(h->h_bf16);
   delete h;
 }
 

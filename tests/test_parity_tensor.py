@@ -1,0 +1,101 @@
+"""GPU parity of the tensor-core path (bf16 factors and operands, fp32 accumulate).
+
+The oracle receives the factors as the library stores them (sigma fp32,
+u and v bf16); the bound 2e-2 covers the kernels' bf16 operand rounding of
+x, h and tau'.  Full-size workloads are checked on sampled streams (streams
+are independent, so the oracle runs on those streams alone).
+"""
+import numpy as np
+import pytest
+
+from parity_util import (BF16_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run, run_gpu,
+                         synthetic_layer, workload_inputs)
+from paper_1905_00689_gb300 import PATH_SIMT, PATH_TENSOR, Q_LAST_PATH
+from workloads import draw_factor_set, draw_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+def _sample(got, streams, T=None):
+    out = {"h": got["h"][:, streams]}
+    if "c_last" in got:
+        out["c_last"] = got["c_last"][:, streams]
+    for k in ("ckpt_h", "ckpt_c"):
+        if k in got:
+            out[k] = got[k][:, :, streams]
+    return out
+
+
+@pytest.mark.parametrize("D,H,T,B,K,nz,cps", [
+    (64, 128, 3, 16, 64, 96, []),            # one tile of everything
+    (40, 200, 4, 3, 80, 70, [16, 48, 80]),    # ragged H, B, K; depths inside and at the end of chunks
+    (300, 136, 2, 130, 128, 150, [64]),       # two stream tiles, ragged tail
+])
+def test_tensor_path_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
+    gates = [draw_factor_set(H, D + H, K, nz, 5100 + 7 * D + g) for g in range(4)]
+    rng = np.random.default_rng(H)
+    for g in gates:
+        g["bias"] = 0.2 * rng.standard_normal(H)
+    x = draw_inputs(T, B, D, "uniform", 66)
+    h0 = 0.3 * rng.standard_normal((1, B, H))
+    c0 = 0.3 * rng.standard_normal((1, B, H))
+    got, m = run_gpu([gates], x, K, dtype="bf16", h0=h0, c0=c0, checkpoints=cps, force_path=PATH_TENSOR)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    ref = oracle_run([gates], x, K, dtype="bf16", h0=h0, c0=c0, checkpoints=cps)
+    assert_parity(got, ref, BF16_TOL)
+
+
+def test_tensor_path_matches_cuda_core_path(cuda_device):
+    """Same factors through both bf16 paths: agreement well inside the bound."""
+    D, H, T, B, K = 96, 256, 5, 40, 96
+    gates = [draw_factor_set(H, D + H, K, 120, 5300 + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "relu", 2)
+    a, _ = run_gpu([gates], x, K, dtype="bf16", checkpoints=[32], force_path=PATH_TENSOR)
+    b, _ = run_gpu([gates], x, K, dtype="bf16", checkpoints=[32], force_path=PATH_SIMT)
+    assert_parity(a, b, BF16_TOL)
+
+
+@pytest.mark.parametrize("K", [32, 128, 512])
+def test_throughput_workload_full_size(cuda_device, K):
+    """D=1024, H=512, T=20, B=256, keep 50%: checked on sampled streams."""
+    w = WORKLOADS["c3"]
+    layers = [list(synthetic_layer("c3", 0, 512, 0.5))]
+    x = workload_inputs(w)
+    got, m = run_gpu(layers, x, K, dtype="bf16", max_rank=512)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    streams = [0, 77, 255]
+    ref = oracle_run(layers, x[:, streams], K, dtype="bf16")
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+def test_throughput_workload_decomposed_factors(cuda_device):
+    w = WORKLOADS["c3"]
+    layers = [list(decomposed_layer("c3", 0, 32, 0.5))]
+    x = workload_inputs(w, T=4, B=64)
+    got, _ = run_gpu(layers, x, 32, dtype="bf16", checkpoints=[16, 32])
+    ref = oracle_run(layers, x, 32, dtype="bf16", checkpoints=[16, 32])
+    assert_parity(got, ref, BF16_TOL)
+
+
+@pytest.mark.parametrize("keep,K", [(0.5, 128), (0.1, 512)])
+def test_large_batch_workload_full_size(cuda_device, keep, K):
+    """D=2048, H=1024, T=64, B=1024: checked on sampled streams."""
+    w = WORKLOADS["c4"]
+    layers = [list(synthetic_layer("c4", 0, K, keep))]
+    x = workload_inputs(w)
+    got, _ = run_gpu(layers, x, K, dtype="bf16", max_rank=K)
+    streams = [0, 513, 1023]
+    ref = oracle_run(layers, x[:, streams], K, dtype="bf16")
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+def test_two_layer_progressive_workload_full_size(cuda_device):
+    """2 layers, D=4096, H=2048, T=16, B=64, K=1024, outputs at 16/64/256/1024."""
+    w = WORKLOADS["c5"]
+    layers = [list(synthetic_layer("c5", l, 1024, 0.3)) for l in range(2)]
+    x = workload_inputs(w)
+    cps = list(w.checkpoints)
+    got, _ = run_gpu(layers, x, 1024, dtype="bf16", checkpoints=cps, max_rank=1024)
+    streams = [5, 63]
+    ref = oracle_run(layers, x[:, streams], 1024, dtype="bf16", checkpoints=cps)
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
