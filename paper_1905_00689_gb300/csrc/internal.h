@@ -166,8 +166,8 @@ cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& 
 // TMA tiles of 64 inner elements x box_rows rows, 128-byte swizzled.
 bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
                  uint32_t box_rows);
-int tc_rows_tile_n(int n_cols);  // column tile of launch_tc_rows for n_cols columns
-int tc_gates_tile_n(int B);      // stream tile of launch_tc_gates
+int tc_rows_tile_n(int n_cols, int row_tiles);  // column tile of launch_tc_rows
+int tc_gates_tile_n(int H, int B);               // stream tile of launch_tc_gates
 
 struct TcRowsArgs {
   int Kdim;          // reduction length (D of the layer, or H)
@@ -183,7 +183,8 @@ struct TcRowsArgs {
   int* err;
   long long limit_ns;
 };
-cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s);
+// `bn` (64, 128 or 256) must match the box rows of Bm's map.
+cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s);
 
 struct TcGatesArgs {
   int H, K, Ks, B;
@@ -201,7 +202,8 @@ struct TcGatesArgs {
   int* err;
   long long limit_ns;
 };
-cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s);
+// `nt` (32, 64 or 128) must match the box rows of Tau's map.
+cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s);
 
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s);
 cudaError_t launch_tc_init_state(const float* h0, const float* c0, int B, int H, __nv_bfloat16* h_bf16, int ldh,

@@ -10,8 +10,11 @@
 // warp 0 streams K-major tiles of both operands with TMA (128-byte swizzle)
 // through an S-stage mbarrier ring, one thread of warp 1 issues
 // tcgen05.mma (M = 128, N = BN, K = 16 per instruction) into a tensor-memory
-// accumulator, and warps 4..7 read the accumulator back with tcgen05.ld for
-// the epilogue (store P, or form tau' in bf16).
+// accumulator, and warps 4..11 (two per 32-lane quarter of tensor memory)
+// read it back with tcgen05.ld for the epilogue: store P, or form tau' in
+// bf16.  For tau' the epilogue warps first load the P_t tile and store it
+// into the accumulator with tcgen05.st while the mainloop streams, so the
+// MMAs accumulate on top of it and the epilogue reads no global memory.
 //
 // tc_gates_kernel computes, for 128 hidden units x NT streams, the four gate
 // sums at once in four tensor-memory accumulators and runs the cell update
@@ -36,7 +39,7 @@ namespace {
 
 using namespace lstm_approx_dev;
 
-constexpr int kTcThreads = 256;
+constexpr int kTcThreads = 384;  // warps 0..3: TMA, MMA, TMEM, spare; warps 4..11: epilogue
 constexpr int kTileM = 128;
 constexpr int kTileK = 64;  // bf16 elements in one 128-byte swizzled row
 constexpr uint32_t kABytes = kTileM * kTileK * 2;
@@ -57,9 +60,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   const uint32_t sA = base, sB = base + S * kABytes;
-  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | tmem slot
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 2));
-  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
+  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | pinit | tmem slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 3));
+  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u, pinit_bar = accum_bar + 16u;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.x / a.kt_per_gate, kt = blockIdx.x % a.kt_per_gate;
@@ -68,6 +71,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int nkb = (a.Kdim + kTileK - 1) / kTileK;
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
+  const bool add_p = a.mode == 1;  // accumulate on top of P_t, preloaded into tensor memory
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -76,6 +80,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
+    mbar_init(pinit_bar, 8 * 32);
     fence_mbarrier_init_cluster();
   }
   if (warp == 2) {
@@ -109,7 +114,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, BN);
     bool ok = true;
-    for (int kb = 0; kb < nkb; ++kb) {
+    if (add_p) {  // the accumulator starts from P_t
+      ok = wait_cta(pinit_bar, 0, limit, err);
+      tc_fence_after();
+    }
+    for (int kb = 0; kb < nkb && ok; ++kb) {
       const int s = kb % S;
       if (!(ok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
       tc_fence_after();
@@ -117,37 +126,59 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint64_t db = umma_desc_sw128(sB + s * kBBytes);
 #pragma unroll
       for (int kk = 0; kk < kTileK / 16; ++kk)
-        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (add_p || (kb | kk) != 0) ? 1u : 0u);
       umma_commit(bar0 + 8u * (S + s));  // frees the stage once these MMAs are done
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
     umma_commit(accum_bar);
     umma_commit(drain_bar);
     wait_cta(drain_bar, 0, limit, err);
-  } else if (warp >= 4) {  // ---- epilogue ----
-    const int q = warp - 4;
-    const bool ok = wait_cta(accum_bar, 0, limit, err);
-    tc_fence_after();
+  } else if (warp >= 4) {  // ---- epilogue: warps 4..11, two per lane quarter ----
+    const int ep = warp - 4, q = ep & 3;
+    constexpr int kHalf = BN / 2;
+    const int cbeg = (ep >> 2) * kHalf;
     const int lrow = 32 * q + lane;
     const int k = kt * kTileM + lrow;
     const int row = row0 + lrow;
     const bool row_ok = k < a.K;
-    const float sig = (a.mode == 1 && row_ok) ? a.sigma[row] : 0.f;
+    const uint32_t trow = tmem + ((32u * q) << 16);
+    if (add_p) {  // P_t of this tile -> tensor memory, while the mainloop runs
+      const float* __restrict__ P = a.P;
+#pragma unroll 1
+      for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 64) {
+        float pv[4][16];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int n = col0 + c0 + 16 * u + j;
+            pv[u][j] = (row_ok && n < a.N && c0 + 16 * u < cbeg + kHalf) ? __ldg(P + (long long)n * a.ldp + row) : 0.f;
+          }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (c0 + 16 * u < cbeg + kHalf) tmem_st16(trow + c0 + 16 * u, pv[u]);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(pinit_bar);
+    }
+    const bool ok = wait_cta(accum_bar, 0, limit, err);
+    tc_fence_after();
+    const float sig = (add_p && row_ok) ? a.sigma[row] : 0.f;
     const bool write = ok && *err == 0;
-    for (int c0 = 0; c0 < BN; c0 += 16) {
+    for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 16) {
       float v[16];
-      tmem_ld16(tmem + ((32u * q) << 16) + c0, v);
+      tmem_ld16(trow + c0, v);
       tmem_wait_ld();
       if (!write) continue;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int n = col0 + c0 + j;
         if (n >= a.N) break;
-        if (a.mode == 0) {
+        if (!add_p) {
           if (row_ok) a.P[(long long)n * a.ldp + row] = v[j];
         } else {
-          const float t = row_ok ? sig * (v[j] + a.P[(long long)n * a.ldp + row]) : 0.f;
-          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(t);
+          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(row_ok ? sig * v[j] : 0.f);
         }
       }
     }
@@ -194,7 +225,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
     mbar_init(ckpt_bar, 1);
-    mbar_init(ckpt_done, 4 * 32);
+    mbar_init(ckpt_done, 8 * 32);
     fence_mbarrier_init_cluster();
   }
   if (warp == 2) {
@@ -267,8 +298,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     umma_commit(accum_bar);
     umma_commit(drain_bar);
     wait_cta(drain_bar, 0, limit, err);
-  } else if (warp >= 4) {  // ---- epilogue: cell update of Sec. II ----
-    const int q = warp - 4;
+  } else if (warp >= 4) {  // ---- epilogue: cell update of Sec. II (warps 4..11, two per lane quarter) ----
+    const int ep = warp - 4, q = ep & 3;
+    constexpr int kHalf = NT / 2;
+    const int cbeg = (ep >> 2) * kHalf;
     const int j = j0 + 32 * q + lane;  // hidden unit of this thread
     const bool unit_ok = j < a.H;
     float bias[4] = {0.f, 0.f, 0.f, 0.f};
@@ -281,7 +314,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)(step & 1), limit, err);
       tc_fence_after();
       const bool write = ok && *err == 0 && unit_ok;
-      for (int c0 = 0; c0 < NT; c0 += 16) {
+      for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 16) {
+        float cp[16];  // c_{t-1}, loaded before any store of this chunk
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int n = n0 + c0 + c;
+          cp[c] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+        }
         float y[4][16];
 #pragma unroll
         for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
@@ -293,8 +332,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           if (n >= a.B) break;
           const long long sj = (long long)n * a.H + j;
           float hh, cc;
-          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], a.c_state[sj],
-                      hh, cc);
+          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
           if (!final_sums) {
             const long long o = (long long)step * a.ck_stride + sj;
             if (a.ckpt_h) a.ckpt_h[o] = hh;
@@ -368,7 +406,7 @@ EncodeTiled encoder() {
 
 template <int BN, int S>
 size_t rows_smem() {
-  return 1024 + S * (kABytes + BN * kTileK * 2) + 8 * (2 * S + 2) + 16;
+  return 1024 + S * (kABytes + BN * kTileK * 2) + 8 * (2 * S + 3) + 16;
 }
 template <int NT, int S>
 size_t gates_smem() {
@@ -425,20 +463,34 @@ bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint
   return r == CUDA_SUCCESS;
 }
 
-int tc_rows_tile_n(int n_cols) { return n_cols >= 256 ? 256 : n_cols > 64 ? 128 : 64; }
-int tc_gates_tile_n(int B) { return B >= 128 ? 128 : 64; }
+int tc_rows_tile_n(int n_cols, int row_tiles) {
+  // few columns (tau' over B streams): the widest tile that keeps one wave;
+  // many columns (the projection over T*B): 256
+  for (int bn : {64, 128, 256})
+    if ((long long)row_tiles * ((n_cols + bn - 1) / bn) <= 148) return bn;
+  return 256;
+}
+int tc_gates_tile_n(int H, int B) {
+  const int unit_tiles = (H + kTileM - 1) / kTileM;
+  for (int nt : {32, 64, 128})
+    if ((long long)unit_tiles * ((B + nt - 1) / nt) <= 148) return nt;
+  return 128;
+}
 
-cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
-  switch (tc_rows_tile_n(n_cols)) {
+cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s) {
+  switch (bn) {
     case 256: return launch_rows_t<256, 4>(A, Bm, a, n_cols, s);
     case 128: return launch_rows_t<128, 6>(A, Bm, a, n_cols, s);
     default: return launch_rows_t<64, 8>(A, Bm, a, n_cols, s);
   }
 }
 
-cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s) {
-  if (tc_gates_tile_n(a.B) == 128) return launch_gates_t<128, 6>(U, Tau, a, s);
-  return launch_gates_t<64, 8>(U, Tau, a, s);
+cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s) {
+  switch (nt) {
+    case 128: return launch_gates_t<128, 6>(U, Tau, a, s);
+    case 64: return launch_gates_t<64, 8>(U, Tau, a, s);
+    default: return launch_gates_t<32, 8>(U, Tau, a, s);
+  }
 }
 
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s) {

@@ -224,8 +224,10 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
       in_bf16 = static_cast<__nv_bfloat16*>(h->seq_bf16);
       ld_in = h->ldh;
     }
+    const int kt = (K + 127) / 128;
+    const int bnx = tc_rows_tile_n(TB, 4 * kt);
     TcMap mx;
-    if (!tc_make_map(&mx, in_bf16, D, TB, (uint64_t)ld_in * 2, tc_rows_tile_n(TB)))
+    if (!tc_make_map(&mx, in_bf16, D, TB, (uint64_t)ld_in * 2, bnx))
       return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
     TcRowsArgs ra{};
     ra.Kdim = D;
@@ -238,7 +240,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.ldp = (int)ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(s.map_vx, mx, ra, TB, h->stream), "input projection launch");
+    LA_CUDA(h, launch_tc_rows(s.map_vx, mx, ra, TB, bnx, h->stream), "input projection launch");
     h->launches += 1;
   }
   PhaseTimer pt(h, 1);
@@ -247,9 +249,11 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
   LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
   h->launches += 1;
+  const int bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
+  const int nt = tc_gates_tile_n(H, B);
   TcMap mh, mt;
-  if (!tc_make_map(&mh, hb, H, B, (uint64_t)h->ldh * 2, tc_rows_tile_n(B)) ||
-      !tc_make_map(&mt, tau, ldp, B, (uint64_t)ldp * 2, tc_gates_tile_n(B)))
+  if (!tc_make_map(&mh, hb, H, B, (uint64_t)h->ldh * 2, bnh) ||
+      !tc_make_map(&mt, tau, ldp, B, (uint64_t)ldp * 2, nt))
     return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the state");
   for (int t = 0; t < T; ++t) {
     TcRowsArgs ra{};
@@ -266,7 +270,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.ldt = (int)ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(s.map_vh, mh, ra, B, h->stream), "recurrent projection launch");
+    LA_CUDA(h, launch_tc_rows(s.map_vh, mh, ra, B, bnh, h->stream), "recurrent projection launch");
     TcGatesArgs ga{};
     ga.H = H;
     ga.K = K;
@@ -285,7 +289,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ga.ck_stride = (long long)T * B * H;
     ga.err = h->err;
     ga.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_gates(s.map_u, mt, ga, h->stream), "gate GEMM launch");
+    LA_CUDA(h, launch_tc_gates(s.map_u, mt, ga, nt, h->stream), "gate GEMM launch");
     h->launches += 2;
   }
   if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, cs, (size_t)B * H * sizeof(float), cudaMemcpyDeviceToDevice, h->stream),
