@@ -293,6 +293,9 @@ def run_ours(args):
                       "p50_us_per_timestep": 1e3 * med / T,
                       "effective_factor_gbs": algorithmic_bytes_per_timestep(H, C, nz, K) * T / (med / 1e3) / 1e9})
 
+    # ---- large-batch tensor-core path (bf16 factors) -------------------------
+    large = [] if (args.quick or args.no_large) else large_batch_sweep(dev, stream, peaks_bf16())
+
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
     oh = torch.empty((T, B, H), dtype=torch.float32).pin_memory()
@@ -346,6 +349,7 @@ def run_ours(args):
             "recurrence_path": {1: "simt", 2: "persistent", 3: "tensor"}.get(path, str(path)),
             "cluster_ctas": cluster,
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
+            "large_batch": large,
         }
         if ws == 1 and not (args.no_cpu_baseline or args.quick):
             line["cpu_baseline"] = cpu_baseline()
@@ -355,6 +359,94 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+LARGE_BATCH = (("c3", 0.5, 512, ()), ("c4", 0.5, 512, ()), ("c4", 0.1, 128, ()),
+               ("c5", 0.3, 1024, (16, 64, 256, 1024)))
+
+
+def peaks_bf16():
+    try:
+        pk = json.load(open(os.path.join(HERE, "MEASURED_PEAKS.json")))
+        return float(pk["bf16_tflops"]), "measured (MEASURED_PEAKS.json bf16_tflops)"
+    except (OSError, ValueError, KeyError):
+        return 1900.0, "fallback 1900 TFLOP/s"
+
+
+def large_batch_sweep(dev, stream, peak):
+    """The bf16 workloads on the tensor-core path: throughput, and the hoisted
+    input projection (the large dense contraction) against the bf16 peak."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, OPT_TIMING, Q_LAST_PATH
+    peak_tf, peak_src = peak
+    out = []
+    for name, keep, K, cps in LARGE_BATCH:
+        w = WORKLOADS[name]
+        m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, K, w.B, "bf16", stream=stream)
+        for l in range(w.L):
+            m.set_layer(l, synthetic_layer_factors(w, l, K, keep))
+        x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+        oh = torch.empty((w.T, w.B, w.H), device=dev)
+        ck = torch.empty((max(1, len(cps)), w.T, w.B, w.H), device=dev)
+        run = lambda: m.run(x, K, oh, checkpoints=list(cps), ckpt_h=ck if cps else None)
+        for _ in range(3):
+            run()
+        m.sync()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+        for a, b in evs:
+            a.record(stream)
+            run()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+        m.set_option(OPT_TIMING, 1)
+        ph = []
+        for _ in range(5):
+            run()
+            ph.append(m.phase_times())
+        m.set_option(OPT_TIMING, 0)
+        xp_ms = statistics.median(p[0] for p in ph)
+        exec_fl = sum(w.T * w.B * (2 * 4 * K * w.C(l) + 2 * 4 * K * w.H) for l in range(w.L))
+        xp_fl = sum(w.T * w.B * 2 * 4 * K * w.input_dim(l) for l in range(w.L))
+        xp_tf = xp_fl / (xp_ms / 1e3) / 1e12
+        out.append({
+            "workload": w.name, "keep": keep, "K": K, "checkpoints": list(cps),
+            "path": {1: "simt", 2: "persistent", 3: "tensor"}.get(m.query(Q_LAST_PATH)),
+            "ms_per_run": ms, "value": w.T * w.B / (ms / 1e3), "unit": UNIT,
+            "executed_tflops": exec_fl / (ms / 1e3) / 1e12,
+            "input_projection": {"ms": xp_ms, "tflops": xp_tf, "peak": peak_tf, "frac": xp_tf / peak_tf,
+                                 "peak_source": peak_src},
+            "recurrence_ms": statistics.median(p[1] for p in ph),
+        })
+        del m, x, oh, ck
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_profile(args):
+    """Run one workload's path `--steps` times and print a short JSON line.
+
+    Used as the target of ncu captures: c1/c2 take the fp32 persistent path,
+    c3/c4/c5 the bf16 tensor-core path, at their largest listed K.
+    """
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, Q_LAST_PATH
+    w = WORKLOADS[args.profile]
+    keep = w.keeps[0]
+    K = max(w.Ks)
+    dev = torch.device("cuda", 0)
+    m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, K, w.B, w.dtype)
+    for l in range(w.L):
+        m.set_layer(l, synthetic_layer_factors(w, l, K, keep))
+    x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+    oh = torch.empty((w.T, w.B, w.H), device=dev)
+    cps = list(w.checkpoints)
+    ck = torch.empty((max(1, len(cps)), w.T, w.B, w.H), device=dev)
+    for _ in range(args.warmup + args.steps):
+        m.run(x, K, oh, checkpoints=cps, ckpt_h=ck if cps else None)
+    m.sync()
+    print(json.dumps({"profile": w.name, "K": K, "keep": keep, "runs": args.warmup + args.steps,
+                      "path": m.query(Q_LAST_PATH)}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -362,12 +454,17 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-large", action="store_true", help="skip the large-batch tensor-core measurements")
+    ap.add_argument("--profile", choices=sorted(WORKLOADS), default=None,
+                    help="only run one workload's path (warmup + steps runs), for profilers")
     ap.add_argument("--quick", action="store_true",
                     help="main timed loop only (short side measurements, no K sweep, no CPU baseline)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
-    if args.impl == "reference":
+    if args.profile:
+        run_profile(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

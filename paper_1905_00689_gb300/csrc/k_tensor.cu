@@ -360,14 +360,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
-// x (fp32 [N][D]) -> bf16 [N][ld] with zero columns D..ld-1
+// x (fp32 [N][D]) -> bf16 [N][ld] with zero columns D..ld-1: one thread per
+// 8 output elements (one 16-byte store), vector loads when D is a multiple of 8
 __global__ void to_bf16_kernel(const float* __restrict__ x, int N, int D, __nv_bfloat16* __restrict__ out, int ld) {
-  const long long total = (long long)N * ld;
+  const int c8 = ld >> 3;  // 8-element chunks per output row (ld is a multiple of 8)
+  const long long total = (long long)N * c8;
+  const bool vec = (D & 7) == 0;
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
        i += (long long)gridDim.x * blockDim.x) {
-    const long long n = i / ld;
-    const int d = (int)(i % ld);
-    out[i] = __float2bfloat16_rn(d < D ? x[n * D + d] : 0.f);
+    const int n = (int)(i / c8), d0 = (int)(i % c8) * 8;
+    float v[8];
+    if (vec && d0 + 8 <= D) {
+      const float4* src = reinterpret_cast<const float4*>(x + (long long)n * D + d0);
+      const float4 a = __ldg(src), b = __ldg(src + 1);
+      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = d0 + e < D ? __ldg(x + (long long)n * D + d0 + e) : 0.f;
+    }
+    uint4 o;
+    __nv_bfloat162 p0 = __floats2bfloat162_rn(v[0], v[1]), p1 = __floats2bfloat162_rn(v[2], v[3]),
+                    p2 = __floats2bfloat162_rn(v[4], v[5]), p3 = __floats2bfloat162_rn(v[6], v[7]);
+    o.x = *reinterpret_cast<uint32_t*>(&p0);
+    o.y = *reinterpret_cast<uint32_t*>(&p1);
+    o.z = *reinterpret_cast<uint32_t*>(&p2);
+    o.w = *reinterpret_cast<uint32_t*>(&p3);
+    reinterpret_cast<uint4*>(out)[i] = o;
   }
 }
 
@@ -494,7 +512,7 @@ cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs&
 }
 
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s) {
-  const long long total = (long long)N * ld;
+  const long long total = (long long)N * (ld >> 3);
   const int blocks = (int)std::min<long long>((total + 255) / 256, 152LL * 16);
   to_bf16_kernel<<<blocks, 256, 0, s>>>(x, N, D, out, ld);
   return cudaGetLastError();

