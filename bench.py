@@ -460,7 +460,7 @@ def main():
     ap.add_argument("--quick", action="store_true",
                     help="main timed loop only (short side measurements, no K sweep, no CPU baseline)")
     args = ap.parse_args()
-    if args.warmup < 3:
+    if args.warmup < 3 and not args.profile:
         ap.error("--warmup must be >= 3")
     if args.profile:
         run_profile(args)
