@@ -432,18 +432,20 @@ def run_profile(args):
     w = WORKLOADS[args.profile]
     keep = w.keeps[0]
     K = max(w.Ks)
+    cps = list(w.checkpoints)
+    if w.name == WL.name:  # the configuration of the main timed loop
+        keep, K, cps = KEEP, K_MAIN, list(CKPTS)
     dev = torch.device("cuda", 0)
     m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, K, w.B, w.dtype)
     for l in range(w.L):
         m.set_layer(l, synthetic_layer_factors(w, l, K, keep))
     x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
     oh = torch.empty((w.T, w.B, w.H), device=dev)
-    cps = list(w.checkpoints)
     ck = torch.empty((max(1, len(cps)), w.T, w.B, w.H), device=dev)
     for _ in range(args.warmup + args.steps):
         m.run(x, K, oh, checkpoints=cps, ckpt_h=ck if cps else None)
     m.sync()
-    print(json.dumps({"profile": w.name, "K": K, "keep": keep, "runs": args.warmup + args.steps,
+    print(json.dumps({"profile": w.name, "K": K, "keep": keep, "checkpoints": cps, "runs": args.warmup + args.steps,
                       "path": m.query(Q_LAST_PATH)}), flush=True)
 
 

@@ -130,8 +130,8 @@ cudaError_t launch_cell_step(const CellArgs& a, cudaStream_t s);
 struct PersistentPlan {
   int CS = 0;        // CTAs per cluster
   int RA = 0;        // coefficient rows per CTA (multiple of 4)
-  int UB = 0;        // hidden units per CTA (16 * upl)
-  int upl = 0;       // hidden units per warp (1, 2 or 4)
+  int UB = 0;        // hidden units per CTA (ceil(H / CS) rounded up to 4)
+  int upl = 0;       // hidden units per warp (1, 2, 4, 8 or 16; four warps per gate)
   int kpw = 0;       // refinement terms per lane (1, 2, 4 or 8)
   size_t smem = 0;   // dynamic shared memory bytes
 };

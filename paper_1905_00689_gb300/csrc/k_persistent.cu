@@ -14,23 +14,30 @@
 //            tau' = sigma * (V_h h + P_t) for a group of rows is pushed into
 //            every CTA's tau buffer with one 16-byte st.async per CTA, which
 //            completes the transaction count of the receiver's mbarrier.
-//   phase B  CTA c owns UB = 16 * UPW hidden units, warp w the UPW units
-//            w*UPW + i.  The warp's slice of U (UPW units x 4 gates x K terms)
-//            lives in registers for the whole launch, lane l holding terms
-//            [l*KPL, (l+1)*KPL).  The 4*UPW gate sums are reduced across the
-//            lanes with a transposed butterfly, the cell update runs on lane i
-//            for unit i (which keeps c_t in a register), and h_t is pushed to
-//            every CTA like tau.  Outputs at the intermediate depths k_j are
-//            computed after h_t has left, off the critical path, from masked
-//            sums over the same registers.
+//   phase B  CTA c owns UBv hidden units in four blocks of UW; warp w
+//            serves gate w & 3 of unit block w >> 2, lane l the terms
+//            [l*KT, (l+1)*KT).  The warp's slice of U (UW units x 32*KT terms
+//            of one gate) lives in registers for the whole launch, so a lane
+//            reads only its own KT values of tau' per step.  The UW partial
+//            sums are reduced over the lanes by a transposed butterfly that
+//            pairs neighbouring lanes first: after s steps lanes 0 .. 2^s - 1
+//            hold the sums over the terms below KT * 2^s, so the gate sums at
+//            the intermediate depths k_j of progressive inference fall out of
+//            the same reduction (depths of another form take one masked pass
+//            more).  After one block barrier thread (depth set n, unit u)
+//            runs the cell update of Sec. II from the four gate sums: set 0
+//            carries the state (c_t stays in a register), the other sets are
+//            the outputs at the intermediate depths, computed from h_{t-1} and
+//            c_{t-1} of the full-depth chain.  Warp 0 then pushes h_t to every
+//            CTA like tau.
 //
-// No block-wide barrier sits in the time loop: every warp waits on the two
-// mbarriers itself (arrival count = number of warps) and re-arms them after
-// its own wait.  Both exchanges are double-buffered by timestep parity.
-// Every wait is bounded in wall time; a warp whose wait runs out writes the
-// device status word and leaves the loop, the others notice the word and
-// leave too, and the cluster meets at one final barrier so that no CTA exits
-// while a peer may still address its shared memory.
+// Each warp waits on the exchange mbarriers itself (arrival count = number of
+// warps) and re-arms them after its own wait; the partial sums, c_{t-1} and
+// both exchanges are double-buffered by timestep parity, so the time loop
+// holds one block barrier.  Every wait is bounded in wall time; a warp whose
+// wait runs out writes the device status word, the whole CTA leaves the loop
+// at that block barrier, and the cluster meets at one final barrier so that
+// no CTA exits while a peer may still address its shared memory.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -43,33 +50,39 @@ using namespace lstm_approx_dev;
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTauSlack = 256;  // >= 32 * KPL: the widest read past the last row
+constexpr int kTauSlack = 256;  // >= 32 * KT - Kp: lane reads past the last gate's rows
 constexpr int kMaxGroupsPerWarp = 8;
 
 struct DevPlan {
-  int CS, RA, UB, Kp;
+  int CS, RA, UBv, Kp, nset;
 };
 
 struct SmemLayout {
-  uint32_t vh, tau, h, total;  // float offsets after the barriers
+  uint32_t vh, tau, h, part, cs, hsend, total;  // float offsets after the barriers
 };
 
-__host__ __device__ inline SmemLayout smem_layout(const DevPlan& p, int H) {
+// S4 = 4 * UW unit slots per CTA (the first UBv are real units).
+__host__ __device__ inline SmemLayout smem_layout(const DevPlan& p, int H, int S4) {
   SmemLayout L;
   uint32_t o = 0;
-  L.vh = o;  o += max(p.RA * H, 8 * p.UB);  // V_h slice; also the U staging area
-  L.tau = o; o += 2 * (p.CS * p.RA + kTauSlack);
-  L.h = o;   o += 2 * p.CS * p.UB;
+  L.vh = o;    o += p.RA * H;
+  L.tau = o;   o += 2 * (p.CS * p.RA + kTauSlack);
+  L.h = o;     o += 2 * p.CS * p.UBv;
+  L.part = o;  o += 2 * p.nset * 4 * S4;
+  L.cs = o;    o += 2 * S4;
+  L.hsend = o; o += S4;
   L.total = o;
   return L;
 }
-constexpr uint32_t kBarrierBytes = 64;
+constexpr uint32_t kBarrierBytes = 128;  // 5 mbarriers, then the depths k_j
 
-// Sum of NV values over the 32 lanes, transposed: after the call lane l
-// holds in v[0] the total of value index l >> (5 - log2(NV)).
+__host__ __device__ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v >> 1); }
+
+// Sum of NV values over the 32 lanes, transposed, pairing the high lane bits
+// first: after the call lane l holds in v[0] the total of value l >> (5 - log2 NV).
 template <int NV>
 __device__ __forceinline__ void butterfly_transpose(float (&v)[NV], int lane) {
-  constexpr int kSteps = NV == 32 ? 5 : NV == 16 ? 4 : NV == 8 ? 3 : NV == 4 ? 2 : NV == 2 ? 1 : 0;
+  constexpr int kSteps = ilog2(NV);
 #pragma unroll
   for (int s = 0; s < kSteps; ++s) {
     const int half = NV >> (s + 1);
@@ -86,135 +99,108 @@ __device__ __forceinline__ void butterfly_transpose(float (&v)[NV], int lane) {
   for (int mask = 16 >> kSteps; mask > 0; mask >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], mask);
 }
 
-// Terms held by a lane: slot s of lane l is term k(l, s).  Lanes take
-// interleaved 16-byte runs (4 l + 128 q + r for KPL >= 4) so that the
-// 128-bit shared-memory reads of tau' are free of bank conflicts.
-template <int KPL>
-__device__ __forceinline__ int term_of(int lane, int s) {
-  if constexpr (KPL >= 4) return 4 * lane + 128 * (s >> 2) + (s & 3);
-  else return KPL * lane + s;
-}
-
-template <int KPL>
-__device__ __forceinline__ void load_tau(const float* tau, int g, int Kp, int lane, float (&tv)[KPL]) {
-  const float* src = tau + g * Kp;
-  if constexpr (KPL >= 4) {
+// Partial gate sums of the warp's UW units over this lane's terms s < lim
+// (lim >= KT: all of them): v[i] = sum_s u[unit i][KT*lane + s] tau'[KT*lane + s].
+template <int UW, int KT>
+__device__ __forceinline__ void lane_partials(const float (&ureg)[UW][KT], const float* tau_lane, int lim,
+                                              float (&v)[UW]) {
+  float tv[KT];
+  if constexpr (KT >= 4) {
 #pragma unroll
-    for (int q = 0; q < KPL / 4; ++q) {
-      const float4 f = *reinterpret_cast<const float4*>(src + 4 * lane + 128 * q);
+    for (int q = 0; q < KT / 4; ++q) {
+      const float4 f = *reinterpret_cast<const float4*>(tau_lane + 4 * q);
       tv[4 * q] = f.x; tv[4 * q + 1] = f.y; tv[4 * q + 2] = f.z; tv[4 * q + 3] = f.w;
     }
-  } else if constexpr (KPL == 2) {
-    const float2 f = *reinterpret_cast<const float2*>(src + 2 * lane);
+  } else if constexpr (KT == 2) {
+    const float2 f = *reinterpret_cast<const float2*>(tau_lane);
     tv[0] = f.x; tv[1] = f.y;
   } else {
-    tv[0] = src[lane];
+    tv[0] = tau_lane[0];
+  }
+#pragma unroll
+  for (int s = 0; s < KT; ++s) tv[s] = s < lim ? tv[s] : 0.f;
+#pragma unroll
+  for (int i = 0; i < UW; ++i) {
+    float acc = 0.f;
+#pragma unroll
+    for (int s = 0; s < KT; ++s) acc = fmaf(ureg[i][s], tv[s], acc);
+    v[i] = acc;
   }
 }
 
-// Partial gate sums of the warp's units over this lane's terms for NS depth
-// cut-offs at once (set 0 = the full depth K; sets 1.. = intermediate depths):
-// v[n][i*4 + g] = sum over the lane's terms k < cut[n] of u_{g,k}[unit i] tau'_{g,k}.
-// The lane's terms come in runs of G = min(KPL, 4) consecutive terms; one
-// accumulator per run is kept and the depth sets are formed from the runs
-// with selects, so the FMA count does not grow with NS.  Exact when every
-// cut-off is a multiple of G (the caller checks that).
-template <int UPW, int KPL, int NS>
-__device__ __forceinline__ void gate_partials(const float (&ureg)[UPW][4][KPL], const float* tau, int Kp, int lane,
-                                              const int (&cut)[NS], float (&v)[NS][4 * UPW]) {
-  constexpr int G = KPL < 4 ? KPL : 4;
-  constexpr int NR = KPL / G;  // runs per lane
-  float acc[NR][4 * UPW];
+// Writes the values a lane holds after S steps of the neighbour-first
+// butterfly: sums over the lanes 0 .. 2^S - 1, i.e. over the terms below
+// KT * 2^S.  While S < log2 UW lane l < 2^S holds UW >> S values whose index
+// has bit-reversed l as its top S bits; afterwards lane l < UW holds value
+// bitrev(l).
+template <int UW>
+__device__ __forceinline__ void capture(const float (&v)[UW], int S, int lane, float* dst) {
+  constexpr int L = ilog2(UW);
+  if (S < L) {
+    if (lane < (1 << S)) {
+      const int base = S == 0 ? 0 : static_cast<int>(__brev(static_cast<unsigned>(lane)) >> (32 - S)) << (L - S);
 #pragma unroll
-  for (int r = 0; r < NR; ++r)
-#pragma unroll
-    for (int i = 0; i < 4 * UPW; ++i) acc[r][i] = 0.f;
-#pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    float tv[KPL];
-    load_tau<KPL>(tau, g, Kp, lane, tv);
-#pragma unroll
-    for (int s = 0; s < KPL; ++s)
-#pragma unroll
-      for (int i = 0; i < UPW; ++i) acc[s / G][i * 4 + g] = fmaf(ureg[i][g][s], tv[s], acc[s / G][i * 4 + g]);
-  }
-#pragma unroll
-  for (int n = 0; n < NS; ++n) {
-#pragma unroll
-    for (int i = 0; i < 4 * UPW; ++i) v[n][i] = 0.f;
-#pragma unroll
-    for (int r = 0; r < NR; ++r) {
-      const bool in = term_of<KPL>(lane, r * G) < cut[n];  // the whole run is below the cut-off
-#pragma unroll
-      for (int i = 0; i < 4 * UPW; ++i) v[n][i] += in ? acc[r][i] : 0.f;
+      for (int i = 0; i < UW; ++i)
+        if (i < (UW >> S)) dst[base + i] = v[i];
     }
+  } else if (lane < UW) {
+    dst[L == 0 ? 0 : static_cast<int>(__brev(static_cast<unsigned>(lane)) >> (32 - L))] = v[0];
   }
 }
 
-// Partial gate sums over this lane's terms k < kcut, term by term (any kcut).
-template <int UPW, int KPL>
-__device__ __forceinline__ void masked_partials(const float (&ureg)[UPW][4][KPL], const float* tau, int Kp, int lane,
-                                                int kcut, float (&v)[4 * UPW]) {
+// Reduces the UW partials over the 32 lanes, neighbouring lanes first, and
+// writes depth set n (bit n of cap[S]) to dst + n * set_stride after S steps.
+template <int UW>
+__device__ __forceinline__ void butterfly_depths(float (&v)[UW], int lane, const uint32_t (&cap)[6], float* dst,
+                                                 int set_stride) {
+  constexpr int L = ilog2(UW);
 #pragma unroll
-  for (int i = 0; i < 4 * UPW; ++i) v[i] = 0.f;
+  for (int S = 0; S <= 5; ++S) {
+    if (S > 0) {
+      const int m = 1 << (S - 1);  // the step that makes S
+      if (S - 1 < L) {
+        const int half = UW >> S;
+        const bool upper = (lane & m) != 0;
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    float tv[KPL];
-    load_tau<KPL>(tau, g, Kp, lane, tv);
-#pragma unroll
-    for (int s = 0; s < KPL; ++s) {
-      const float t = term_of<KPL>(lane, s) < kcut ? tv[s] : 0.f;
-#pragma unroll
-      for (int i = 0; i < UPW; ++i) v[i * 4 + g] = fmaf(ureg[i][g][s], t, v[i * 4 + g]);
+        for (int i = 0; i < UW / 2; ++i) {
+          if (i < half) {
+            const float keep = upper ? v[i + half] : v[i];
+            const float send = upper ? v[i] : v[i + half];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+          }
+        }
+      } else {
+        v[0] += __shfl_xor_sync(0xffffffffu, v[0], m);
+      }
     }
+    for (uint32_t c = cap[S]; c != 0u; c &= c - 1u) capture<UW>(v, S, lane, dst + (__ffs(c) - 1) * set_stride);
   }
 }
 
-// Reduce one set of partials over the lanes and gather: lane i < UPW gets the
-// four gate pre-activations of unit w*UPW + i in y[0..3].
-template <int UPW>
-__device__ __forceinline__ void reduce_gates(float (&v)[4 * UPW], int lane, float (&y)[4]) {
-  constexpr int NV = 4 * UPW;
-  constexpr int kShift = NV == 16 ? 1 : NV == 8 ? 2 : 3;  // 5 - log2(NV)
-  butterfly_transpose<NV>(v, lane);
-  const int src_unit = lane < UPW ? lane : 0;
-#pragma unroll
-  for (int g = 0; g < 4; ++g) y[g] = __shfl_sync(0xffffffffu, v[0], (src_unit * 4 + g) << kShift);
-}
-
-template <int UPW>
-__device__ __forceinline__ void send_h(uint32_t dst, uint32_t bar, const float (&hv)[UPW]) {
-  if constexpr (UPW == 4) {
-    st_async_v4(dst, hv[0], hv[1], hv[2], hv[3], bar);
-  } else if constexpr (UPW == 2) {
-    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(dst),
-                 "f"(hv[0]), "f"(hv[1]), "r"(bar)
-                 : "memory");
-  } else {
-    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(dst),
-                 "r"(__float_as_uint(hv[0])), "r"(bar)
-                 : "memory");
-  }
-}
-
-template <int UPW, int KPL, int NCK>
+template <int UW, int KT>
 __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs a, DevPlan p) {
+  constexpr int S4 = 4 * UW;  // unit slots per CTA
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0,1] tau, [2,3] h
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0,1] tau, [2,3] h, [4] set-up
+  int* ck_s = reinterpret_cast<int*>(smem_raw + 48);        // the intermediate depths k_j
   float* sm = reinterpret_cast<float*>(smem_raw + kBarrierBytes);
-  const SmemLayout S = smem_layout(p, a.H);
-  float* vh_s = sm + S.vh;
-  float* tau_s = sm + S.tau;
-  float* h_s = sm + S.h;
+  const SmemLayout SL = smem_layout(p, a.H, S4);
+  float* vh_s = sm + SL.vh;
+  float* tau_s = sm + SL.tau;
+  float* h_s = sm + SL.h;
+  float* part_s = sm + SL.part;    // [2][set][gate][S4] gate sums
+  float* c_s = sm + SL.cs;         // [2][S4] c_{t-1} for the intermediate-depth cells
+  float* hsend_s = sm + SL.hsend;  // [S4] h_t of this CTA's units
+  const int part_buf = p.nset * 4 * S4;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
   const int b = blockIdx.x / p.CS;  // one cluster per stream
-  const int H = a.H, K = a.K;
+  const int H = a.H, K = a.K, J = a.ck.n;
   const int tau_len = p.CS * p.RA + kTauSlack;
-  const int h_len = p.CS * p.UB;
+  const int h_len = p.CS * p.UBv;
   const uint32_t bytes_tau = p.CS * p.RA * 4u;
-  const uint32_t bytes_h = p.CS * p.UB * 4u;
+  const uint32_t bytes_h = p.CS * p.UBv * 4u;
   const uint64_t limit_ns = static_cast<uint64_t>(a.wait_limit_ns);
   const volatile int* err = a.err;
 
@@ -232,7 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   }
   __syncthreads();
   if (lane == 0) {
-    // first use of each barrier: every warp arrives once, warp 0 with the bytes
+    // first use of each exchange barrier: every warp arrives once, warp 0 with the bytes
     for (int i = 0; i < 4; ++i) {
       const uint32_t bytes = (i < 2 ? bytes_tau : bytes_h) + ((i == 0 && a.test_stall) ? 16u : 0u);
       if (warp == 0) mbar_arrive_expect_tx(smem_u32(&bars[i]), bytes);
@@ -260,50 +246,42 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   }
   const long long p_stride = 4LL * a.Ks;
 
-  // U slice in registers: unit w*UPW + i, gate g, slot s <-> term
-  // term_of(lane, s).  U is K-major ([4][H][Ks]), so a lane's terms are
-  // contiguous runs and the loads below are coalesced 128-bit reads, all
-  // issued before any is used.
-  float ureg[UPW][4][KPL];
-  float bias_r[4] = {0.f, 0.f, 0.f, 0.f};
-  float c_reg = 0.f;
-  const int my_unit = warp * UPW + (lane < UPW ? lane : 0);
-  const int my_j = rank * p.UB + my_unit;
-  const bool cell_lane = lane < UPW && my_j < H;
-  const bool u_vec = (a.Ks % 4 == 0) && ((reinterpret_cast<uintptr_t>(a.U) & 15u) == 0);
+  // U slice in registers: gate gw, unit slot ub*UW + i, term KT*lane + s.
+  // U is K-major ([4][H][Ks]), so a lane's terms are one contiguous run and
+  // the warp's reads are coalesced; all are issued before any is used.
+  const int gw = warp & 3, ub = warp >> 2;
+  const int k_lane = KT * lane;
+  float ureg[UW][KT];
+  const bool u_vec = (KT % 4 == 0) && (a.Ks % 4 == 0) && ((reinterpret_cast<uintptr_t>(a.U) & 15u) == 0);
 #pragma unroll
-  for (int i = 0; i < UPW; ++i) {
-    const int j = rank * p.UB + warp * UPW + i;
+  for (int i = 0; i < UW; ++i) {
+    const int slot = ub * UW + i;
+    const int j = rank * p.UBv + slot;
+    const bool own = slot < p.UBv && j < H;
+    const float* row = a.U + ((long long)gw * H + (own ? j : 0)) * a.Ks + k_lane;
+    if constexpr (KT >= 4) {
 #pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      const float* row = a.U + ((long long)g * H + (j < H ? j : 0)) * a.Ks;
-      if constexpr (KPL >= 4) {
-#pragma unroll
-        for (int q = 0; q < KPL / 4; ++q) {
-          const int k0 = 4 * lane + 128 * q;
-          float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (j < H && k0 < K) {
-            if (u_vec) {
-              f = __ldg(reinterpret_cast<const float4*>(row + k0));
-            } else {
-              f.x = __ldg(row + k0);
-              f.y = k0 + 1 < K ? __ldg(row + k0 + 1) : 0.f;
-              f.z = k0 + 2 < K ? __ldg(row + k0 + 2) : 0.f;
-              f.w = k0 + 3 < K ? __ldg(row + k0 + 3) : 0.f;
-            }
+      for (int q = 0; q < KT / 4; ++q) {
+        const int kq = k_lane + 4 * q;
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (own && kq < K) {
+          if (u_vec) {
+            f = __ldg(reinterpret_cast<const float4*>(row + 4 * q));
+          } else {
+            f.x = __ldg(row + 4 * q);
+            f.y = kq + 1 < K ? __ldg(row + 4 * q + 1) : 0.f;
+            f.z = kq + 2 < K ? __ldg(row + 4 * q + 2) : 0.f;
+            f.w = kq + 3 < K ? __ldg(row + 4 * q + 3) : 0.f;
           }
-          ureg[i][g][4 * q + 0] = k0 + 0 < K ? f.x : 0.f;
-          ureg[i][g][4 * q + 1] = k0 + 1 < K ? f.y : 0.f;
-          ureg[i][g][4 * q + 2] = k0 + 2 < K ? f.z : 0.f;
-          ureg[i][g][4 * q + 3] = k0 + 3 < K ? f.w : 0.f;
         }
-      } else {
-#pragma unroll
-        for (int sl = 0; sl < KPL; ++sl) {
-          const int k = term_of<KPL>(lane, sl);
-          ureg[i][g][sl] = (j < H && k < K) ? __ldg(row + k) : 0.f;
-        }
+        ureg[i][4 * q + 0] = kq + 0 < K ? f.x : 0.f;
+        ureg[i][4 * q + 1] = kq + 1 < K ? f.y : 0.f;
+        ureg[i][4 * q + 2] = kq + 2 < K ? f.z : 0.f;
+        ureg[i][4 * q + 3] = kq + 3 < K ? f.w : 0.f;
       }
+    } else {
+#pragma unroll
+      for (int s = 0; s < KT; ++s) ureg[i][s] = (own && k_lane + s < K) ? __ldg(row + s) : 0.f;
     }
   }
   // V_h rows owned by this CTA (run row gr = rank*RA + lr = g*Kp + k): one
@@ -321,16 +299,40 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       for (int c4 = 0; c4 < H4; ++c4) dst[c4] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
-  // every lane holds the bias of unit lane % UPW (the combined reduction
-  // below lets lane n*UPW + i run the cell of depth set n, unit i)
-  {
-    const int jb = rank * p.UB + warp * UPW + lane % UPW;
-    if (jb < H) {
+  // cell work: item n*S4 + u is depth set n of unit slot u; a thread takes
+  // the items tid, tid + 512, ... which all have unit slot u = tid % S4
+  const int cu = tid & (S4 - 1);
+  const int cj = rank * p.UBv + cu;
+  const bool unit_ok = cu < p.UBv && cj < H;
+  float bias_r[4] = {0.f, 0.f, 0.f, 0.f};
+  float c_reg = 0.f;  // the carried c of unit cu (threads tid < S4)
+  if (unit_ok) {
 #pragma unroll
-      for (int g = 0; g < 4; ++g) bias_r[g] = a.bias[g * H + jb];
-    }
+    for (int g = 0; g < 4; ++g) bias_r[g] = a.bias[g * H + cj];
+    if (tid < S4 && a.c0 != nullptr) c_reg = a.c0[(long long)b * H + cj];
   }
-  if (cell_lane) c_reg = a.c0 != nullptr ? a.c0[(long long)b * H + my_j] : 0.f;
+  if (tid < S4) c_s[tid] = c_reg;
+  // where each depth set leaves the butterfly: set 0 (the full depth) and
+  // every depth k_j >= K after all five steps, k_j = KT * 2^S after S steps;
+  // other depths take a masked pass of their own
+  uint32_t cap[6] = {0u, 0u, 0u, 0u, 0u, 1u};
+  uint32_t masked = 0u;
+#pragma unroll
+  for (int n = 1; n <= kMaxCheckpoints; ++n) {
+    if (n > J) break;
+    const int c = a.ck.k[n - 1];
+    if (tid == 0) ck_s[n - 1] = c;
+    bool placed = c >= K;
+    if (placed) cap[5] |= 1u << n;
+#pragma unroll
+    for (int S = 0; S < 5; ++S) {
+      if (!placed && c == (KT << S)) {
+        cap[S] |= 1u << n;
+        placed = true;
+      }
+    }
+    if (!placed) masked |= 1u << n;
+  }
   float p_cur = p_off >= 0 ? __ldg(a.P + (long long)b * p_stride + p_off) : 0.f;
 
   const bool setup_ok = __syncthreads_and(mbar_wait_bounded<false>(bar_setup, 0, limit_ns, err));
@@ -342,15 +344,9 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const uint32_t tau_base = smem_u32(tau_s);
   const uint32_t h_base = smem_u32(h_s);
 
-  // intermediate depths handled in the fused pass: the leading ones (at most
-  // NCK) that fall on a run boundary of the lanes' terms
-  int nfused = 0;
-  {
-    constexpr int G = KPL < 4 ? KPL : 4;
-    while (nfused < NCK && nfused < a.ck.n && a.ck.k[nfused] % G == 0) ++nfused;
-  }
   for (int t = 0; t < (setup_ok ? a.T : 0); ++t) {
     const int hb = t & 1;
+    int fail = 0;  // error code of a wait of this warp that ran out
     // prefetch the next step's projection for this lane's row
     const float p_next = (p_off >= 0 && t + 1 < a.T)
                              ? __ldg(a.P + ((long long)(t + 1) * a.B + b) * p_stride + p_off)
@@ -359,10 +355,8 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     if (t > 0) {
       const bool ok = mbar_wait_bounded<true>(bar_h0 + 8u * hb, ((t - 1) >> 1) & 1, limit_ns, err);
       if (!__all_sync(0xffffffffu, ok)) {
-        if (lane == 0) atomicCAS(a.err, 0, kErrWaitTimeoutB);
-        break;
-      }
-      if (lane == 0) {
+        fail = kErrWaitTimeoutB;
+      } else if (lane == 0) {
         if (warp == 0) mbar_arrive_expect_tx(bar_h0 + 8u * hb, bytes_h);
         else mbar_arrive(bar_h0 + 8u * hb);
       }
@@ -370,8 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
 
     // ---- phase A: tau' = sigma * (V_h h_{t-1} + P_t) for the owned rows ---
     const float4* h4 = reinterpret_cast<const float4*>(h_s + hb * h_len);
-    const float tpr_lane = sig_r;  // sigma of this lane's row (0 for padding rows)
-    for (int q = 0; q < kMaxGroupsPerWarp; ++q) {
+    for (int q = 0; fail == 0 && q < kMaxGroupsPerWarp; ++q) {
       const int grp = warp + kWarps * q;
       if (grp >= ngroups) break;
       const int lr0 = grp * 4;
@@ -399,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       // lane 4q + r finishes row r of group q, then the senders gather the four
       const int r = lane & 3;
       const float mine = __shfl_sync(0xffffffffu, rs[0], r << 3);
-      const float tpr = tpr_lane * (mine + p_cur);
+      const float tpr = sig_r * (mine + p_cur);
       const float t0 = __shfl_sync(0xffffffffu, tpr, 4 * q + 0);
       const float t1 = __shfl_sync(0xffffffffu, tpr, 4 * q + 1);
       const float t2 = __shfl_sync(0xffffffffu, tpr, 4 * q + 2);
@@ -411,117 +404,98 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     }
 
     // ---- wait for every CTA's tau' ----------------------------------------
-    {
+    if (fail == 0) {
       const bool ok = mbar_wait_bounded<true>(bar_tau0 + 8u * hb, (t >> 1) & 1, limit_ns, err);
       if (!__all_sync(0xffffffffu, ok)) {
-        if (lane == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
-        break;
-      }
-      if (lane == 0) {
+        fail = kErrWaitTimeoutA;
+      } else if (lane == 0) {
         if (warp == 0) mbar_arrive_expect_tx(bar_tau0 + 8u * hb, bytes_tau);
         else mbar_arrive(bar_tau0 + 8u * hb);
       }
     }
 
-    // ---- phase B: gate sums (full depth + fused intermediate depths) ------
-    const float* tau = tau_s + hb * tau_len;
-    constexpr int NS = 1 + NCK;
-    int cut[NS];
-    cut[0] = K;
-#pragma unroll
-    for (int n = 1; n < NS; ++n) cut[n] = n - 1 < nfused ? a.ck.k[n - 1] : 0;
-    float v[NS][4 * UPW];
-    gate_partials<UPW, KPL, NS>(ureg, tau, p.Kp, lane, cut, v);
-    const float c_prev = c_reg;
-    float h_new = 0.f;
-    constexpr int NT = NS * 4 * UPW;  // values to reduce over the lanes
-    if constexpr (NS > 1 && NT <= 32) {
-      // one transposed butterfly over every (depth set, unit, gate) value;
-      // lane n*UPW + i then runs the cell of set n, unit i, all in parallel
-      constexpr int P = NT <= 16 ? 16 : 32;
-      constexpr int kShiftP = P == 32 ? 0 : 1;
-      float w[P];
-#pragma unroll
-      for (int n = 0; n < NS; ++n)
-#pragma unroll
-        for (int e = 0; e < 4 * UPW; ++e) w[n * 4 * UPW + e] = v[n][e];
-#pragma unroll
-      for (int e = NT; e < P; ++e) w[e] = 0.f;
-      butterfly_transpose<P>(w, lane);
-      const int L = lane < NS * UPW ? lane : 0;
-      const int n = L / UPW, iu = L % UPW;
-      float yy[4];
-#pragma unroll
-      for (int g = 0; g < 4; ++g) yy[g] = __shfl_sync(0xffffffffu, w[0], (n * 4 * UPW + iu * 4 + g) << kShiftP);
-      const float cp = __shfl_sync(0xffffffffu, c_reg, iu);
-      const int jl = rank * p.UB + warp * UPW + iu;
-      const long long tbl = ((long long)t * a.B + b) * H + jl;
-      if (lane < NS * UPW && jl < H) {
-        float hh, cc;
-        lstm_cell_f(yy[0] + bias_r[0], yy[1] + bias_r[1], yy[2] + bias_r[2], yy[3] + bias_r[3], cp, hh, cc);
+    // ---- phase B: gate sums of this warp's (gate, unit block) -------------
+    float* pb = part_s + hb * part_buf;
+    if (fail == 0) {
+      const float* tau_lane = tau_s + hb * tau_len + gw * p.Kp + k_lane;
+      float* dst = pb + gw * S4 + ub * UW;
+      float v[UW];
+      lane_partials<UW, KT>(ureg, tau_lane, KT, v);
+      butterfly_depths<UW>(v, lane, cap, dst, 4 * S4);
+      for (uint32_t m = masked; m != 0u; m &= m - 1u) {  // depths of another form
+        const int n = __ffs(m) - 1;
+        lane_partials<UW, KT>(ureg, tau_lane, ck_s[n - 1] - k_lane, v);
+        butterfly_transpose<UW>(v, lane);
+        // lane l holds the total of value l >> (5 - log2 UW)
+        constexpr int kSh = 5 - ilog2(UW);
+        if ((lane & ((1 << kSh) - 1)) == 0) dst[n * 4 * S4 + (lane >> kSh)] = v[0];
+      }
+    }
+    // the one block barrier of the step: a wait that ran out in any warp ends
+    // the time loop for the whole CTA here
+    if (fail != 0 && lane == 0) atomicCAS(a.err, 0, fail);
+    if (__syncthreads_or(fail)) break;
+
+    // ---- the cell update (Sec. II) for every (depth set, unit) ------------
+    const long long tbo = ((long long)t * a.B + b) * H;
+    for (int item = tid; item < p.nset * S4; item += kThreads) {
+      const int n = item / S4;
+      const float* src = pb + n * 4 * S4 + cu;
+      float hh = 0.f, cc = 0.f;
+      if (unit_ok) {
+        const float c_prev = n == 0 ? c_reg : c_s[hb * S4 + cu];
+        lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3],
+                    c_prev, hh, cc);
         if (n == 0) {
           c_reg = cc;
-          h_new = hh;
-          a.out_h[tbl] = hh;
-        } else if (n - 1 < nfused) {
-          const long long o = (long long)(n - 1) * a.T * a.B * H + tbl;
+          a.out_h[tbo + cj] = hh;
+        } else {
+          const long long o = (long long)(n - 1) * a.T * a.B * H + tbo + cj;
           if (a.ckpt_h) a.ckpt_h[o] = hh;
           if (a.ckpt_c) a.ckpt_c[o] = cc;
         }
       }
-    } else {
-      float y[4];
-      reduce_gates<UPW>(v[0], lane, y);
-      if (cell_lane) {
-        float cn;
-        lstm_cell_f(y[0] + bias_r[0], y[1] + bias_r[1], y[2] + bias_r[2], y[3] + bias_r[3], c_prev, h_new, cn);
-        c_reg = cn;
-        a.out_h[((long long)t * a.B + b) * H + my_j] = h_new;
+      if (n == 0) {
+        c_s[(hb ^ 1) * S4 + cu] = c_reg;
+        hsend_s[cu] = hh;
       }
     }
-    const long long tb = ((long long)t * a.B + b) * H + my_j;
+    // ---- push h_t of this CTA's units to every CTA of the cluster ---------
     if (t + 1 < a.T) {
-      float hv[UPW];
-#pragma unroll
-      for (int i = 0; i < UPW; ++i) hv[i] = __shfl_sync(0xffffffffu, h_new, i);
-      if (lane < p.CS) {
+      bool send = false;
+      if constexpr (S4 <= 32) {
+        if (warp == 0) {
+          __syncwarp();
+          send = true;
+        }
+      } else {
+        if (tid < S4) {
+          asm volatile("bar.sync 1, %0;" ::"n"(S4) : "memory");  // the unit-slot threads of set 0
+          send = warp == 0;
+        }
+      }
+      if (send) {
         const int nb = (t + 1) & 1;
-        const uint32_t off = 4u * (nb * h_len + rank * p.UB + warp * UPW);
-        send_h<UPW>(mapa_shared(h_base + off, lane), mapa_shared(bar_h0 + 8u * nb, lane), hv);
-      }
-    }
-    // ---- intermediate depths not covered above, after h_t has left --------
-    const int first_seq = (NS > 1 && NT <= 32) ? nfused : 0;
-    for (int jj = first_seq; jj < a.ck.n; ++jj) {
-      float yk[4];
-      if (jj < nfused) {
-#pragma unroll
-        for (int n = 1; n < NS; ++n)
-          if (n - 1 == jj) reduce_gates<UPW>(v[n], lane, yk);
-      } else {  // depths beyond the fused ones: one more pass each
-        float v1[4 * UPW];
-        masked_partials<UPW, KPL>(ureg, tau, p.Kp, lane, a.ck.k[jj], v1);
-        reduce_gates<UPW>(v1, lane, yk);
-      }
-      if (cell_lane) {
-        float hh, cc;
-        lstm_cell_f(yk[0] + bias_r[0], yk[1] + bias_r[1], yk[2] + bias_r[2], yk[3] + bias_r[3], c_prev, hh, cc);
-        const long long o = (long long)jj * a.T * a.B * H + tb;
-        if (a.ckpt_h) a.ckpt_h[o] = hh;
-        if (a.ckpt_c) a.ckpt_c[o] = cc;
+        const int nchunks = p.UBv >> 2;
+        for (int m = lane; m < nchunks * p.CS; m += 32) {
+          const int qd = m / p.CS, d = m - qd * p.CS;
+          const float4 hv = *reinterpret_cast<const float4*>(hsend_s + 4 * qd);
+          const uint32_t off = 4u * (nb * h_len + rank * p.UBv + 4 * qd);
+          st_async_v4(mapa_shared(h_base + off, d), hv.x, hv.y, hv.z, hv.w, mapa_shared(bar_h0 + 8u * nb, d));
+        }
       }
     }
     p_cur = p_next;
   }
 
-  if (cell_lane && a.c_last != nullptr) a.c_last[(long long)b * H + my_j] = c_reg;
+  if (unit_ok && tid < S4 && a.c_last != nullptr) a.c_last[(long long)b * H + cj] = c_reg;
   __syncthreads();
   cluster_sync_all();  // no CTA leaves while others may still address its shared memory
 }
 
-template <int UPW, int KPL, int NCK>
+template <int UW, int KT>
 cudaError_t launch_t(const DevPlan& dp, size_t smem, const PersistentArgs& a, cudaStream_t s) {
-  auto kern = persistent_kernel<UPW, KPL, NCK>;
+  auto kern = persistent_kernel<UW, KT>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(dp.CS * a.B);
   cfg.blockDim = dim3(kThreads);
@@ -568,7 +542,6 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
                      std::string* why) {
   (void)sm_count;
   (void)T;
-  (void)ck;
   if (H % 4 != 0) {
     *why = "hidden size not a multiple of 4";
     return false;
@@ -579,8 +552,8 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
   }
   const int Kp = (K + 3) & ~3;
   const int rows = 4 * Kp;
-  int kpl = 1;
-  while (32 * kpl < K) kpl *= 2;
+  int kt = 1;  // terms per lane: the smallest power of two that covers K with 32 lanes
+  while (32 * kt < K) kt *= 2;
   const int cs_list[] = {1, 2, 4, 8, 16};
   PersistentPlan best;
   bool found = false;
@@ -589,17 +562,16 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
     PersistentPlan p;
     p.CS = cs;
     p.RA = (((rows + cs - 1) / cs) + 3) & ~3;
-    const int units = (H + cs - 1) / cs;
-    p.upl = units <= 16 ? 1 : units <= 32 ? 2 : units <= 64 ? 4 : 0;  // units per warp
-    if (p.upl == 0) continue;
-    if (p.upl * 4 * kpl > 64) continue;
+    p.UB = (((H + cs - 1) / cs) + 3) & ~3;  // units owned by a CTA, a multiple of 4
+    int uw = 1;                            // units per warp: four blocks cover UB
+    while (4 * uw < p.UB) uw *= 2;
+    if (uw > 16 || uw * kt > 64) continue;  // U registers per thread
     if ((p.RA / 4 + kWarps - 1) / kWarps > kMaxGroupsPerWarp) continue;
-    p.UB = 16 * p.upl;
-    p.kpw = kpl;
+    p.upl = uw;
+    p.kpw = kt;
     DevPlan dp{};
-    dp.CS = p.CS; dp.RA = p.RA; dp.UB = p.UB; dp.Kp = Kp;
-    const SmemLayout L = smem_layout(dp, H);
-    p.smem = kBarrierBytes + 4ull * L.total;
+    dp.CS = p.CS; dp.RA = p.RA; dp.UBv = p.UB; dp.Kp = Kp; dp.nset = 1 + ck.n;
+    p.smem = kBarrierBytes + 4ull * smem_layout(dp, H, 4 * uw).total;
     if (p.smem > 227u * 1024u) continue;
     best = p;
     found = true;
@@ -617,15 +589,15 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
 
 cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s) {
   DevPlan dp{};
-  dp.CS = plan.CS; dp.RA = plan.RA; dp.UB = plan.UB; dp.Kp = (a.K + 3) & ~3;
+  dp.CS = plan.CS; dp.RA = plan.RA; dp.UBv = plan.UB; dp.Kp = (a.K + 3) & ~3; dp.nset = 1 + a.ck.n;
   const int u = plan.upl, k = plan.kpw;
-  const bool fused = a.ck.n > 0;
-#define LA_CASE(U_, K_)                                            \
-  if (u == U_ && k == K_)                                          \
-    return fused ? launch_t<U_, K_, 2>(dp, plan.smem, a, s) : launch_t<U_, K_, 0>(dp, plan.smem, a, s);
+#define LA_CASE(U_, K_) \
+  if (u == U_ && k == K_) return launch_t<U_, K_>(dp, plan.smem, a, s);
   LA_CASE(1, 1) LA_CASE(1, 2) LA_CASE(1, 4) LA_CASE(1, 8)
   LA_CASE(2, 1) LA_CASE(2, 2) LA_CASE(2, 4) LA_CASE(2, 8)
-  LA_CASE(4, 1) LA_CASE(4, 2) LA_CASE(4, 4)
+  LA_CASE(4, 1) LA_CASE(4, 2) LA_CASE(4, 4) LA_CASE(4, 8)
+  LA_CASE(8, 1) LA_CASE(8, 2) LA_CASE(8, 4) LA_CASE(8, 8)
+  LA_CASE(16, 1) LA_CASE(16, 2) LA_CASE(16, 4)
 #undef LA_CASE
   return cudaErrorInvalidValue;
 }

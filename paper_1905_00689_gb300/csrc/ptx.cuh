@@ -115,23 +115,49 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
                : "memory");
 }
 
+// Makes a value opaque to the compiler, so that it stays in its register for
+// the rest of a persistent kernel instead of being loaded again from memory
+// where it is used.
+__device__ __forceinline__ void keep_in_register(float& v) { asm volatile("" : "+f"(v)); }
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-// Logistic function from the hardware exponential and a correctly rounded
-// reciprocal: relative error a few units in the last place of fp32.
-__device__ __forceinline__ float sigmoid_f(float z) { return __frcp_rn(1.0f + __expf(-z)); }
+// 1/x from the hardware approximation (rcp.approx: about 1 ulp; 1/inf = 0).
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// Logistic function 1 / (1 + e^-z) from the hardware exponential and
+// reciprocal: absolute error of a few 1e-7 over the whole range.
+__device__ __forceinline__ float sigmoid_f(float z) { return rcp_approx(1.0f + __expf(-z)); }
+
+// tanh z with a relative error of a few 1e-7: (1 - e) / (1 + e), e = exp(-2|z|),
+// for |z| >= 1/4, and the Taylor series of tanh to z^9 below (its first
+// omitted term, 1382 z^11 / 155925, is under 3e-9 there), which avoids the
+// cancellation of 1 - e at small |z|.
+__device__ __forceinline__ float tanh_f(float z) {
+  const float a = fabsf(z);
+  const float e = __expf(-2.0f * a);
+  const float big = copysignf((1.0f - e) * rcp_approx(1.0f + e), z);
+  const float z2 = z * z;
+  const float poly = z2 * fmaf(z2, fmaf(z2, fmaf(z2, 62.0f / 2835.0f, -17.0f / 315.0f), 2.0f / 15.0f), -1.0f / 3.0f);
+  const float small = fmaf(z, poly, z);
+  return a < 0.25f ? small : big;
+}
 
 // Gate nonlinearities and cell update (Sec. II): i, f, o sigmoid, g tanh;
 // c = f c_prev + i g; h = o tanh(c).  Pre-activations already include bias.
 __device__ __forceinline__ void lstm_cell_f(float yi, float yf, float yg, float yo, float c_prev,
                                             float& h_out, float& c_out) {
-  const float i = sigmoid_f(yi), f = sigmoid_f(yf), g = tanhf(yg), o = sigmoid_f(yo);
+  const float i = sigmoid_f(yi), f = sigmoid_f(yf), g = tanh_f(yg), o = sigmoid_f(yo);
   c_out = fmaf(f, c_prev, i * g);
-  h_out = o * tanhf(c_out);
+  h_out = o * tanh_f(c_out);
 }
 
 
