@@ -133,6 +133,8 @@ struct PersistentPlan {
   int UB = 0;        // hidden units per CTA (ceil(H / CS) rounded up to 4)
   int upl = 0;       // hidden units per warp (1, 2, 4, 8 or 16; four warps per gate)
   int kpw = 0;       // refinement terms per lane (1, 2, 4 or 8)
+  int hc = 0;        // 16-value chunks of h per lane in the recurrent product (1 or 2)
+  int tcols = 0;     // tensor-memory columns holding the CTA's V_h rows
   size_t smem = 0;   // dynamic shared memory bytes
 };
 

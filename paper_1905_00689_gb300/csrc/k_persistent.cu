@@ -4,44 +4,47 @@
 // of Sec. II) has two all-to-all dependencies: every refinement coefficient
 // tau_{g,k} = prune(v_{g,k})^T [x_t; h_{t-1}] needs all of h_{t-1}, and every
 // gate output y_g[j] = sum_k sigma_{g,k} u_{g,k}[j] tau_{g,k} needs all tau.
-// One cluster of CS CTAs (CS <= 16) serves one stream:
+// One cluster of CS CTAs (CS <= 16) serves one stream, and both halves of the
+// factors stay on chip for the whole launch:
 //
-//   phase A  CTA c owns RA coefficient rows (gate-major row g*Kp + k), in
-//            groups of four per warp.  Its rows of the pruned V_h
-//            (masked-dense, fp32) stay in shared memory for the whole launch;
-//            the x part was hoisted into P = V_x X for all t by an earlier
-//            launch and is prefetched one step ahead into registers.
-//            tau' = sigma * (V_h h + P_t) for a group of rows is pushed into
-//            every CTA's tau buffer with one 16-byte st.async per CTA, which
-//            completes the transaction count of the receiver's mbarrier.
-//   phase B  CTA c owns UBv hidden units in four blocks of UW; warp w
-//            serves gate w & 3 of unit block w >> 2, lane l the terms
-//            [l*KT, (l+1)*KT).  The warp's slice of U (UW units x 32*KT terms
-//            of one gate) lives in registers for the whole launch, so a lane
-//            reads only its own KT values of tau' per step.  The UW partial
-//            sums are reduced over the lanes by a transposed butterfly that
-//            pairs neighbouring lanes first: after s steps lanes 0 .. 2^s - 1
-//            hold the sums over the terms below KT * 2^s, so the gate sums at
-//            the intermediate depths k_j of progressive inference fall out of
-//            the same reduction (depths of another form take one masked pass
-//            more).  After one block barrier thread (depth set n, unit u)
-//            runs the cell update of Sec. II from the four gate sums: set 0
-//            carries the state (c_t stays in a register), the other sets are
-//            the outputs at the intermediate depths, computed from h_{t-1} and
-//            c_{t-1} of the full-depth chain.  Warp 0 then pushes h_t to every
-//            CTA like tau.
+//   phase A  CTA c owns RA coefficient rows (gate-major row g*Kp + k) in
+//            groups of four; warp w takes groups w, w + 16, ...  Its rows of
+//            the pruned V_h (masked-dense, fp32) stay on chip: for hidden
+//            sizes above 256 in tensor memory (HC = 1, 2), where lane l of the
+//            warp holds the four rows' values at h indices
+//            [16*HC*l, 16*HC*(l+1)) and reads them with tcgen05.ld, so the
+//            only shared-memory traffic is h itself; for smaller hidden sizes
+//            (HC = 0) in shared memory, read with 128-bit loads.  The x part was hoisted
+//            into P = V_x X for all t by an earlier launch and is prefetched
+//            one step ahead.  tau' = sigma * (V_h h + P_t) of a group is
+//            pushed into every CTA's tau buffer with one 16-byte st.async
+//            per CTA, which completes the transaction count of the
+//            receiver's mbarrier.
+//   phase B  CTA c owns UBv hidden units in four blocks of UW; warp w serves
+//            gate w & 3 of unit block w >> 2, lane l the terms
+//            [l*KT, (l+1)*KT).  The warp's slice of U lives in registers, so
+//            a lane reads only its own KT values of tau'.  The partial sums
+//            are reduced over the lanes by a transposed butterfly that pairs
+//            neighbouring lanes first: after s steps lanes 0 .. 2^s - 1 hold
+//            the sums over the terms below KT * 2^s, so the gate sums at the
+//            intermediate depths k_j of progressive inference fall out of the
+//            same reduction (depths of another form take one masked pass
+//            more).  The four warps of a unit block meet at a named barrier;
+//            the block's leader warp then runs the cell update of Sec. II for
+//            every (depth set, unit) of the block, keeping c_t of the full
+//            depth in registers (the intermediate depths use h_{t-1} and
+//            c_{t-1} of the full-depth chain), and pushes h_t of its units
+//            to every CTA like tau.
 //
 // Each warp waits on the exchange mbarriers itself (arrival count = number of
-// warps) and re-arms them after its own wait; the partial sums, c_{t-1} and
-// both exchanges are double-buffered by timestep parity, so the time loop
-// holds one block barrier.  Every wait is bounded in wall time; a warp whose
-// wait runs out writes the device status word, the whole CTA leaves the loop
-// at that block barrier, and the cluster meets at one final barrier so that
-// no CTA exits while a peer may still address its shared memory.
+// warps) and re-arms them after its own wait; the partial sums and both
+// exchanges are double-buffered by timestep parity.  Every wait is bounded in
+// wall time; a warp whose wait runs out writes the device status word and its
+// unit block leaves the loop at the block barrier, the other blocks see the
+// status word in their own waits, and the cluster meets at one final barrier
+// so that no CTA exits while a peer may still address its shared memory.
 #include "internal.h"
 #include "ptx.cuh"
-
-#include <algorithm>
 
 namespace lstm_approx_impl {
 namespace {
@@ -50,33 +53,40 @@ using namespace lstm_approx_dev;
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTauSlack = 256;  // >= 32 * KT - Kp: lane reads past the last gate's rows
-constexpr int kMaxGroupsPerWarp = 8;
+constexpr int kTauSlack = 256;          // >= 32 * KT - Kp: lane reads past the last gate's rows
+constexpr int kMaxGroupsTmem = 2;       // groups of four V_h rows per warp, V_h in tensor memory
+constexpr int kMaxGroupsSmem = 8;       // the same, V_h in shared memory
+constexpr uint32_t kHeaderBytes = 128;  // 5 mbarriers, the TMEM address, the depths k_j
+constexpr size_t kMinSmemBytes = 116 * 1024;
 
 struct DevPlan {
-  int CS, RA, UBv, Kp, nset;
+  int CS, RA, UBv, Kp, nset, tcols;
 };
 
 struct SmemLayout {
-  uint32_t vh, tau, h, part, cs, hsend, total;  // float offsets after the barriers
+  uint32_t vh, tau, h, part, total;  // float offsets after the header
 };
 
+__host__ __device__ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v >> 1); }
+
+// h buffer length: the CS * UBv received values, and at least the 32 * HL
+// values the lanes of a tensor-memory phase A read (the tail stays zero).
+__host__ __device__ inline int h_buffer_len(const DevPlan& p, int HC) {
+  const int a = p.CS * p.UBv, b = 32 * 16 * HC;
+  return a > b ? a : b;
+}
+
 // S4 = 4 * UW unit slots per CTA (the first UBv are real units).
-__host__ __device__ inline SmemLayout smem_layout(const DevPlan& p, int H, int S4) {
+__host__ __device__ inline SmemLayout smem_layout(const DevPlan& p, int H, int HC, int S4) {
   SmemLayout L;
   uint32_t o = 0;
-  L.vh = o;    o += p.RA * H;
-  L.tau = o;   o += 2 * (p.CS * p.RA + kTauSlack);
-  L.h = o;     o += 2 * p.CS * p.UBv;
-  L.part = o;  o += 2 * p.nset * 4 * S4;
-  L.cs = o;    o += 2 * S4;
-  L.hsend = o; o += S4;
+  L.vh = o;   o += HC == 0 ? p.RA * H : 0;
+  L.tau = o;  o += 2 * (p.CS * p.RA + kTauSlack);
+  L.h = o;    o += 2 * h_buffer_len(p, HC);
+  L.part = o; o += 2 * p.nset * 4 * S4;
   L.total = o;
   return L;
 }
-constexpr uint32_t kBarrierBytes = 128;  // 5 mbarriers, then the depths k_j
-
-__host__ __device__ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v >> 1); }
 
 // Sum of NV values over the 32 lanes, transposed, pairing the high lane bits
 // first: after the call lane l holds in v[0] the total of value l >> (5 - log2 NV).
@@ -125,6 +135,50 @@ __device__ __forceinline__ void lane_partials(const float (&ureg)[UW][KT], const
 #pragma unroll
     for (int s = 0; s < KT; ++s) acc = fmaf(ureg[i][s], tv[s], acc);
     v[i] = acc;
+  }
+}
+
+// The same with the warp's slice of U in tensor memory at column u_col:
+// value i*KT + s of the lane (unit i, term s) in column u_col + i*KT + s.
+template <int UW, int KT>
+__device__ __forceinline__ void lane_partials_tmem(uint32_t u_col, const float* tau_lane, int lim, float (&v)[UW]) {
+  constexpr int NV = UW * KT;
+  constexpr int NCH = (NV + 15) / 16;
+  float tv[KT];
+  if constexpr (KT >= 4) {
+#pragma unroll
+    for (int q = 0; q < KT / 4; ++q) {
+      const float4 f = *reinterpret_cast<const float4*>(tau_lane + 4 * q);
+      tv[4 * q] = f.x; tv[4 * q + 1] = f.y; tv[4 * q + 2] = f.z; tv[4 * q + 3] = f.w;
+    }
+  } else if constexpr (KT == 2) {
+    const float2 f = *reinterpret_cast<const float2*>(tau_lane);
+    tv[0] = f.x; tv[1] = f.y;
+  } else {
+    tv[0] = tau_lane[0];
+  }
+#pragma unroll
+  for (int s = 0; s < KT; ++s) tv[s] = s < lim ? tv[s] : 0.f;
+#pragma unroll
+  for (int i = 0; i < UW; ++i) v[i] = 0.f;
+#pragma unroll
+  for (int c = 0; c < NCH; c += 2) {
+    float ua[16], ub[16];
+    if (c + 1 < NCH) {
+      tmem_ld16x2_sync(u_col + 16 * c, u_col + 16 * c + 16, ua, ub);
+    } else {
+      tmem_ld16_sync(u_col + 16 * c, ua);
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int idx = 16 * c + j;
+      if (j < 16 || c + 1 < NCH) {
+        if (idx < NV) {
+          const float u = j < 16 ? ua[j] : ub[j - 16];
+          v[idx / KT] = fmaf(u, tv[idx % KT], v[idx / KT]);
+        }
+      }
+    }
   }
 }
 
@@ -177,20 +231,53 @@ __device__ __forceinline__ void butterfly_depths(float (&v)[UW], int lane, const
   }
 }
 
-template <int UW, int KT>
+// Named barrier of the `count` threads of one unit block; returns whether any
+// of them passed `pred`.
+__device__ __forceinline__ bool block_barrier_or(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+      "barrier.cta.red.or.pred q, %2, %3, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(pred ? 1u : 0u), "r"(id), "r"(count)
+      : "memory");
+  return r != 0u;
+}
+
+// One st.async of n = 1, 2 or 4 floats into (possibly remote) shared memory.
+__device__ __forceinline__ void st_async_piece(uint32_t dst, const float (&v)[4], int n, uint32_t bar) {
+  if (n == 4) {
+    st_async_v4(dst, v[0], v[1], v[2], v[3], bar);
+  } else if (n == 2) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(dst),
+                 "f"(v[0]), "f"(v[1]), "r"(bar)
+                 : "memory");
+  } else {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(dst),
+                 "r"(__float_as_uint(v[0])), "r"(bar)
+                 : "memory");
+  }
+}
+
+template <int UW, int KT, int HC>
 __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs a, DevPlan p) {
-  constexpr int S4 = 4 * UW;  // unit slots per CTA
+  constexpr int S4 = 4 * UW;              // unit slots per CTA
+  constexpr int HL = 16 * HC;             // h values per lane in a tensor-memory phase A
+  constexpr bool kTmem = HC > 0;
+  constexpr bool kUTmem = HC == 1;                     // U in tensor memory too
+  constexpr int UKC = kUTmem ? (UW * KT + 15) / 16 * 16 : 0;  // its columns per warp
+  constexpr int kMaxGroups = kTmem ? kMaxGroupsTmem : kMaxGroupsSmem;
+  constexpr int PIECE = UW < 4 ? UW : 4;  // units per h message
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0,1] tau, [2,3] h, [4] set-up
-  int* ck_s = reinterpret_cast<int*>(smem_raw + 48);        // the intermediate depths k_j
-  float* sm = reinterpret_cast<float*>(smem_raw + kBarrierBytes);
-  const SmemLayout SL = smem_layout(p, a.H, S4);
-  float* vh_s = sm + SL.vh;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);          // [0,1] tau, [2,3] h, [4] set-up
+  uint32_t* taddr_s = reinterpret_cast<uint32_t*>(smem_raw + 40);  // TMEM base address
+  int* ck_s = reinterpret_cast<int*>(smem_raw + 48);                // the intermediate depths k_j
+  float* sm = reinterpret_cast<float*>(smem_raw + kHeaderBytes);
+  const SmemLayout SL = smem_layout(p, a.H, HC, S4);
+  float* vh_s = sm + SL.vh;  // V_h rows when they live in shared memory
   float* tau_s = sm + SL.tau;
   float* h_s = sm + SL.h;
-  float* part_s = sm + SL.part;    // [2][set][gate][S4] gate sums
-  float* c_s = sm + SL.cs;         // [2][S4] c_{t-1} for the intermediate-depth cells
-  float* hsend_s = sm + SL.hsend;  // [S4] h_t of this CTA's units
+  float* part_s = sm + SL.part;  // [2][set][gate][S4] gate sums
   const int part_buf = p.nset * 4 * S4;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -198,25 +285,38 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const int b = blockIdx.x / p.CS;  // one cluster per stream
   const int H = a.H, K = a.K, J = a.ck.n;
   const int tau_len = p.CS * p.RA + kTauSlack;
-  const int h_len = p.CS * p.UBv;
+  const int h_len = h_buffer_len(p, HC);
   const uint32_t bytes_tau = p.CS * p.RA * 4u;
   const uint32_t bytes_h = p.CS * p.UBv * 4u;
   const uint64_t limit_ns = static_cast<uint64_t>(a.wait_limit_ns);
   const volatile int* err = a.err;
+  const int ngroups = p.RA >> 2;
 
-  // ---- set-up: barriers, resident factors, initial state -----------------
+  // ---- set-up: barriers, tensor memory, resident factors, initial state ---
+  const uint32_t bar_setup = smem_u32(&bars[4]);
   if (tid == 0) {
     for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&bars[i]), kWarps);
-    mbar_init(smem_u32(&bars[4]), 1);
-    int nvalid = 0;  // V_h rows of this CTA that exist (the rest is padding)
-    for (int lr = 0; lr < p.RA; ++lr) {
-      const int gr = rank * p.RA + lr;
-      nvalid += (gr / p.Kp < 4 && gr % p.Kp < K) ? 1 : 0;
+    mbar_init(bar_setup, 1);
+    if constexpr (!kTmem) {
+      int nvalid = 0;  // V_h rows of this CTA that exist (the rest is padding)
+      for (int lr = 0; lr < p.RA; ++lr) {
+        const int gr = rank * p.RA + lr;
+        nvalid += (gr / p.Kp < 4 && gr % p.Kp < K) ? 1 : 0;
+      }
+      mbar_arrive_expect_tx(bar_setup, 4u * H * nvalid);
     }
-    mbar_arrive_expect_tx(smem_u32(&bars[4]), 4u * H * nvalid);
     fence_mbarrier_init_cluster();
   }
+  if constexpr (kTmem) {
+    if (warp == 0) {
+      tmem_alloc(smem_u32(taddr_s), p.tcols);
+      tmem_relinquish();
+    }
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = kTmem ? *taddr_s : 0u;
   if (lane == 0) {
     // first use of each exchange barrier: every warp arrives once, warp 0 with the bytes
     for (int i = 0; i < 4; ++i) {
@@ -226,22 +326,69 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     }
   }
   for (int i = tid; i < 2 * tau_len; i += kThreads) tau_s[i] = 0.f;
-  for (int i = tid; i < h_len; i += kThreads)
+  for (int i = tid; i < h_len; i += kThreads) {
     h_s[i] = (a.h0 != nullptr && i < H) ? a.h0[(long long)b * H + i] : 0.f;
+    h_s[h_len + i] = 0.f;
+  }
 
-  // per-lane row data for phase A: lane 4q + r <-> row r of this warp's q-th group
-  const int ngroups = p.RA >> 2;
-  const int my_q = lane >> 2;
-  const int my_group = warp + kWarps * my_q;
-  const bool row_lane = my_q < kMaxGroupsPerWarp && my_group < ngroups;
+  // V_h rows of this CTA into tensor memory.  Thread (warp w, lane l) holds,
+  // for its groups q (group w + 16 q), the values of the group's four rows at
+  // h indices [HL*l, HL*(l+1)) in its TMEM lane 32*(w & 3) + l: h quad e4
+  // (indices HL*l + 4*e4 + i) of row r at column
+  // (w >> 2) * (G*4*HL) + q*4*HL + 16*e4 + 4*r + i, so that one 16-column
+  // load brings one h quad of all four rows.
+  const int G = (ngroups + kWarps - 1) / kWarps;
+  const uint32_t t_lane = tmem_base + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+  const uint32_t t_col0 = static_cast<uint32_t>((warp >> 2) * G * 4 * HL);
+  for (int q = 0; kTmem && q < G; ++q) {
+    const int grp = warp + kWarps * q;
+#pragma unroll
+    for (int e4 = 0; e4 < HL / 4; ++e4) {
+      const int hi = HL * lane + 4 * e4;
+      float v[16];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int gr = rank * p.RA + grp * 4 + r;
+        const int g = gr / p.Kp, k = gr % p.Kp;
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (grp < ngroups && g < 4 && k < K && hi < H)
+          f = __ldg(reinterpret_cast<const float4*>(a.Vh + ((long long)g * a.Ks + k) * a.ldh + hi));
+        v[4 * r] = f.x; v[4 * r + 1] = f.y; v[4 * r + 2] = f.z; v[4 * r + 3] = f.w;
+      }
+      tmem_st16(t_lane + t_col0 + q * 4 * HL + 16 * e4, v);
+    }
+  }
+  if constexpr (kTmem) {
+    tmem_wait_st();
+  } else {
+    // V_h rows into shared memory: one bulk copy per row, completing on the
+    // set-up barrier; padding rows are cleared with plain stores
+    for (int lr = tid; lr < p.RA; lr += kThreads) {
+      const int gr = rank * p.RA + lr;
+      const int g = gr / p.Kp, k = gr % p.Kp;
+      if (g < 4 && k < K) {
+        bulk_copy_g2s(smem_u32(vh_s + lr * H), a.Vh + ((long long)g * a.Ks + k) * a.ldh, 4u * H, bar_setup);
+      } else {
+        float4* dst = reinterpret_cast<float4*>(vh_s + lr * H);
+        for (int c4 = 0; c4 < (H >> 2); ++c4) dst[c4] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+  }
+
+  // per-lane row data for phase A: lane 8r + q (tensor memory) or lane
+  // 4q + r (shared memory) <-> row r of this warp's group q
   long long p_off = -1;  // offset of this lane's row inside one (t, b) slice of P
   float sig_r = 0.f;
-  if (row_lane) {
-    const int gr = rank * p.RA + my_group * 4 + (lane & 3);
-    const int g = gr / p.Kp, k = gr % p.Kp;
-    if (g < 4 && k < K) {
-      p_off = (long long)g * a.Ks + k;
-      sig_r = a.sigma[p_off];
+  {
+    const int q = kTmem ? (lane & 7) : (lane >> 2), r = kTmem ? (lane >> 3) : (lane & 3);
+    const int grp = warp + kWarps * q;
+    if (q < kMaxGroups && grp < ngroups) {
+      const int gr = rank * p.RA + grp * 4 + r;
+      const int g = gr / p.Kp, k = gr % p.Kp;
+      if (g < 4 && k < K) {
+        p_off = (long long)g * a.Ks + k;
+        sig_r = a.sigma[p_off];
+      }
     }
   }
   const long long p_stride = 4LL * a.Ks;
@@ -284,34 +431,37 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       for (int s = 0; s < KT; ++s) ureg[i][s] = (own && k_lane + s < K) ? __ldg(row + s) : 0.f;
     }
   }
-  // V_h rows owned by this CTA (run row gr = rank*RA + lr = g*Kp + k): one
-  // bulk copy per row into shared memory, completing on the set-up barrier;
-  // padding rows are cleared with plain stores.
-  const int H4 = H >> 2;
-  const uint32_t bar_setup = smem_u32(&bars[4]);
-  for (int lr = tid; lr < p.RA; lr += kThreads) {
-    const int gr = rank * p.RA + lr;
-    const int g = gr / p.Kp, k = gr % p.Kp;
-    if (g < 4 && k < K) {
-      bulk_copy_g2s(smem_u32(vh_s + lr * H), a.Vh + ((long long)g * a.Ks + k) * a.ldh, 4u * H, bar_setup);
-    } else {
-      float4* dst = reinterpret_cast<float4*>(vh_s + lr * H);
-      for (int c4 = 0; c4 < H4; ++c4) dst[c4] = make_float4(0.f, 0.f, 0.f, 0.f);
+  // with U in tensor memory: lane l of warp w holds its UW*KT values in
+  // columns 16*G*HL + (w >> 2) * UKC + [0, UW*KT)
+  const uint32_t u_col = t_lane + static_cast<uint32_t>(16 * G * HL + (warp >> 2) * UKC);
+  if constexpr (kUTmem) {
+#pragma unroll
+    for (int c = 0; c < UKC / 16; ++c) {
+      float uv[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int idx = 16 * c + j;
+        uv[j] = idx < UW * KT ? ureg[idx / KT][idx % KT] : 0.f;
+      }
+      tmem_st16(u_col + 16 * c, uv);
     }
+    tmem_wait_st();
   }
-  // cell work: item n*S4 + u is depth set n of unit slot u; a thread takes
-  // the items tid, tid + 512, ... which all have unit slot u = tid % S4
-  const int cu = tid & (S4 - 1);
-  const int cj = rank * p.UBv + cu;
-  const bool unit_ok = cu < p.UBv && cj < H;
+  // cell state in the unit block's leader, the warp of gate ub (so that the
+  // four leaders sit on different SM sub-partitions): lane n*UW + i runs
+  // depth set n of unit slot ub*UW + i; lanes i < UW carry c of the full depth
+  const bool leader = gw == ub;
+  const int ci = lane & (UW - 1);
+  const int c_slot = ub * UW + ci;
+  const int cj = rank * p.UBv + c_slot;
+  const bool unit_ok = c_slot < p.UBv && cj < H;
   float bias_r[4] = {0.f, 0.f, 0.f, 0.f};
-  float c_reg = 0.f;  // the carried c of unit cu (threads tid < S4)
-  if (unit_ok) {
+  float c_reg = 0.f;
+  if (leader && unit_ok) {
 #pragma unroll
     for (int g = 0; g < 4; ++g) bias_r[g] = a.bias[g * H + cj];
-    if (tid < S4 && a.c0 != nullptr) c_reg = a.c0[(long long)b * H + cj];
+    if (lane < UW && a.c0 != nullptr) c_reg = a.c0[(long long)b * H + cj];
   }
-  if (tid < S4) c_s[tid] = c_reg;
   // where each depth set leaves the butterfly: set 0 (the full depth) and
   // every depth k_j >= K after all five steps, k_j = KT * 2^S after S steps;
   // other depths take a masked pass of their own
@@ -335,16 +485,23 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   }
   float p_cur = p_off >= 0 ? __ldg(a.P + (long long)b * p_stride + p_off) : 0.f;
 
-  const bool setup_ok = __syncthreads_and(mbar_wait_bounded<false>(bar_setup, 0, limit_ns, err));
-  if (!setup_ok && tid == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
-  cluster_sync_all();  // every CTA's barriers are armed before any st.async
-
+  // remote addresses of the exchange buffers in CTA (lane mod CS)
+  const uint32_t peer = static_cast<uint32_t>(lane) & static_cast<uint32_t>(p.CS - 1);
   const uint32_t bar_tau0 = smem_u32(&bars[0]);
   const uint32_t bar_h0 = smem_u32(&bars[2]);
-  const uint32_t tau_base = smem_u32(tau_s);
-  const uint32_t h_base = smem_u32(h_s);
+  const uint32_t r_tau = mapa_shared(smem_u32(tau_s), peer);
+  const uint32_t r_bar_tau = mapa_shared(bar_tau0, peer);
+  const uint32_t r_h = mapa_shared(smem_u32(h_s), peer);
+  const uint32_t r_bar_h = mapa_shared(bar_h0, peer);
+  const int lcs = ilog2(p.CS);
 
-  for (int t = 0; t < (setup_ok ? a.T : 0); ++t) {
+  bool setup_ok = true;
+  if constexpr (!kTmem) setup_ok = mbar_wait_bounded<false>(bar_setup, 0, limit_ns, err);
+  if (!__syncthreads_and(setup_ok) && tid == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
+  cluster_sync_all();  // every CTA's barriers are armed before any st.async
+
+  const int t_end = *err == 0 ? a.T : 0;  // nothing to do after a failed set-up
+  for (int t = 0; t < t_end; ++t) {
     const int hb = t & 1;
     int fail = 0;  // error code of a wait of this warp that ran out
     // prefetch the next step's projection for this lane's row
@@ -363,43 +520,87 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     }
 
     // ---- phase A: tau' = sigma * (V_h h_{t-1} + P_t) for the owned rows ---
-    const float4* h4 = reinterpret_cast<const float4*>(h_s + hb * h_len);
-    for (int q = 0; fail == 0 && q < kMaxGroupsPerWarp; ++q) {
-      const int grp = warp + kWarps * q;
-      if (grp >= ngroups) break;
-      const int lr0 = grp * 4;
-      float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-      const float4* v0 = reinterpret_cast<const float4*>(vh_s + (lr0 + 0) * H);
-      const float4* v1 = reinterpret_cast<const float4*>(vh_s + (lr0 + 1) * H);
-      const float4* v2 = reinterpret_cast<const float4*>(vh_s + (lr0 + 2) * H);
-      const float4* v3 = reinterpret_cast<const float4*>(vh_s + (lr0 + 3) * H);
+    if constexpr (!kTmem) {
+      const float4* h4 = reinterpret_cast<const float4*>(h_s + hb * h_len);
+      const int H4 = H >> 2;
+      for (int q = 0; fail == 0 && q < kMaxGroups; ++q) {
+        const int grp = warp + kWarps * q;
+        if (grp >= ngroups) break;
+        const int lr0 = grp * 4;
+        float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+        const float4* v0 = reinterpret_cast<const float4*>(vh_s + (lr0 + 0) * H);
+        const float4* v1 = reinterpret_cast<const float4*>(vh_s + (lr0 + 1) * H);
+        const float4* v2 = reinterpret_cast<const float4*>(vh_s + (lr0 + 2) * H);
+        const float4* v3 = reinterpret_cast<const float4*>(vh_s + (lr0 + 3) * H);
 #pragma unroll 1
-      for (int c4 = lane; c4 < H4; c4 += 32) {
-        const float4 hv = h4[c4];
-        float4 w = v0[c4];
-        acc0 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc0))));
-        w = v1[c4];
-        acc1 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc1))));
-        w = v2[c4];
-        acc2 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc2))));
-        w = v3[c4];
-        acc3 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc3))));
+        for (int c4 = lane; c4 < H4; c4 += 32) {
+          const float4 hv = h4[c4];
+          float4 w = v0[c4];
+          acc0 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc0))));
+          w = v1[c4];
+          acc1 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc1))));
+          w = v2[c4];
+          acc2 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc2))));
+          w = v3[c4];
+          acc3 = fmaf(w.x, hv.x, fmaf(w.y, hv.y, fmaf(w.z, hv.z, fmaf(w.w, hv.w, acc3))));
+        }
+        // transposed reduction: lanes 8r .. 8r+7 then hold row r's full sum;
+        // lane 4q + r finishes row r, then the senders gather the four
+        float rs[4] = {acc0, acc1, acc2, acc3};
+        butterfly_transpose<4>(rs, lane);
+        const float mine = __shfl_sync(0xffffffffu, rs[0], (lane & 3) << 3);
+        const float tpr = sig_r * (mine + p_cur);
+        const float t0 = __shfl_sync(0xffffffffu, tpr, 4 * q + 0);
+        const float t1 = __shfl_sync(0xffffffffu, tpr, 4 * q + 1);
+        const float t2 = __shfl_sync(0xffffffffu, tpr, 4 * q + 2);
+        const float t3 = __shfl_sync(0xffffffffu, tpr, 4 * q + 3);
+        if (lane < p.CS) {
+          const uint32_t off = 4u * (hb * tau_len + rank * p.RA + lr0);
+          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
+        }
       }
-      // transposed reduction of the four row sums: afterwards lane l holds the
-      // full sum of row (l >> 3) of the group
-      float rs[4] = {acc0, acc1, acc2, acc3};
-      butterfly_transpose<4>(rs, lane);
-      // lane 4q + r finishes row r of group q, then the senders gather the four
-      const int r = lane & 3;
-      const float mine = __shfl_sync(0xffffffffu, rs[0], r << 3);
-      const float tpr = sig_r * (mine + p_cur);
-      const float t0 = __shfl_sync(0xffffffffu, tpr, 4 * q + 0);
-      const float t1 = __shfl_sync(0xffffffffu, tpr, 4 * q + 1);
-      const float t2 = __shfl_sync(0xffffffffu, tpr, 4 * q + 2);
-      const float t3 = __shfl_sync(0xffffffffu, tpr, 4 * q + 3);
-      if (lane < p.CS) {
-        const uint32_t off = 4u * (hb * tau_len + rank * p.RA + lr0);
-        st_async_v4(mapa_shared(tau_base + off, lane), t0, t1, t2, t3, mapa_shared(bar_tau0 + 8u * hb, lane));
+    }
+    if (kTmem && fail == 0) {
+      const float* hsrc = h_s + hb * h_len + HL * lane;
+#pragma unroll 1
+      for (int q = 0; q < G; ++q) {
+        const int grp = warp + kWarps * q;
+        if (grp >= ngroups) break;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        // two h quads per round: two 16-column loads, one wait
+#pragma unroll
+        for (int e8 = 0; e8 < HL / 8; ++e8) {
+          const float4 ha = *reinterpret_cast<const float4*>(hsrc + 8 * e8);
+          const float4 hb4 = *reinterpret_cast<const float4*>(hsrc + 8 * e8 + 4);
+          float va[16], vb[16];
+          const uint32_t col = t_lane + t_col0 + q * 4 * HL + 32 * e8;
+          tmem_ld16x2_sync(col, col + 16, va, vb);
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            float s0 = acc[r];
+            s0 = fmaf(va[4 * r + 0], ha.x, s0);
+            s0 = fmaf(va[4 * r + 1], ha.y, s0);
+            s0 = fmaf(va[4 * r + 2], ha.z, s0);
+            s0 = fmaf(va[4 * r + 3], ha.w, s0);
+            s0 = fmaf(vb[4 * r + 0], hb4.x, s0);
+            s0 = fmaf(vb[4 * r + 1], hb4.y, s0);
+            s0 = fmaf(vb[4 * r + 2], hb4.z, s0);
+            s0 = fmaf(vb[4 * r + 3], hb4.w, s0);
+            acc[r] = s0;
+          }
+        }
+        // transposed reduction of the four row sums: afterwards lanes
+        // 8r .. 8r+7 hold the full sum of row r of the group
+        butterfly_transpose<4>(acc, lane);
+        const float tpr = sig_r * (acc[0] + p_cur);  // valid on lane 8r + q
+        const float t0 = __shfl_sync(0xffffffffu, tpr, q);
+        const float t1 = __shfl_sync(0xffffffffu, tpr, 8 + q);
+        const float t2 = __shfl_sync(0xffffffffu, tpr, 16 + q);
+        const float t3 = __shfl_sync(0xffffffffu, tpr, 24 + q);
+        if (lane < p.CS) {
+          const uint32_t off = 4u * (hb * tau_len + rank * p.RA + grp * 4);
+          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
+        }
       }
     }
 
@@ -420,82 +621,82 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       const float* tau_lane = tau_s + hb * tau_len + gw * p.Kp + k_lane;
       float* dst = pb + gw * S4 + ub * UW;
       float v[UW];
-      lane_partials<UW, KT>(ureg, tau_lane, KT, v);
+      if constexpr (kUTmem) lane_partials_tmem<UW, KT>(u_col, tau_lane, KT, v);
+      else lane_partials<UW, KT>(ureg, tau_lane, KT, v);
       butterfly_depths<UW>(v, lane, cap, dst, 4 * S4);
       for (uint32_t m = masked; m != 0u; m &= m - 1u) {  // depths of another form
         const int n = __ffs(m) - 1;
-        lane_partials<UW, KT>(ureg, tau_lane, ck_s[n - 1] - k_lane, v);
+        if constexpr (kUTmem) lane_partials_tmem<UW, KT>(u_col, tau_lane, ck_s[n - 1] - k_lane, v);
+        else lane_partials<UW, KT>(ureg, tau_lane, ck_s[n - 1] - k_lane, v);
         butterfly_transpose<UW>(v, lane);
         // lane l holds the total of value l >> (5 - log2 UW)
         constexpr int kSh = 5 - ilog2(UW);
         if ((lane & ((1 << kSh) - 1)) == 0) dst[n * 4 * S4 + (lane >> kSh)] = v[0];
       }
     }
-    // the one block barrier of the step: a wait that ran out in any warp ends
-    // the time loop for the whole CTA here
     if (fail != 0 && lane == 0) atomicCAS(a.err, 0, fail);
-    if (__syncthreads_or(fail)) break;
+    // the four warps of the unit block meet; a wait that ran out in any of
+    // them ends the time loop for the whole block here
+    if (block_barrier_or(1 + ub, 128, fail != 0)) break;
 
-    // ---- the cell update (Sec. II) for every (depth set, unit) ------------
-    const long long tbo = ((long long)t * a.B + b) * H;
-    for (int item = tid; item < p.nset * S4; item += kThreads) {
-      const int n = item / S4;
-      const float* src = pb + n * 4 * S4 + cu;
-      float hh = 0.f, cc = 0.f;
-      if (unit_ok) {
-        const float c_prev = n == 0 ? c_reg : c_s[hb * S4 + cu];
-        lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3],
-                    c_prev, hh, cc);
-        if (n == 0) {
-          c_reg = cc;
-          a.out_h[tbo + cj] = hh;
-        } else {
-          const long long o = (long long)(n - 1) * a.T * a.B * H + tbo + cj;
-          if (a.ckpt_h) a.ckpt_h[o] = hh;
-          if (a.ckpt_c) a.ckpt_c[o] = cc;
+    // ---- cell update (Sec. II) and h_t exchange, in the block's leader ----
+    if (leader) {
+      const long long tbo = ((long long)t * a.B + b) * H;
+      const float cp = __shfl_sync(0xffffffffu, c_reg, ci);  // c_{t-1} of unit ci
+      float h_new = 0.f;
+      for (int n0 = 0; n0 < p.nset; n0 += 32 / UW) {
+        const int n = n0 + lane / UW;
+        if (n < p.nset && unit_ok) {
+          const float* src = pb + n * 4 * S4 + c_slot;
+          float hh, cc;
+          lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3], cp,
+                      hh, cc);
+          if (n == 0) {
+            c_reg = cc;
+            h_new = hh;
+            a.out_h[tbo + cj] = hh;
+          } else {
+            const long long o = (long long)(n - 1) * a.T * a.B * H + tbo + cj;
+            if (a.ckpt_h) a.ckpt_h[o] = hh;
+            if (a.ckpt_c) a.ckpt_c[o] = cc;
+          }
         }
       }
-      if (n == 0) {
-        c_s[(hb ^ 1) * S4 + cu] = c_reg;
-        hsend_s[cu] = hh;
-      }
-    }
-    // ---- push h_t of this CTA's units to every CTA of the cluster ---------
-    if (t + 1 < a.T) {
-      bool send = false;
-      if constexpr (S4 <= 32) {
-        if (warp == 0) {
-          __syncwarp();
-          send = true;
-        }
-      } else {
-        if (tid < S4) {
-          asm volatile("bar.sync 1, %0;" ::"n"(S4) : "memory");  // the unit-slot threads of set 0
-          send = warp == 0;
-        }
-      }
-      if (send) {
+      if (t + 1 < a.T) {
+        // lane m takes (piece m >> log2 CS, CTA m & (CS-1)), then m + 32
         const int nb = (t + 1) & 1;
-        const int nchunks = p.UBv >> 2;
-        for (int m = lane; m < nchunks * p.CS; m += 32) {
-          const int qd = m / p.CS, d = m - qd * p.CS;
-          const float4 hv = *reinterpret_cast<const float4*>(hsend_s + 4 * qd);
-          const uint32_t off = 4u * (nb * h_len + rank * p.UBv + 4 * qd);
-          st_async_v4(mapa_shared(h_base + off, d), hv.x, hv.y, hv.z, hv.w, mapa_shared(bar_h0 + 8u * nb, d));
+        constexpr int kPieces = UW / PIECE;
+#pragma unroll
+        for (int m0 = 0; m0 < 64; m0 += 32) {
+          const int pc = (m0 + lane) >> lcs;
+          const int src0 = (pc < kPieces ? pc : 0) * PIECE;
+          float hv[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) hv[e] = __shfl_sync(0xffffffffu, h_new, src0 + (e < PIECE ? e : 0));
+          const int slot = ub * UW + pc * PIECE;
+          if (pc < kPieces && slot < p.UBv) {
+            const uint32_t off = 4u * (nb * h_len + rank * p.UBv + slot);
+            st_async_piece(r_h + off, hv, PIECE, r_bar_h + 8u * nb);
+          }
         }
       }
     }
     p_cur = p_next;
   }
 
-  if (unit_ok && tid < S4 && a.c_last != nullptr) a.c_last[(long long)b * H + cj] = c_reg;
+  if (leader && lane < UW && unit_ok && a.c_last != nullptr) a.c_last[(long long)b * H + cj] = c_reg;
+  tc_fence_before();
   __syncthreads();
+  if (kTmem && warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tcols);
+  }
   cluster_sync_all();  // no CTA leaves while others may still address its shared memory
 }
 
-template <int UW, int KT>
+template <int UW, int KT, int HC>
 cudaError_t launch_t(const DevPlan& dp, size_t smem, const PersistentArgs& a, cudaStream_t s) {
-  auto kern = persistent_kernel<UW, KT>;
+  auto kern = persistent_kernel<UW, KT, HC>;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(dp.CS * a.B);
   cfg.blockDim = dim3(kThreads);
@@ -550,10 +751,15 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
     *why = "K above 256";
     return false;
   }
+  if (H > 1024) {
+    *why = "hidden size above 1024";
+    return false;
+  }
   const int Kp = (K + 3) & ~3;
   const int rows = 4 * Kp;
   int kt = 1;  // terms per lane: the smallest power of two that covers K with 32 lanes
   while (32 * kt < K) kt *= 2;
+  const int hc = H <= 256 ? 0 : H <= 512 ? 1 : 2;  // V_h in shared memory (0) or tensor memory
   const int cs_list[] = {1, 2, 4, 8, 16};
   PersistentPlan best;
   bool found = false;
@@ -566,13 +772,29 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
     int uw = 1;                            // units per warp: four blocks cover UB
     while (4 * uw < p.UB) uw *= 2;
     if (uw > 16 || uw * kt > 64) continue;  // U registers per thread
-    if ((p.RA / 4 + kWarps - 1) / kWarps > kMaxGroupsPerWarp) continue;
+    if (hc > 0 && uw < 8) continue;         // the tensor-memory variant is built for UW >= 8
+    if (hc == 2 && uw != 16) continue;
+    const int groups = (p.RA / 4 + kWarps - 1) / kWarps;
+    if (groups > (hc > 0 ? kMaxGroupsTmem : kMaxGroupsSmem)) continue;
+    int tcols = 0;
+    if (hc > 0) {
+      const int ukc = hc == 1 ? (uw * kt + 15) / 16 * 16 : 0;  // U in tensor memory for hc == 1
+      const int need = 4 * (groups * 4 * 16 * hc + ukc);
+      if (need > 512) continue;
+      tcols = 32;
+      while (tcols < need) tcols *= 2;
+    }
     p.upl = uw;
     p.kpw = kt;
+    p.hc = hc;
+    p.tcols = tcols;
     DevPlan dp{};
-    dp.CS = p.CS; dp.RA = p.RA; dp.UBv = p.UB; dp.Kp = Kp; dp.nset = 1 + ck.n;
-    p.smem = kBarrierBytes + 4ull * smem_layout(dp, H, 4 * uw).total;
+    dp.CS = p.CS; dp.RA = p.RA; dp.UBv = p.UB; dp.Kp = Kp; dp.nset = 1 + ck.n; dp.tcols = tcols;
+    p.smem = kHeaderBytes + 4ull * smem_layout(dp, H, hc, 4 * uw).total;
     if (p.smem > 227u * 1024u) continue;
+    // at least half of an SM's shared memory, so that no other CTA of this
+    // kernel shares the SM (and its tensor memory) with this one
+    if (p.smem < kMinSmemBytes) p.smem = kMinSmemBytes;
     best = p;
     found = true;
     if (want_cs != 0) break;
@@ -580,7 +802,7 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
     if ((size_t)p.RA * H * 4 <= 32u * 1024u) break;
   }
   if (!found) {
-    *why = "shape does not fit the persistent kernel (hidden size, K or shared memory)";
+    *why = "shape does not fit the persistent kernel (hidden size, K or on-chip memory)";
     return false;
   }
   *plan = best;
@@ -590,14 +812,18 @@ bool plan_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, in
 cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s) {
   DevPlan dp{};
   dp.CS = plan.CS; dp.RA = plan.RA; dp.UBv = plan.UB; dp.Kp = (a.K + 3) & ~3; dp.nset = 1 + a.ck.n;
-  const int u = plan.upl, k = plan.kpw;
-#define LA_CASE(U_, K_) \
-  if (u == U_ && k == K_) return launch_t<U_, K_>(dp, plan.smem, a, s);
-  LA_CASE(1, 1) LA_CASE(1, 2) LA_CASE(1, 4) LA_CASE(1, 8)
-  LA_CASE(2, 1) LA_CASE(2, 2) LA_CASE(2, 4) LA_CASE(2, 8)
-  LA_CASE(4, 1) LA_CASE(4, 2) LA_CASE(4, 4) LA_CASE(4, 8)
-  LA_CASE(8, 1) LA_CASE(8, 2) LA_CASE(8, 4) LA_CASE(8, 8)
-  LA_CASE(16, 1) LA_CASE(16, 2) LA_CASE(16, 4)
+  dp.tcols = plan.tcols;
+  const int u = plan.upl, k = plan.kpw, h = plan.hc;
+#define LA_CASE(U_, K_, H_) \
+  if (u == U_ && k == K_ && h == H_) return launch_t<U_, K_, H_>(dp, plan.smem, a, s);
+  LA_CASE(1, 1, 0) LA_CASE(1, 2, 0) LA_CASE(1, 4, 0) LA_CASE(1, 8, 0)
+  LA_CASE(2, 1, 0) LA_CASE(2, 2, 0) LA_CASE(2, 4, 0) LA_CASE(2, 8, 0)
+  LA_CASE(4, 1, 0) LA_CASE(4, 2, 0) LA_CASE(4, 4, 0) LA_CASE(4, 8, 0)
+  LA_CASE(8, 1, 0) LA_CASE(8, 2, 0) LA_CASE(8, 4, 0) LA_CASE(8, 8, 0)
+  LA_CASE(16, 1, 0) LA_CASE(16, 2, 0) LA_CASE(16, 4, 0)
+  LA_CASE(8, 1, 1) LA_CASE(8, 2, 1) LA_CASE(8, 4, 1) LA_CASE(8, 8, 1)
+  LA_CASE(16, 1, 1) LA_CASE(16, 2, 1) LA_CASE(16, 4, 1)
+  LA_CASE(16, 1, 2) LA_CASE(16, 2, 2) LA_CASE(16, 4, 2)
 #undef LA_CASE
   return cudaErrorInvalidValue;
 }

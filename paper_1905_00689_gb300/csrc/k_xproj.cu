@@ -8,7 +8,7 @@
 // block r by chunk q of the input, four k-groups of 64 threads each
 // accumulate 4 x 4 register tiles, the k-groups are summed in shared memory,
 // and the 8 chunk partials are summed through distributed shared memory in
-// chunk order (deterministic), each CTA finishing 128 of the 1024 outputs.
+// chunk order (deterministic), each CTA finishing 1/kSplit of the outputs.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -133,9 +133,10 @@ __global__ void __launch_bounds__(kThreads) xproj_cluster_kernel(const TF* __res
     part[o] = red[o] + red[1024 + o] + red[2048 + o] + red[3072 + o];
   cluster_sync_all();
 
-  // this CTA finishes outputs [q*128, q*128 + 128) from the 8 chunk partials
-  if (tid < 128) {
-    const int o = q * 128 + tid;
+  // this CTA finishes outputs [q*OPC, (q+1)*OPC) from the kSplit chunk partials
+  constexpr int kOPC = kRows * kCols / kSplit;
+  for (int i = tid; i < kOPC; i += kThreads) {
+    const int o = q * kOPC + i;
     const uint32_t la = smem_u32(&part[o]);
     float s = 0.f;
 #pragma unroll
