@@ -99,11 +99,13 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
                              int N, int Kdim, float* out, int ldo, int mode, const float* sigma,
                              const float* P, int ldp, cudaStream_t s);
 
-// Same product for few columns (N = T*B <= 32): 8-CTA clusters split the
-// D axis and reduce through distributed shared memory (deterministic).
-bool xproj_cluster_fits(int N);
+// Same product for few columns (N = T*B <= 32): clusters split the D axis,
+// rows are staged by bulk copies and reduced through distributed shared
+// memory (deterministic).  Needs D % 8 == 0 and 16-byte aligned rows; a
+// staged load that does not complete within limit_ns sets *err.
+bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16);
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
-                                 int N, int D, float* out, int ldo, cudaStream_t s);
+                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s);
 
 // One timestep of the refinement sums over u (a3), the intermediate outputs
 // (a6) and the cell update (a4) for B streams.

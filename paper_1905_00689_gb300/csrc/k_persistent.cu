@@ -483,6 +483,9 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     }
     if (!placed) masked |= 1u << n;
   }
+  // everything above only read the factors; P is written by the projection
+  // launched just before this kernel, which may still be running
+  griddep_wait();
   float p_cur = p_off >= 0 ? __ldg(a.P + (long long)b * p_stride + p_off) : 0.f;
 
   // remote addresses of the exchange buffers in CTA (lane mod CS)
@@ -702,13 +705,16 @@ cudaError_t launch_t(const DevPlan& dp, size_t smem, const PersistentArgs& a, cu
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = dp.CS;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // may start while the projection before it finishes (set-up overlaps it)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   // function attributes once per instantiation (the largest shared memory any
   // plan may ask for); the co-residency check once per (cluster size, smem)
   static thread_local bool attrs_set = false;

@@ -3,12 +3,15 @@
 // columns of x~ = [x_t; h_{t-1}], Sec. III, split off Eq. 1's dot products).
 //
 // With T*B this small the product is a skinny matrix times a thin one and
-// the whole packed V_x is read once.  To spread it over the GPU the D axis is
-// split over the 8 CTAs of a cluster: CTA (r, q) multiplies the 32 rows of
-// block r by chunk q of the input, four k-groups of 64 threads each
-// accumulate 4 x 4 register tiles, the k-groups are summed in shared memory,
-// and the 8 chunk partials are summed through distributed shared memory in
-// chunk order (deterministic), each CTA finishing 1/kSplit of the outputs.
+// the whole packed V_x is read once, so the kernel is about latency: every
+// CTA owns 32 rows and one of S chunks of D (S CTAs of a cluster along D).
+// It stages up to 256 values of D of its 32 rows of V_x and of the x columns
+// in shared memory with one bulk copy (TMA engine) per row, all in flight at
+// once and completing on one mbarrier; its 8 warps then split the staged
+// range again, each lane accumulating a 4-row x NC-column register tile.
+// The 8 warp partials are summed in shared memory in warp order and the S
+// chunk partials through distributed shared memory in chunk order, so the
+// result does not depend on timing.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -19,53 +22,30 @@ using namespace lstm_approx_dev;
 
 constexpr int kRows = 32;     // rows per CTA
 constexpr int kCols = 32;     // max columns (T*B)
-constexpr int kSplit = 8;     // CTAs per cluster along D
-constexpr int kTileD = 128;   // D tile staged in shared memory
-constexpr int kThreads = 256;
+constexpr int kWarps = 8;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kSub = 256;     // values of D staged per round
+constexpr int kPadF = 4;      // floats of padding after each staged row
+constexpr int kMaxSplit = 8;  // CTAs per cluster along D
 
-// 16 consecutive elements [d, d+16) of row `row` (ld = lda) as fp32, zero
-// outside [0, d_hi) or for row < 0; vector loads when the run is aligned.
-__device__ __forceinline__ void load16(const float* A, long long row, int lda, int d, int d_hi, float (&v)[16]) {
-  if (row < 0) {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = 0.f;
-    return;
-  }
-  const float* src = A + row * lda + d;
-  if (d + 16 <= d_hi && ((reinterpret_cast<uintptr_t>(src) & 15u) == 0)) {
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 f = __ldg(reinterpret_cast<const float4*>(src) + q);
-      v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
-    }
-  } else {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = d + e < d_hi ? __ldg(src + e) : 0.f;
-  }
+template <typename TF>
+constexpr int v_stride() {  // staged V_x row stride in elements (16-byte multiple)
+  return kSub + kPadF * 4 / (int)sizeof(TF);
 }
-__device__ __forceinline__ void load16(const __nv_bfloat16* A, long long row, int lda, int d, int d_hi,
-                                       float (&v)[16]) {
-  if (row < 0) {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = 0.f;
-    return;
-  }
-  const __nv_bfloat16* src = A + row * lda + d;
-  if (d + 16 <= d_hi && ((reinterpret_cast<uintptr_t>(src) & 15u) == 0)) {
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const uint4 f = __ldg(reinterpret_cast<const uint4*>(src) + q);
-      const uint32_t w[4] = {f.x, f.y, f.z, f.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        v[8 * q + 2 * i] = __uint_as_float(w[i] << 16);
-        v[8 * q + 2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-      }
-    }
-  } else {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = d + e < d_hi ? __bfloat162float(src[e]) : 0.f;
-  }
+constexpr int kXStride = kSub + kPadF;
+
+template <typename TF>
+constexpr size_t smem_bytes() {
+  const size_t tiles = (size_t)kRows * v_stride<TF>() * sizeof(TF) + (size_t)kCols * kXStride * 4;
+  const size_t parts = (size_t)kWarps * kRows * kCols * 4;
+  return 16 + (tiles > parts ? tiles : parts) + (size_t)kRows * kCols * 4;
+}
+
+__device__ __forceinline__ float4 lds4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 lds4(const __nv_bfloat16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u), __uint_as_float(u.y << 16),
+                     __uint_as_float(u.y & 0xFFFF0000u));
 }
 
 __device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
@@ -74,102 +54,186 @@ __device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
   return v;
 }
 
-template <typename TF>
-__global__ void __launch_bounds__(kThreads) xproj_cluster_kernel(const TF* __restrict__ A, int lda, int K, int Ks,
-                                                                 const float* __restrict__ X, int ldxin, int N,
-                                                                 int D, float* __restrict__ out, int ldo) {
-  __shared__ __align__(16) float Vs[kTileD][kRows + 4];
-  __shared__ __align__(16) float Xs[kTileD][kCols];
-  __shared__ float part[kRows * kCols];  // o = n * 32 + r
+// Lane (rg = lane >> 2, cg = lane & 3) of every warp owns rows 4*rg .. 4*rg+3
+// of the CTA's 32 and columns cg*NC .. cg*NC + NC - 1.
+template <typename TF, int NC>
+__global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ A, int lda, int K, int Ks,
+                                                         const float* __restrict__ X, int ldxin, int N, int D,
+                                                         int dchunk, float* __restrict__ out, int ldo, int S,
+                                                         int* err, long long limit_ns) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
+  TF* vs = reinterpret_cast<TF*>(smem_raw + 16);  // [32][v_stride]
+  float* xs = reinterpret_cast<float*>(smem_raw + 16 + (size_t)kRows * v_stride<TF>() * sizeof(TF));  // [32][kXStride]
+  float* part = reinterpret_cast<float*>(smem_raw + 16);  // [warp][n * 32 + r], after the last round
+  float* red = reinterpret_cast<float*>(smem_raw + smem_bytes<TF>() - (size_t)kRows * kCols * 4);
+  constexpr int VS = v_stride<TF>();
 
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rg = lane >> 2, cg = lane & 3;
   const int rb = blockIdx.x;
-  const uint32_t q = cluster_ctarank();  // chunk of D (blockIdx.y within the cluster)
+  const uint32_t q = S > 1 ? cluster_ctarank() : 0u;  // chunk of D
   const int nrows = 4 * K;
-  const int dc = ((D + kSplit - 1) / kSplit + 3) & ~3;
-  const int d_lo = min(D, (int)q * dc), d_hi = min(D, d_lo + dc);
+  const int c_lo = min(D, (int)q * dchunk), c_hi = min(D, c_lo + dchunk);
+  const uint32_t mb = smem_u32(bar);
 
-  const int kg = tid >> 6, m = tid & 63;
-  const int r0 = (m >> 3) << 2, n0 = (m & 7) << 2;
-  float acc[4][4] = {};
-
-  // loader mapping: 32 rows (or columns) x 8 slices of 16 d
-  const int lrow = tid >> 3, lseg = (tid & 7) * 16;
-  const int ar = rb * kRows + lrow;
-  const long long asrow = ar < nrows ? (long long)(ar / K) * Ks + ar % K : -1;
-
-  for (int d0 = d_lo; d0 < d_hi; d0 += kTileD) {
-    const int dbase = d0 + lseg;
-    float vv[16], xx[16];
-    load16(A, asrow, lda, dbase, d_hi, vv);
-    load16(X, lrow < N ? (long long)lrow : -1LL, ldxin, dbase, d_hi, xx);
-#pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      Vs[lseg + e][lrow] = vv[e];
-      Xs[lseg + e][lrow] = xx[e];
-    }
-    __syncthreads();
-#pragma unroll 4
-    for (int d = kg; d < kTileD; d += 4) {
-      const float4 a = *reinterpret_cast<const float4*>(&Vs[d][r0]);
-      const float4 x = *reinterpret_cast<const float4*>(&Xs[d][n0]);
-      const float av[4] = {a.x, a.y, a.z, a.w}, xv[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], xv[j], acc[i][j]);
-    }
-    __syncthreads();
+  griddep_launch_dependents();  // the recurrence kernel may start its set-up
+  if (tid == 0) {
+    mbar_init(mb, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  // rows and columns that are never loaded read as zero
+  for (int i = tid; i < kRows * VS; i += kThreads)
+    if (rb * kRows + i / VS >= nrows) vs[i] = TF(0.f);
+  for (int i = tid; i < kCols * kXStride; i += kThreads)
+    if (i / kXStride >= N) xs[i] = 0.f;
+  __syncthreads();
 
-  // sum the four k-groups (reusing the V tile as scratch: 4 x 1024 floats)
-  float* red = &Vs[0][0];
+  float acc[4][NC];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) red[kg * 1024 + (n0 + j) * kRows + (r0 + i)] = acc[i][j];
-  __syncthreads();
-  for (int o = tid; o < kRows * kCols; o += kThreads)
-    part[o] = red[o] + red[1024 + o] + red[2048 + o] + red[3072 + o];
-  cluster_sync_all();
+    for (int j = 0; j < NC; ++j) acc[i][j] = 0.f;
 
-  // this CTA finishes outputs [q*OPC, (q+1)*OPC) from the kSplit chunk partials
-  constexpr int kOPC = kRows * kCols / kSplit;
-  for (int i = tid; i < kOPC; i += kThreads) {
-    const int o = q * kOPC + i;
-    const uint32_t la = smem_u32(&part[o]);
+  bool ok = true;
+  uint32_t phase = 0;
+  for (int d0 = c_lo; d0 < c_hi; d0 += kSub) {
+    const int len = min(kSub, c_hi - d0);
+    const int vrows = min(kRows, nrows - rb * kRows);
+    if (tid == 0) mbar_arrive_expect_tx(mb, (uint32_t)(len * (vrows * (int)sizeof(TF) + N * 4)));
+    if (tid < vrows) {
+      const int r = rb * kRows + tid;
+      bulk_copy_g2s(smem_u32(vs + tid * VS), A + (long long)((r / K) * Ks + r % K) * lda + d0,
+                    (uint32_t)(len * sizeof(TF)), mb);
+    } else if (tid >= kRows && tid < kRows + N) {
+      const int n = tid - kRows;
+      bulk_copy_g2s(smem_u32(xs + n * kXStride), X + (long long)n * ldxin + d0, (uint32_t)(len * 4), mb);
+    }
+    ok = __syncthreads_and(ok && mbar_wait_bounded<false>(mb, phase, static_cast<uint64_t>(limit_ns), err));
+    phase ^= 1u;
+    if (!ok) break;
+    // this warp's share of the staged range, in multiples of 4
+    const int wlen = ((len + kWarps - 1) / kWarps + 3) & ~3;
+    const int e_lo = min(len, warp * wlen), e_hi = min(len, e_lo + wlen);
+    for (int e = e_lo; e < e_hi; e += 4) {
+      float4 va[4], xb[NC];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) va[i] = lds4(vs + (4 * rg + i) * VS + e);
+#pragma unroll
+      for (int j = 0; j < NC; ++j) xb[j] = lds4(xs + (cg * NC + j) * kXStride + e);
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < NC; ++j) {
+          float s = acc[i][j];
+          s = fmaf(va[i].x, xb[j].x, s);
+          s = fmaf(va[i].y, xb[j].y, s);
+          s = fmaf(va[i].z, xb[j].z, s);
+          s = fmaf(va[i].w, xb[j].w, s);
+          acc[i][j] = s;
+        }
+    }
+    __syncthreads();  // the staged tiles are free for the next round (and the partials)
+  }
+  if (!ok && tid == 0) atomicCAS(err, 0, kErrTcTimeout);
+
+  // warp partials, then their sum in warp order
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
+      const int n = cg * NC + j;
+      if (n < kCols) part[(warp * kCols + n) * kRows + 4 * rg + i] = acc[i][j];
+    }
+  __syncthreads();
+  for (int o = tid; o < kRows * kCols; o += kThreads) {
     float s = 0.f;
 #pragma unroll
-    for (int c = 0; c < kSplit; ++c) s += ld_cluster_f32(mapa_shared(la, c));
-    const int n = o / kRows, r = rb * kRows + o % kRows;
-    if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = s;
+    for (int w = 0; w < kWarps; ++w) s += part[w * kRows * kCols + o];
+    red[o] = s;
   }
-  cluster_sync_all();  // partials stay readable until every CTA has summed
+  if (S > 1) {
+    cluster_sync_all();
+    // this CTA finishes outputs [q*OPC, (q+1)*OPC) from the S chunk sums, in chunk order
+    const int opc = kRows * kCols / S;
+    for (int i = tid; i < opc; i += kThreads) {
+      const int o = (int)q * opc + i;
+      const uint32_t la = smem_u32(&red[o]);
+      float s = 0.f;
+      for (int c = 0; c < S; ++c) s += ld_cluster_f32(mapa_shared(la, c));
+      const int n = o / kRows, r = rb * kRows + o % kRows;
+      if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = s;
+    }
+    cluster_sync_all();  // chunk sums stay readable until every CTA has summed
+  } else {
+    __syncthreads();
+    for (int o = tid; o < kRows * kCols; o += kThreads) {
+      const int n = o / kRows, r = rb * kRows + o % kRows;
+      if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = red[o];
+    }
+  }
 }
 
-}  // namespace
-
-bool xproj_cluster_fits(int N) { return N >= 1 && N <= kCols; }
-
-cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
-                                 int N, int D, float* out, int ldo, cudaStream_t s) {
+template <typename TF, int NC>
+cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
+                      int ldo, int* err, long long limit_ns, cudaStream_t s) {
+  auto kern = xproj_kernel<TF, NC>;
+  constexpr size_t smem = smem_bytes<TF>();
+  static thread_local bool attr_set = false;
+  if (!attr_set) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int row_tiles = (4 * K + kRows - 1) / kRows;
+  int S = 1;  // chunks of D: about one CTA per SM in total, at least 128 values of D each
+  while (S < kMaxSplit && row_tiles * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
+  const int dchunk = (((D + S - 1) / S) + 7) & ~7;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((4 * K + kRows - 1) / kRows, kSplit, 1);
+  cfg.gridDim = dim3(row_tiles, S, 1);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = 0;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = kSplit;
+  attr[0].val.clusterDim.y = S;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, A, lda, K, Ks, X, ldxin, N, D, dchunk, out, ldo, S, err, limit_ns);
+}
+
+template <typename TF>
+cudaError_t launch_typed(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
+                         int ldo, int* err, long long limit_ns, cudaStream_t s) {
+  switch ((N + 3) / 4) {  // columns per lane
+    case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 4: return launch_nc<TF, 4>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 5: return launch_nc<TF, 5>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 6: return launch_nc<TF, 6>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 7: return launch_nc<TF, 7>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 8: return launch_nc<TF, 8>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16) {
+  // bulk copies need 16-byte aligned rows and lengths
+  const int a_align = a_bf16 ? 8 : 4;
+  return N >= 1 && N <= kCols && D % 8 == 0 && lda % a_align == 0 && ldxin % 4 == 0;
+}
+
+cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
+                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s) {
   if (a_bf16)
-    return cudaLaunchKernelEx(&cfg, xproj_cluster_kernel<__nv_bfloat16>, static_cast<const __nv_bfloat16*>(A), lda,
-                              K, Ks, X, ldxin, N, D, out, ldo);
-  return cudaLaunchKernelEx(&cfg, xproj_cluster_kernel<float>, static_cast<const float*>(A), lda, K, Ks, X, ldxin, N,
-                            D, out, ldo);
+    return launch_typed(static_cast<const __nv_bfloat16*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns,
+                        s);
+  return launch_typed(static_cast<const float*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
 }
 
 }  // namespace lstm_approx_impl

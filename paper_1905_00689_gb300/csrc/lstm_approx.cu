@@ -351,8 +351,10 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
     {
       PhaseTimer pt(h, 0);
-      if (xproj_cluster_fits(T * B))
-        LA_CUDA(h, launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->stream),
+      if (xproj_cluster_fits(T * B, s.D, s.ldx, s.D, bf16))
+        LA_CUDA(h,
+                launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->err,
+                                     h->opt_wait_limit_us * 1000LL, h->stream),
                 "input projection launch");
       else
         LA_CUDA(h,

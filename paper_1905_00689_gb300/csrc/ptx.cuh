@@ -115,6 +115,15 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
                : "memory");
 }
 
+// Programmatic dependent launch: the kernel that follows in the stream may
+// start (and run its set-up) once every CTA of this grid has signalled;
+// griddep_wait() in that kernel blocks until this grid has completed and
+// its memory operations are visible.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Makes a value opaque to the compiler, so that it stays in its register for
 // the rest of a persistent kernel instead of being loaded again from memory
 // where it is used.
