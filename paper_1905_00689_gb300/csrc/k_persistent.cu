@@ -11,8 +11,8 @@
 //            groups of four; warp w takes groups w, w + 16, ...  Its rows of
 //            the pruned V_h (masked-dense, fp32) stay on chip: for hidden
 //            sizes above 256 in tensor memory (HC = 1, 2), where lane l of the
-//            warp holds the four rows' values at h indices
-//            [16*HC*l, 16*HC*(l+1)) and reads them with tcgen05.ld, so the
+//            warp holds the four rows' values at the h indices 4l + 128e + i
+//            (e < 4*HC) and reads them with tcgen05.ld, so the
 //            only shared-memory traffic is h itself; for smaller hidden sizes
 //            (HC = 0) in shared memory, read with 128-bit loads.  The x part was hoisted
 //            into P = V_x X for all t by an earlier launch and is prefetched
@@ -53,7 +53,7 @@ using namespace lstm_approx_dev;
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTauSlack = 256;          // >= 32 * KT - Kp: lane reads past the last gate's rows
+constexpr int kTauSlack = 384;          // padding rows of the last CTA and lane reads past gate 3
 constexpr int kMaxGroupsTmem = 2;       // groups of four V_h rows per warp, V_h in tensor memory
 constexpr int kMaxGroupsSmem = 8;       // the same, V_h in shared memory
 constexpr uint32_t kHeaderBytes = 128;  // 5 mbarriers, the TMEM address, the depths k_j
@@ -76,12 +76,22 @@ __host__ __device__ inline int h_buffer_len(const DevPlan& p, int HC) {
   return a > b ? a : b;
 }
 
+// tau' layout: gate g's rows start at g * GP and term k sits at
+// k + 4 * (k / 32), so that the 16-byte reads of neighbouring lanes in
+// phase B fall into different banks; rows past the four gates (padding of
+// the last CTA) follow at 4 * GP.
+__host__ __device__ inline int tau_gate_len(int Kp) { return Kp + 4 * ((Kp + 31) / 32); }
+__host__ __device__ inline int tau_pos(int row, int Kp) {
+  const int g = row / Kp, k = row - g * Kp;
+  return g < 4 ? g * tau_gate_len(Kp) + k + 4 * (k >> 5) : 4 * tau_gate_len(Kp) + (row - 4 * Kp);
+}
+
 // S4 = 4 * UW unit slots per CTA (the first UBv are real units).
 __host__ __device__ inline SmemLayout smem_layout(const DevPlan& p, int H, int HC, int S4) {
   SmemLayout L;
   uint32_t o = 0;
   L.vh = o;   o += HC == 0 ? p.RA * H : 0;
-  L.tau = o;  o += 2 * (p.CS * p.RA + kTauSlack);
+  L.tau = o;  o += 2 * (4 * tau_gate_len(p.Kp) + kTauSlack);
   L.h = o;    o += 2 * h_buffer_len(p, HC);
   L.part = o; o += 2 * p.nset * 4 * S4;
   L.total = o;
@@ -284,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const uint32_t rank = cluster_ctarank();
   const int b = blockIdx.x / p.CS;  // one cluster per stream
   const int H = a.H, K = a.K, J = a.ck.n;
-  const int tau_len = p.CS * p.RA + kTauSlack;
+  const int tau_len = 4 * tau_gate_len(p.Kp) + kTauSlack;
   const int h_len = h_buffer_len(p, HC);
   const uint32_t bytes_tau = p.CS * p.RA * 4u;
   const uint32_t bytes_h = p.CS * p.UBv * 4u;
@@ -333,8 +343,9 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
 
   // V_h rows of this CTA into tensor memory.  Thread (warp w, lane l) holds,
   // for its groups q (group w + 16 q), the values of the group's four rows at
-  // h indices [HL*l, HL*(l+1)) in its TMEM lane 32*(w & 3) + l: h quad e4
-  // (indices HL*l + 4*e4 + i) of row r at column
+  // the h indices 4*l + 128*e4 + i (e4 < HL/4, i < 4; consecutive lanes read
+  // consecutive 16-byte quads of h) in its TMEM lane 32*(w & 3) + l: quad e4
+  // of row r at column
   // (w >> 2) * (G*4*HL) + q*4*HL + 16*e4 + 4*r + i, so that one 16-column
   // load brings one h quad of all four rows.
   const int G = (ngroups + kWarps - 1) / kWarps;
@@ -344,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     const int grp = warp + kWarps * q;
 #pragma unroll
     for (int e4 = 0; e4 < HL / 4; ++e4) {
-      const int hi = HL * lane + 4 * e4;
+      const int hi = 4 * lane + 128 * e4;
       float v[16];
 #pragma unroll
       for (int r = 0; r < 4; ++r) {
@@ -558,13 +569,13 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
         const float t2 = __shfl_sync(0xffffffffu, tpr, 4 * q + 2);
         const float t3 = __shfl_sync(0xffffffffu, tpr, 4 * q + 3);
         if (lane < p.CS) {
-          const uint32_t off = 4u * (hb * tau_len + rank * p.RA + lr0);
+          const uint32_t off = 4u * (hb * tau_len + tau_pos(rank * p.RA + lr0, p.Kp));
           st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
         }
       }
     }
     if (kTmem && fail == 0) {
-      const float* hsrc = h_s + hb * h_len + HL * lane;
+      const float* hsrc = h_s + hb * h_len + 4 * lane;
 #pragma unroll 1
       for (int q = 0; q < G; ++q) {
         const int grp = warp + kWarps * q;
@@ -573,8 +584,8 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
         // two h quads per round: two 16-column loads, one wait
 #pragma unroll
         for (int e8 = 0; e8 < HL / 8; ++e8) {
-          const float4 ha = *reinterpret_cast<const float4*>(hsrc + 8 * e8);
-          const float4 hb4 = *reinterpret_cast<const float4*>(hsrc + 8 * e8 + 4);
+          const float4 ha = *reinterpret_cast<const float4*>(hsrc + 256 * e8);
+          const float4 hb4 = *reinterpret_cast<const float4*>(hsrc + 256 * e8 + 128);
           float va[16], vb[16];
           const uint32_t col = t_lane + t_col0 + q * 4 * HL + 32 * e8;
           tmem_ld16x2_sync(col, col + 16, va, vb);
@@ -601,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
         const float t2 = __shfl_sync(0xffffffffu, tpr, 16 + q);
         const float t3 = __shfl_sync(0xffffffffu, tpr, 24 + q);
         if (lane < p.CS) {
-          const uint32_t off = 4u * (hb * tau_len + rank * p.RA + grp * 4);
+          const uint32_t off = 4u * (hb * tau_len + tau_pos(rank * p.RA + grp * 4, p.Kp));
           st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
         }
       }
@@ -621,7 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     // ---- phase B: gate sums of this warp's (gate, unit block) -------------
     float* pb = part_s + hb * part_buf;
     if (fail == 0) {
-      const float* tau_lane = tau_s + hb * tau_len + gw * p.Kp + k_lane;
+      const float* tau_lane = tau_s + hb * tau_len + gw * tau_gate_len(p.Kp) + k_lane + 4 * (k_lane >> 5);
       float* dst = pb + gw * S4 + ub * UW;
       float v[UW];
       if constexpr (kUTmem) lane_partials_tmem<UW, KT>(u_col, tau_lane, KT, v);
