@@ -88,6 +88,19 @@ def aggregate(values_ms, world_size: int, units_per_rank: int):
     return units_per_rank * world_size / (t / 1e3), t
 
 
+def combine_ranks(times_ms, units_per_rank: int, dist=None, device="cpu"):
+    """Max over ranks of each per-rank time (one all-reduce), and the whole-job
+    throughput for each: the units all ranks processed over the slowest rank."""
+    import torch
+    vals = torch.tensor(list(times_ms), dtype=torch.float64, device=device)
+    ws = 1
+    if dist is not None:
+        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
+        ws = dist.get_world_size()
+    worst = [float(v) for v in vals.cpu()]
+    return [units_per_rank * ws / (t / 1e3) for t in worst], worst
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
 
@@ -313,12 +326,7 @@ def run_ours(args):
     e2e_ms = 1e3 * sum(e2e_t) / len(e2e_t)
 
     # ---- aggregate over ranks ----------------------------------------------
-    vals = torch.tensor([ms_mean, e2e_ms], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
-    ms_max, e2e_max = float(vals[0]), float(vals[1])
-    value = T * B * ws / (ms_max / 1e3)
-    e2e_value = T * B * ws / (e2e_max / 1e3)
+    (value, e2e_value), (ms_max, e2e_max) = combine_ranks([ms_mean, e2e_ms], T * B, dist, dev)
 
     if rank == 0:
         peaks = {}
