@@ -12,9 +12,9 @@
 // tcgen05.mma (M = 128, N = BN, K = 16 per instruction) into a tensor-memory
 // accumulator, and warps 4..11 (two per 32-lane quarter of tensor memory)
 // read it back with tcgen05.ld for the epilogue: store P, or form tau' in
-// bf16.  For tau' the epilogue warps first load the P_t tile and store it
-// into the accumulator with tcgen05.st while the mainloop streams, so the
-// MMAs accumulate on top of it and the epilogue reads no global memory.
+// bf16.  For tau' the epilogue warps load their P_t values while the
+// mainloop streams: into registers for tiles up to 128 columns, otherwise
+// into the accumulator with tcgen05.st so that the MMAs accumulate on top.
 //
 // tc_gates_kernel computes, for 128 hidden units x NT streams, the four gate
 // sums at once in four tensor-memory accumulators and runs the cell update
@@ -71,7 +71,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int nkb = (a.Kdim + kTileK - 1) / kTileK;
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
-  const bool add_p = a.mode == 1;  // accumulate on top of P_t, preloaded into tensor memory
+  const bool add_p = a.mode == 1;  // tau' = sigma * (accumulator + P_t)
+  // BN <= 128: the epilogue threads hold their P_t values in registers; wider
+  // tiles store P_t into the accumulator before the MMAs start
+  constexpr bool kPReg = BN <= 128;
+  const bool p_tmem = add_p && !kPReg;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -114,7 +118,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, BN);
     bool ok = true;
-    if (add_p) {  // the accumulator starts from P_t
+    if (p_tmem) {  // the accumulator starts from P_t
       ok = wait_cta(pinit_bar, 0, limit, err);
       tc_fence_after();
     }
@@ -126,7 +130,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint64_t db = umma_desc_sw128(sB + s * kBBytes);
 #pragma unroll
       for (int kk = 0; kk < kTileK / 16; ++kk)
-        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (add_p || (kb | kk) != 0) ? 1u : 0u);
+        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (p_tmem || (kb | kk) != 0) ? 1u : 0u);
       umma_commit(bar0 + 8u * (S + s));  // frees the stage once these MMAs are done
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
@@ -142,7 +146,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int row = row0 + lrow;
     const bool row_ok = k < a.K;
     const uint32_t trow = tmem + ((32u * q) << 16);
-    if (add_p) {  // P_t of this tile -> tensor memory, while the mainloop runs
+    float preg[kPReg ? kHalf : 1];  // P_t of this thread's row and columns
+    if (add_p && kPReg) {  // loaded while the mainloop runs
+#pragma unroll
+      for (int c = 0; c < (kPReg ? kHalf : 1); ++c) {
+        const int n = col0 + cbeg + c;
+        preg[c] = (row_ok && n < a.N) ? __ldg(a.P + (long long)n * a.ldp + row) : 0.f;
+      }
+    }
+    if (p_tmem) {  // P_t of this tile -> tensor memory, while the mainloop runs
       const float* __restrict__ P = a.P;
 #pragma unroll 1
       for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 64) {
@@ -166,7 +178,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     const float sig = (add_p && row_ok) ? a.sigma[row] : 0.f;
     const bool write = ok && *err == 0;
-    for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 16) {
+#pragma unroll
+    for (int cc = 0; cc < kHalf; cc += 16) {
+      const int c0 = cbeg + cc;
       float v[16];
       tmem_ld16(trow + c0, v);
       tmem_wait_ld();
@@ -178,7 +192,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (!add_p) {
           if (row_ok) a.P[(long long)n * a.ldp + row] = v[j];
         } else {
-          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(row_ok ? sig * v[j] : 0.f);
+          const float acc = kPReg ? v[j] + preg[kPReg ? cc + j : 0] : v[j];
+          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(row_ok ? sig * acc : 0.f);
         }
       }
     }
@@ -332,7 +347,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           if (n >= a.B) break;
           const long long sj = (long long)n * a.H + j;
           float hh, cc;
-          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
+          lstm_cell_hw(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
           if (!final_sums) {
             const long long o = (long long)step * a.ck_stride + sj;
             if (a.ckpt_h) a.ckpt_h[o] = hh;
