@@ -77,6 +77,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   constexpr bool kPReg = BN <= 128;
   const bool p_tmem = add_p && !kPReg;
 
+  griddep_launch_dependents();  // the next kernel may start its own set-up
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(bar0 + 8u * i, 1);
@@ -101,11 +102,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tma_prefetch_map(&tmb);
     int issued = 0;
     bool ok = true;
+    // the factor tiles of the first S stages do not depend on the kernel
+    // before this one: issue them before waiting for it
+    const int npre = nkb < S ? nkb : S;
+    for (int kb = 0; kb < npre; ++kb) {
+      mbar_arrive_expect_tx(bar0 + 8u * kb, kABytes + kBBytes);
+      tma_load_2d(sA + kb * kABytes, &tma, bar0 + 8u * kb, kb * kTileK, row0);
+    }
+    griddep_wait();
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % S;
       if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
-      mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
-      tma_load_2d(sA + s * kABytes, &tma, bar0 + 8u * s, kb * kTileK, row0);
+      if (kb >= npre) {
+        mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
+        tma_load_2d(sA + s * kABytes, &tma, bar0 + 8u * s, kb * kTileK, row0);
+      }
       tma_load_2d(sB + s * kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
       ++issued;
     }
@@ -154,6 +165,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         preg[c] = (row_ok && n < a.N) ? __ldg(a.P + (long long)n * a.ldp + row) : 0.f;
       }
     }
+    griddep_wait();  // the outputs below may still be read by the kernel before this one
     if (p_tmem) {  // P_t of this tile -> tensor memory, while the mainloop runs
       const float* __restrict__ P = a.P;
 #pragma unroll 1
@@ -232,6 +244,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
 
+  griddep_launch_dependents();  // the next kernel may start its own set-up
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
       mbar_init(bar0 + 8u * i, 1);
@@ -258,11 +271,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int nst = 4 * nkb;
     int issued = 0;
     bool ok = true;
+    // U tiles of the first S stages first: they do not depend on the kernel before this one
+    const int npre = nst < S ? nst : S;
+    for (int i = 0; i < npre; ++i) {
+      mbar_arrive_expect_tx(bar0 + 8u * i, kABytes + kBBytes);
+      tma_load_2d(sA + i * kABytes, &tmu, bar0 + 8u * i, (i >> 2) * kTileK, (i & 3) * a.H + j0);
+    }
+    griddep_wait();
     for (int i = 0; i < nst; ++i) {
       const int s = i % S, kb = i >> 2, g = i & 3;
       if (i >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((i / S) - 1) & 1, limit, err))) break;
-      mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
-      tma_load_2d(sA + s * kABytes, &tmu, bar0 + 8u * s, kb * kTileK, g * a.H + j0);
+      if (i >= npre) {
+        mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
+        tma_load_2d(sA + s * kABytes, &tmu, bar0 + 8u * s, kb * kTileK, g * a.H + j0);
+      }
       tma_load_2d(sB + s * kBBytes, &tmt, bar0 + 8u * s, g * a.Ks + kb * kTileK, n0);
       ++issued;
     }
@@ -324,6 +346,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
       for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
     const uint32_t trow = tmem + ((32u * q) << 16);
+    griddep_wait();  // c_t-1 and the outputs are shared with the kernels before this one
     for (int step = 0; step <= J; ++step) {
       const bool final_sums = step == J;
       const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)(step & 1), limit, err);
@@ -437,6 +460,24 @@ EncodeTiled encoder() {
   return fn;
 }
 
+// Launch with programmatic stream serialization: the kernel may start while
+// the one before it in the stream finishes, and waits on it (griddep_wait)
+// only where it reads that kernel's results or writes what it reads.
+template <typename Kern, typename... Args>
+cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 template <int BN, int S>
 size_t rows_smem() {
   return 1024 + S * (kABytes + BN * kTileK * 2) + 8 * (2 * S + 3) + 16;
@@ -456,10 +497,9 @@ cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, 
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid(4 * a.kt_per_gate, (n_cols + BN - 1) / BN);
-  kern<<<grid, kTcThreads, smem, s>>>(*reinterpret_cast<const CUtensorMap*>(A.bytes),
-                                      *reinterpret_cast<const CUtensorMap*>(Bm.bytes), a);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(4 * a.kt_per_gate, (n_cols + BN - 1) / BN), smem, s,
+                    *reinterpret_cast<const CUtensorMap*>(A.bytes), *reinterpret_cast<const CUtensorMap*>(Bm.bytes),
+                    a);
 }
 
 template <int NT, int S>
@@ -472,10 +512,9 @@ cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& 
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT);
-  kern<<<grid, kTcThreads, smem, s>>>(*reinterpret_cast<const CUtensorMap*>(U.bytes),
-                                      *reinterpret_cast<const CUtensorMap*>(Tau.bytes), a);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT), smem, s,
+                    *reinterpret_cast<const CUtensorMap*>(U.bytes), *reinterpret_cast<const CUtensorMap*>(Tau.bytes),
+                    a);
 }
 
 }  // namespace
