@@ -299,24 +299,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     int jj = 0;
     for (int kb = 0; kb < nkb && ok; ++kb) {
       uint64_t da[4], db[4];
-      for (int g = 0; g < 4 && ok; ++g) {
-        const int i = 4 * kb + g, s = i % S;
-        ok = wait_cta(bar0 + 8u * s, (i / S) & 1, limit, err);
-        da[g] = umma_desc_sw128(sA + s * kABytes);
-        db[g] = umma_desc_sw128(sB + s * kBBytes);
-      }
-      if (!ok) break;
-      tc_fence_after();
-      // 16-term slices of this chunk, cut where an intermediate depth ends
+      // 16-term slices of this chunk, cut where an intermediate depth ends;
+      // each gate's stage is used as soon as it lands and freed as soon as
+      // its last slice is issued
       int kk0 = 0;
       while (kk0 < 4 && ok) {
         int kk1 = 4;
         const bool cut_here = jj < J && a.ck.k[jj] <= (kb + 1) * kTileK;
         if (cut_here) kk1 = (a.ck.k[jj] - kb * kTileK) / 16;
-        for (int g = 0; g < 4; ++g)
+        for (int g = 0; g < 4 && ok; ++g) {
+          const int i = 4 * kb + g, s = i % S;
+          if (kk0 == 0) {
+            if (!(ok = wait_cta(bar0 + 8u * s, (i / S) & 1, limit, err))) break;
+            tc_fence_after();
+            da[g] = umma_desc_sw128(sA + s * kABytes);
+            db[g] = umma_desc_sw128(sB + s * kBBytes);
+          }
           for (int kk = kk0; kk < kk1; ++kk)
             umma_bf16(tmem + g * NT, da[g] + 2ull * kk, db[g] + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
-        if (cut_here) {  // partial sums up to depth k_jj are complete: hand them to the epilogue
+          if (kk1 == 4) umma_commit(bar0 + 8u * (S + s));  // frees this gate's stage
+        }
+        if (ok && cut_here) {  // partial sums up to depth k_jj are complete: hand them to the epilogue
           umma_commit(ckpt_bar);
           ok = wait_cta(ckpt_done, jj & 1, limit, err);
           tc_fence_after();
@@ -324,7 +327,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         kk0 = kk1;
       }
-      for (int g = 0; g < 4; ++g) umma_commit(bar0 + 8u * (S + (4 * kb + g) % S));
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
     while (jj < J) {  // release epilogue warps still waiting for a depth (abort only)
