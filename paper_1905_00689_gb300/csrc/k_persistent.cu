@@ -353,20 +353,35 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const uint32_t t_col0 = static_cast<uint32_t>((warp >> 2) * G * 4 * HL);
   for (int q = 0; kTmem && q < G; ++q) {
     const int grp = warp + kWarps * q;
+    const float* rowp[4];  // the group's four rows (null: padding)
 #pragma unroll
-    for (int e4 = 0; e4 < HL / 4; ++e4) {
-      const int hi = 4 * lane + 128 * e4;
-      float v[16];
+    for (int r = 0; r < 4; ++r) {
+      const int gr = rank * p.RA + grp * 4 + r;
+      const int g = gr / p.Kp, k = gr % p.Kp;
+      rowp[r] = (grp < ngroups && g < 4 && k < K) ? a.Vh + ((long long)g * a.Ks + k) * a.ldh : nullptr;
+    }
+    // all loads of a half (up to 8 h quads x 4 rows) are issued before the
+    // first store, so the set-up pays one memory round trip per half
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const int gr = rank * p.RA + grp * 4 + r;
-        const int g = gr / p.Kp, k = gr % p.Kp;
-        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (grp < ngroups && g < 4 && k < K && hi < H)
-          f = __ldg(reinterpret_cast<const float4*>(a.Vh + ((long long)g * a.Ks + k) * a.ldh + hi));
-        v[4 * r] = f.x; v[4 * r + 1] = f.y; v[4 * r + 2] = f.z; v[4 * r + 3] = f.w;
+    for (int h0 = 0; h0 < HL / 4; h0 += 4) {
+      float4 f[4][4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int hi = 4 * lane + 128 * (h0 + e);
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          f[e][r] = (rowp[r] != nullptr && hi < H) ? __ldg(reinterpret_cast<const float4*>(rowp[r] + hi))
+                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
       }
-      tmem_st16(t_lane + t_col0 + q * 4 * HL + 16 * e4, v);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float v[16];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          v[4 * r] = f[e][r].x; v[4 * r + 1] = f[e][r].y; v[4 * r + 2] = f[e][r].z; v[4 * r + 3] = f[e][r].w;
+        }
+        tmem_st16(t_lane + t_col0 + q * 4 * HL + 16 * (h0 + e), v);
+      }
     }
   }
   if constexpr (kTmem) {
