@@ -308,6 +308,7 @@ def run_ours(args):
 
     # ---- large-batch tensor-core path (bf16 factors) -------------------------
     large = [] if (args.quick or args.no_large) else large_batch_sweep(dev, stream, peaks_bf16())
+    paper_case = None if (args.quick or args.no_large) else paper_case_sweep(dev, stream)
 
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
@@ -358,6 +359,7 @@ def run_ours(args):
             "cluster_ctas": cluster,
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
             "large_batch": large,
+            "paper_case_study": paper_case,
         }
         if ws == 1 and not (args.no_cpu_baseline or args.quick):
             line["cpu_baseline"] = cpu_baseline()
@@ -427,6 +429,64 @@ def large_batch_sweep(dev, stream, peak):
         del m, x, oh, ck
         torch.cuda.empty_cache()
     return out
+
+
+# the paper's FPGA latencies for one timestep of its case-study LSTM (Table I),
+# by kept entries per v; context only (another machine, K chosen by the paper)
+PAPER_FPGA_MS = {4160: 0.36190, 130: 0.03924, 32: 0.00072}
+
+
+def paper_case_sweep(dev, stream):
+    """The paper's case-study shape (H=64, C=8320, one timestep, one stream,
+    fp32): device time of one whole call (projection + recurrence) per K and
+    NZ, warm caches.  Calls this short are bound by the host's launch path, so
+    each call is also captured once as a CUDA graph and replayed: the graph
+    time is the device time of the call's kernels alone."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, Q_LAST_PATH
+    w = WORKLOADS["f1"]
+    cs = torch.cuda.Stream(dev)
+    x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+    oh = torch.empty((w.T, w.B, w.H), device=dev)
+    out = []
+
+    def timed(fn, n):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        with torch.cuda.stream(cs):
+            for a, b in evs:
+                a.record(cs)
+                fn()
+                b.record(cs)
+        torch.cuda.synchronize(dev)
+        return 1e3 * statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    for keep in w.keeps:
+        nz = nz_from_keep(keep, w.C())
+        m = LSTMApprox(1, [w.D], w.H, max(w.Ks), w.B, "fp32", stream=cs)
+        m.set_layer(0, synthetic_layer_factors(w, 0, max(w.Ks), keep))
+        for K in w.Ks:
+            call = lambda K=K: m.run(x, K, oh)
+            for _ in range(10):
+                call()
+            m.sync()
+            us_call = timed(call, 200)
+            us_graph = None
+            try:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cs):
+                    call()
+                g.replay()
+                torch.cuda.synchronize(dev)
+                us_graph = timed(g.replay, 200)
+            except RuntimeError:
+                pass
+            out.append({"NZ": nz, "K": K, "us_per_timestep": us_call, "us_per_timestep_graph": us_graph,
+                        "path": {1: "simt", 2: "persistent", 3: "tensor"}.get(m.query(Q_LAST_PATH)),
+                        "paper_fpga_us_any_K": 1e3 * PAPER_FPGA_MS[nz]})
+        m.sync()
+        del m
+    return {"workload": w.name, "dtype": "f32", "T": w.T, "B": w.B, "points": out,
+            "note": "paper figure: Xilinx ZC706 FPGA at 100 MHz, K chosen per KL bound (Table I); context only"}
 
 
 def run_profile(args):

@@ -42,6 +42,12 @@ struct LayerStore {
   int mask_words = 0;
   int Kset[4] = {0, 0, 0, 0};
   int nz[4] = {0, 0, 0, 0};
+  // compressed x part (fp32 factors): device CSR per gate and its host offsets
+  int* xoff[4] = {nullptr, nullptr, nullptr, nullptr};
+  int* xidx[4] = {nullptr, nullptr, nullptr, nullptr};
+  float* xval[4] = {nullptr, nullptr, nullptr, nullptr};
+  size_t xcap[4] = {0, 0, 0, 0};  // entries allocated in xidx / xval
+  std::vector<int> xoff_h[4];
   bool maps_ready = false;  // tensor maps of Vx, Vh, U (bf16 path), built on first use
   TcMap map_vx, map_vh, map_u;
 };
@@ -104,6 +110,17 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
 // memory (deterministic).  Needs D % 8 == 0 and 16-byte aligned rows; a
 // staged load that does not complete within limit_ns sets *err.
 bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16);
+
+// Compressed x part of the pruned v (fp32 factors): per gate, the kept x
+// columns of row k are entries off[g][k] .. off[g][k+1] of idx[g] / val[g].
+struct SparseXRows {
+  const int* off[4];
+  const int* idx[4];
+  const float* val[4];
+};
+// The same product from the compressed rows, for T*B <= 32 columns.
+cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const float* X, int ldxin, int N, float* out,
+                                int ldo, cudaStream_t s);
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
                                  int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s);
 

@@ -220,7 +220,75 @@ cudaError_t launch_typed(const TF* A, int lda, int K, int Ks, const float* X, in
   }
 }
 
+// ---------------------------------------------------------------------------
+// compressed variant for very sparse v (few kept x columns per row): one warp
+// per packed row walks its kept entries (value, column) and gathers the x
+// values; lane partials are summed by a transposed butterfly, so lane l ends
+// with column l >> (5 - log2 NC) of the row
+// ---------------------------------------------------------------------------
+template <int NV>
+__device__ __forceinline__ void lanes_transpose_sum(float (&v)[NV], int lane) {
+  constexpr int kSteps = NV == 32 ? 5 : NV == 16 ? 4 : NV == 8 ? 3 : NV == 4 ? 2 : NV == 2 ? 1 : 0;
+#pragma unroll
+  for (int st = 0; st < kSteps; ++st) {
+    const int half = NV >> (st + 1);
+    const int mask = 16 >> st;
+    const bool upper = (lane & mask) != 0;
+#pragma unroll
+    for (int i = 0; i < half; ++i) {
+      const float keep = upper ? v[i + half] : v[i];
+      const float send = upper ? v[i] : v[i + half];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
+    }
+  }
+#pragma unroll
+  for (int mask = 16 >> kSteps; mask > 0; mask >>= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], mask);
+}
+
+template <int NC>
+__global__ void __launch_bounds__(256) xproj_sparse_kernel(SparseXRows sr, int K, int Ks, const float* __restrict__ X,
+                                                           int ldxin, int N, float* __restrict__ out, int ldo) {
+  griddep_launch_dependents();  // the recurrence kernel may start its set-up
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);  // packed row (g, k)
+  if (r >= 4 * K) return;
+  const int g = r / K, k = r - g * K;
+  const int beg = __ldg(sr.off[g] + k), end = __ldg(sr.off[g] + k + 1);
+  float acc[NC];
+#pragma unroll
+  for (int n = 0; n < NC; ++n) acc[n] = 0.f;
+  for (int e = beg + lane; e < end; e += 32) {
+    const float v = __ldg(sr.val[g] + e);
+    const int c = __ldg(sr.idx[g] + e);
+#pragma unroll
+    for (int n = 0; n < NC; ++n)
+      if (n < N) acc[n] = fmaf(v, __ldg(X + (long long)n * ldxin + c), acc[n]);
+  }
+  lanes_transpose_sum<NC>(acc, lane);
+  constexpr int kShift = NC == 32 ? 0 : NC == 16 ? 1 : NC == 8 ? 2 : NC == 4 ? 3 : NC == 2 ? 4 : 5;
+  const int n = lane >> kShift;
+  if ((lane & ((1 << kShift) - 1)) == 0 && n < N) out[(long long)n * ldo + (long long)g * Ks + k] = acc[0];
+}
+
+template <int NC>
+cudaError_t launch_sparse_nc(const SparseXRows& sr, int K, int Ks, const float* X, int ldxin, int N, float* out,
+                             int ldo, cudaStream_t s) {
+  xproj_sparse_kernel<NC><<<(4 * K + 7) / 8, 256, 0, s>>>(sr, K, Ks, X, ldxin, N, out, ldo);
+  return cudaGetLastError();
+}
+
 }  // namespace
+
+cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const float* X, int ldxin, int N, float* out,
+                                int ldo, cudaStream_t s) {
+  if (N <= 1) return launch_sparse_nc<1>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  if (N <= 2) return launch_sparse_nc<2>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  if (N <= 4) return launch_sparse_nc<4>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  if (N <= 8) return launch_sparse_nc<8>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  if (N <= 16) return launch_sparse_nc<16>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  if (N <= 32) return launch_sparse_nc<32>(sr, K, Ks, X, ldxin, N, out, ldo, s);
+  return cudaErrorInvalidValue;
+}
 
 bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16) {
   // bulk copies need 16-byte aligned rows and lengths

@@ -177,6 +177,18 @@ void clear_timing(lstm_approx_t* h) {
   h->timing.phase.clear();
 }
 
+// The compressed x projection pays when v keeps at most 1/8 of the x columns
+// (fp32 factors, few columns).
+bool sparse_x_projection(const lstm_approx_t* h, const LayerStore& s, int K, int N) {
+  if (h->dtype != LSTM_APPROX_FP32 || N > 32) return false;
+  long long kept = 0;
+  for (int g = 0; g < 4; ++g) {
+    if (s.xoff[g] == nullptr || (int)s.xoff_h[g].size() <= K) return false;
+    kept += s.xoff_h[g][K];
+  }
+  return kept * 8 <= 4LL * K * s.D;
+}
+
 // The tensor path takes bf16 factors; its intermediate depths must fall on
 // the 16-term slices of one MMA instruction.
 bool tensor_path_fits(const lstm_approx_t* h, const Checkpoints& ck) {
@@ -351,7 +363,16 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
     {
       PhaseTimer pt(h, 0);
-      if (xproj_cluster_fits(T * B, s.D, s.ldx, s.D, bf16))
+      if (sparse_x_projection(h, s, K, T * B)) {
+        SparseXRows sr;
+        for (int g = 0; g < 4; ++g) {
+          sr.off[g] = s.xoff[g];
+          sr.idx[g] = s.xidx[g];
+          sr.val[g] = s.xval[g];
+        }
+        LA_CUDA(h, launch_xproj_sparse(sr, K, h->Ks, in, s.D, T * B, h->Px, (int)ldp, h->stream),
+                "input projection launch");
+      } else if (xproj_cluster_fits(T * B, s.D, s.ldx, s.D, bf16))
         LA_CUDA(h,
                 launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->err,
                                      h->opt_wait_limit_us * 1000LL, h->stream),
@@ -566,6 +587,40 @@ int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz
           cudaMemcpy(s.mask + row0 * s.mask_words, mask.data(), mask.size() * sizeof(uint32_t),
                      cudaMemcpyHostToDevice),
           "factor upload");
+  if (!bf16) {  // the x part again, compressed: kept (column, value) runs of every row k
+    std::vector<int> off(Ks + 1, 0), cols;
+    std::vector<float> vals;
+    for (int k = 0; k < K; ++k) {
+      for (int m = 0; m < nz; ++m) {
+        const int c = v_idx[(size_t)k * nz + m];
+        if (c >= D) break;  // indices ascend: the h columns follow
+        cols.push_back(c);
+        vals.push_back(static_cast<float>(v_val[(size_t)k * nz + m]));
+      }
+      off[k + 1] = static_cast<int>(cols.size());
+    }
+    for (int k = K; k < Ks; ++k) off[k + 1] = off[K];
+    const size_t n = cols.size() > 0 ? cols.size() : 1;
+    if (n > s.xcap[gate] || s.xoff[gate] == nullptr) {
+      dfree(h, s.xidx[gate], s.xcap[gate] * 4);
+      dfree(h, s.xval[gate], s.xcap[gate] * 4);
+      s.xidx[gate] = nullptr;
+      s.xval[gate] = nullptr;
+      s.xcap[gate] = 0;
+      int rc = dmalloc(h, reinterpret_cast<void**>(&s.xidx[gate]), n * 4, "compressed factor storage");
+      if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.xval[gate]), n * 4, "compressed factor storage");
+      if (!rc && s.xoff[gate] == nullptr)
+        rc = dmalloc(h, reinterpret_cast<void**>(&s.xoff[gate]), (Ks + 1) * 4ull, "compressed factor storage");
+      if (rc) return rc;
+      s.xcap[gate] = n;
+    }
+    LA_CUDA(h, cudaMemcpy(s.xoff[gate], off.data(), off.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+    if (!cols.empty()) {
+      LA_CUDA(h, cudaMemcpy(s.xidx[gate], cols.data(), cols.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+      LA_CUDA(h, cudaMemcpy(s.xval[gate], vals.data(), vals.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+    }
+    s.xoff_h[gate] = off;
+  }
   s.Kset[gate] = K;
   s.nz[gate] = nz;
   return LSTM_APPROX_OK;
@@ -669,6 +724,11 @@ void lstm_approx_destroy(lstm_approx_t* h) {
     cudaFree(s.sigma);
     cudaFree(s.bias);
     cudaFree(s.mask);
+    for (int g = 0; g < 4; ++g) {
+      cudaFree(s.xoff[g]);
+      cudaFree(s.xidx[g]);
+      cudaFree(s.xval[g]);
+    }
   }
   cudaFree(h->h_state);
   cudaFree(h->c_state);

@@ -73,6 +73,21 @@ def test_latency_workload_progressive_outputs_in_one_run(cuda_device):
     assert_parity(got, ref, FP32_TOL)
 
 
+@pytest.mark.parametrize("keep", WORKLOADS["f1"].keeps)
+@pytest.mark.parametrize("K", [4, 16])
+def test_paper_case_study_shape(cuda_device, keep, K):
+    """The paper's case-study LSTM (Sec. VI): H = R = 64, C = 8320, fp32, NZ =
+    4160 / 130 / 32, oracle-decomposed factors, three steps of one stream."""
+    w = WORKLOADS["f1"]
+    layers = [list(decomposed_layer("f1", 0, 16, keep))]
+    x = draw_inputs(3, 1, w.D, w.x_dist, 8320 + K)
+    cps = [5, 8] if K == 16 else [2]
+    got, m = run_gpu(layers, x, K, checkpoints=cps, max_rank=16)
+    assert m.query(Q_LAST_PATH) == PATH_PERSISTENT
+    ref = oracle_run(layers, x, K, checkpoints=cps)
+    assert_parity(got, ref, FP32_TOL)
+
+
 @pytest.mark.parametrize("cs", [1, 2, 4, 8, 16])
 def test_every_cluster_size_agrees(cuda_device, cs):
     D, H, T, K = 96, 64, 5, 64

@@ -30,7 +30,7 @@ GATES = ("i", "f", "g", "o")
 class Workload:
     """One LSTM workload: sizes, factor dtype, approximation levels."""
 
-    index: int            # 1..5, used in the seeds
+    index: int            # 1..6, used in the seeds
     name: str
     D: int                # input size of layer 0
     H: int                # hidden size (R in the paper)
@@ -62,6 +62,11 @@ WORKLOADS = {
                    (0.5, 0.1), (8, 32, 128, 512), (), "uniform"),
     "c5": Workload(5, "lstm2-d4096-h2048-t16-b64-bf16", 4096, 2048, 16, 64, 2, "bf16",
                    (0.3,), (1024,), (16, 64, 256, 1024), "uniform"),
+    # the paper's case-study LSTM (Sec. VI): R = 64 hidden units, C = 8320
+    # columns per gate, one timestep of one stream, fp32; NZ = 4160 (no
+    # pruning of half the columns), 130 and 32 kept entries per v
+    "f1": Workload(6, "lstm-d8256-h64-t1-b1-fp32", 8256, 64, 1, 1, 1, "fp32",
+                   (0.5, 130 / 8320, 32 / 8320), (1, 4, 16, 64), (), "relu"),
 }
 
 
