@@ -309,6 +309,7 @@ def run_ours(args):
     # ---- large-batch tensor-core path (bf16 factors) -------------------------
     large = [] if (args.quick or args.no_large) else large_batch_sweep(dev, stream, peaks_bf16())
     paper_case = None if (args.quick or args.no_large) else paper_case_sweep(dev, stream)
+    dense = None if args.quick else dense_comparator(dev, stream, x)
 
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
@@ -360,6 +361,7 @@ def run_ours(args):
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
             "large_batch": large,
             "paper_case_study": paper_case,
+            "dense_lstm_comparator": dense,
         }
         if ws == 1 and not (args.no_cpu_baseline or args.quick):
             line["cpu_baseline"] = cpu_baseline()
@@ -429,6 +431,29 @@ def large_batch_sweep(dev, stream, peak):
         del m, x, oh, ck
         torch.cuda.empty_cache()
     return out
+
+
+def dense_comparator(dev, stream, x, steps: int = 200) -> dict:
+    """A dense fp32 LSTM layer of the benchmark shape (torch.nn.LSTM, the
+    library cuDNN/cuBLAS step) on the same input: the analogue of the paper's
+    dense baselines, for the speed-up of the approximation.  Not part of the
+    timed path."""
+    import torch
+    T, B, D = x.shape
+    lstm = torch.nn.LSTM(D, WL.H).to(dev).float()
+    with torch.no_grad(), torch.cuda.stream(stream):
+        for _ in range(10):
+            lstm(x)
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in evs:
+            a.record(stream)
+            lstm(x)
+            b.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+    return {"kind": "dense torch.nn.LSTM (cuDNN), fp32, same D/H/T/B, warm caches", "ms_per_run": ms,
+            "value": T * B / (ms / 1e3), "unit": UNIT,
+            "dense_weight_bytes": 4 * 4 * WL.H * (D + WL.H)}
 
 
 # the paper's FPGA latencies for one timestep of its case-study LSTM (Table I),

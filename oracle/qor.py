@@ -1,0 +1,97 @@
+"""Quality of result of the approximation against the dense LSTM (oracle side).
+
+TEST AND ANALYSIS INFRASTRUCTURE ONLY, like the rest of this package.
+
+The paper measures the quality of an approximation as the KL divergence of
+the driving model's output distribution from the dense model's (Sec. VI),
+which needs the trained model and its data.  This module measures the same
+kind of curve on the seeded synthetic workloads: the LSTM is run once with
+its dense gate matrices W (Sec. II) and once with the K-term refinement of
+Eq. 1 at each pruning level, and for every (NZ, K) it reports
+
+* the relative error of the hidden states, ||h~ - h|| / ||h|| over all t;
+* the KL divergence KL(p || p~) of softmax(A h_t), averaged over t, for a
+  seeded random linear head A (classes x H, N(0, 1/sqrt(H))) standing in
+  for the model's output layer;
+* the operations per timestep of Sec. III, 4 gates x K (2R + 2NZ + 1),
+  against the dense 4 x 2RC.
+
+``python -m oracle.qor`` prints the tables for the small workload and the
+paper's case-study shape.
+"""
+from __future__ import annotations
+
+import sys
+from typing import Dict, List, Sequence
+
+import numpy as np
+
+from .factors import decompose_gate
+from .recurrence import lstm_cell, op_count, run_lstm
+
+
+def dense_lstm(weights: Sequence[np.ndarray], x: np.ndarray) -> np.ndarray:
+    """h_t of the dense LSTM of Sec. II: y_g = W_g [x_t; h_{t-1}], h0 = c0 = 0."""
+    T, B, _ = x.shape
+    H = weights[0].shape[0]
+    h = np.zeros((B, H))
+    c = np.zeros((B, H))
+    out = np.zeros((T, B, H))
+    for t in range(T):
+        xt = np.concatenate([x[t], h], axis=1)          # [B][C]
+        y = [xt @ W.T for W in weights]                 # four [B][H]
+        h, c = lstm_cell(y, c)
+        out[t] = h
+    return out
+
+
+def softmax(z: np.ndarray) -> np.ndarray:
+    z = z - z.max(axis=-1, keepdims=True)
+    e = np.exp(z)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def qor_table(weights: Sequence[np.ndarray], x: np.ndarray, nzs: Sequence[int], Ks: Sequence[int],
+              classes: int = 10, seed: int = 1905) -> List[Dict]:
+    """One row per (NZ, K): relative h error, head KL, ops per timestep."""
+    H, C = weights[0].shape
+    h_ref = dense_lstm(weights, x)
+    A = np.random.Generator(np.random.PCG64(seed)).normal(0.0, 1.0 / np.sqrt(H), (classes, H))
+    p_ref = softmax(h_ref @ A.T)
+    rows = []
+    for nz in nzs:
+        layer = [decompose_gate(W, max(Ks), nz) for W in weights]
+        for K in Ks:
+            h = run_lstm([layer], x, K)["h"]
+            p = softmax(h @ A.T)
+            kl = float(np.mean(np.sum(p_ref * (np.log(p_ref) - np.log(p)), axis=-1)))
+            rows.append({"NZ": nz, "K": K,
+                         "rel_h_error": float(np.linalg.norm(h - h_ref) / np.linalg.norm(h_ref)),
+                         "head_kl": kl,
+                         "ops": 4 * op_count(H, nz, K), "dense_ops": 4 * 2 * H * C})
+    return rows
+
+
+def markdown(rows: List[Dict]) -> str:
+    lines = ["| NZ | K | rel. h error | head KL | ops / step | fraction of dense ops |", "|---|---|---|---|---|---|"]
+    for r in rows:
+        lines.append(f"| {r['NZ']} | {r['K']} | {r['rel_h_error']:.3g} | {r['head_kl']:.3g} | {r['ops']} | "
+                     f"{r['ops'] / r['dense_ops']:.3g} |")
+    return "\n".join(lines)
+
+
+def main(argv: Sequence[str]) -> None:
+    from workloads import WORKLOADS, draw_inputs, draw_weights, nz_from_keep
+    for name, T in (("c1", 8), ("f1", 4)):
+        w = WORKLOADS[name]
+        weights = draw_weights(w, 0)
+        x = draw_inputs(T, 1, w.D, w.x_dist, 4242)
+        nzs = [nz_from_keep(k, w.C()) for k in w.keeps] if name == "f1" else [w.C(), nz_from_keep(0.5, w.C()),
+                                                                              nz_from_keep(0.125, w.C())]
+        print(f"## {w.name} (H={w.H}, C={w.C()}, T={T})\n")
+        print(markdown(qor_table(weights, x, nzs, w.Ks)))
+        print()
+
+
+if __name__ == "__main__":
+    main(sys.argv[1:])
