@@ -21,5 +21,6 @@ Everything is float64 with plain loops; NumPy's SVD, sort and dot serve as
 library steps.  Pins against the paper and the mathematics live in
 ``tests/test_oracle_*.py``.
 """
-from .factors import decompose_gate, decompose_layer, prune, top_triplet, reconstruct  # noqa: F401
+from .factors import (decompose_gate, decompose_gate_variant, decompose_layer, prune, prune_dense,  # noqa: F401
+                      reconstruct, top_triplet)
 from .recurrence import run_lstm, lstm_cell, refinement_sums, op_count  # noqa: F401

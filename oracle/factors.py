@@ -87,6 +87,54 @@ def decompose_gate(W: np.ndarray, K: int, nz: int, return_residual_norms: bool =
     return out
 
 
+def prune_dense(a: np.ndarray, n: int) -> np.ndarray:
+    """a with all but its n largest-magnitude entries set to zero (same
+    ranking as prune)."""
+    i, p = prune(a, n)
+    out = np.zeros_like(np.asarray(a, dtype=np.float64))
+    out[i] = p
+    return out
+
+
+def decompose_gate_variant(W: np.ndarray, K: int, nz: int, residual: bool = True, nz_u: int = 0) -> dict:
+    """Variants of the scheme around Eq. 1, in the same output format.
+
+    residual=False: the non-residual scheme Sec. III contrasts with Eq. 1 --
+    the first K singular triplets of W itself (truncated SVD), each v pruned
+    to nz.  nz_u > 0 additionally keeps only the nz_u largest-magnitude
+    entries of each u (stored dense, zeros elsewhere); in the residual scheme
+    the pruned u enters the running approximation W~.  residual=True,
+    nz_u=0 is decompose_gate.
+    """
+    W = np.asarray(W, dtype=np.float64)
+    R_rows, C = W.shape
+    sigma = np.empty(K)
+    u = np.empty((K, R_rows))
+    idx = np.empty((K, nz), dtype=np.int32)
+    val = np.empty((K, nz))
+    if not residual:
+        U_all, s_all, Vt_all = np.linalg.svd(W, full_matrices=False)
+        if K > s_all.shape[0]:
+            raise ValueError(f"K={K} above the rank bound {s_all.shape[0]}")
+    W_tilde = np.zeros_like(W)
+    for n in range(K):
+        if residual:
+            s_n, u_n, v_n = top_triplet(W - W_tilde)
+        else:  # n-th triplet of W, with the sign convention of top_triplet
+            s_n, u_n, v_n = float(s_all[n]), U_all[:, n].copy(), Vt_all[n].copy()
+            a = np.abs(v_n)
+            if v_n[int(np.flatnonzero(a == a.max())[0])] < 0:
+                u_n, v_n = -u_n, -v_n
+        if nz_u > 0:
+            u_n = prune_dense(u_n, nz_u)
+        i_n, p_n = prune(v_n, nz)
+        v_pruned = np.zeros(C)
+        v_pruned[i_n] = p_n
+        W_tilde = W_tilde + s_n * np.outer(u_n, v_pruned)
+        sigma[n], u[n], idx[n], val[n] = s_n, u_n, i_n, p_n
+    return {"sigma": sigma, "u": u, "idx": idx, "val": val}
+
+
 def decompose_layer(weights, K: int, nz: int) -> List[dict]:
     """decompose_gate for the four gate matrices (i, f, g, o) of one layer."""
     return [decompose_gate(W, K, nz) for W in weights]

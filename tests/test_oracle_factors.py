@@ -124,3 +124,52 @@ def test_rank1_keep1_is_top_svd_term():
     f = F.decompose_gate(W, 1, 30)
     U, s, Vt = np.linalg.svd(W, full_matrices=False)
     assert np.allclose(F.reconstruct(f, 1, 30), s[0] * np.outer(U[:, 0], Vt[0]), atol=1e-13)
+
+
+# ---- variants of the scheme (non-residual truncated SVD, pruned u) --------
+
+def test_variant_default_is_the_residual_scheme():
+    from oracle import decompose_gate_variant
+    W = np.random.default_rng(11).standard_normal((6, 14))
+    a = F.decompose_gate(W, 4, 5)
+    b = decompose_gate_variant(W, 4, 5)
+    for key in ("sigma", "u", "idx", "val"):
+        np.testing.assert_array_equal(a[key], b[key])
+
+
+def test_unpruned_residual_equals_truncated_svd():
+    """Without pruning, the residual of a rank-n truncation has the (n+1)-th
+    singular triplet of W as its top one (Eckart-Young), so both schemes
+    give the same terms."""
+    from oracle import decompose_gate_variant
+    W = np.random.default_rng(12).standard_normal((5, 9))
+    a = decompose_gate_variant(W, 5, 9, residual=True)
+    b = decompose_gate_variant(W, 5, 9, residual=False)
+    np.testing.assert_allclose(a["sigma"], b["sigma"], rtol=1e-12)
+    np.testing.assert_allclose(np.abs(np.einsum("ki,ki->k", a["u"], b["u"])), 1.0, rtol=1e-10)
+    np.testing.assert_allclose(a["val"], b["val"], rtol=1e-9, atol=1e-12)
+
+
+def test_pruned_residual_beats_pruned_truncated_svd():
+    """With pruning, the residual scheme re-fits what pruning dropped, so its
+    approximation error after K terms is lower than pruning the truncated
+    SVD's vectors -- on average and on most draws (it is greedy, so not on
+    every one)."""
+    from oracle import decompose_gate_variant
+    ratios = []
+    for seed in range(10):
+        W = np.random.default_rng(100 + seed).standard_normal((8, 24))
+        a = decompose_gate_variant(W, 6, 6, residual=True)
+        b = decompose_gate_variant(W, 6, 6, residual=False)
+        ratios.append(np.linalg.norm(W - F.reconstruct(a, 6, 24)) / np.linalg.norm(W - F.reconstruct(b, 6, 24)))
+    ratios = np.array(ratios)
+    assert ratios.mean() < 0.97 and np.count_nonzero(ratios < 1.0) >= 8, ratios
+
+
+def test_pruned_u_keeps_the_largest_entries():
+    from oracle import decompose_gate_variant, prune_dense
+    W = np.random.default_rng(13).standard_normal((10, 12))
+    f = decompose_gate_variant(W, 3, 12, nz_u=4)
+    for n in range(3):
+        assert np.count_nonzero(f["u"][n]) == 4
+    np.testing.assert_array_equal(prune_dense(np.array([0.1, -3.0, 2.0, 2.0]), 2), [0.0, -3.0, 2.0, 0.0])

@@ -88,6 +88,21 @@ def test_paper_case_study_shape(cuda_device, keep, K):
     assert_parity(got, ref, FP32_TOL)
 
 
+@pytest.mark.parametrize("residual,nz_u", [(True, 16), (False, 0), (False, 24)])
+def test_scheme_variants(cuda_device, residual, nz_u):
+    """Factors of the scheme's variants (pruned u, non-residual truncated SVD)
+    go through the same path: the kernels take any factor set."""
+    import oracle
+    from workloads import draw_weights, nz_from_keep
+    w = WORKLOADS["c1"]
+    K, nz = 32, nz_from_keep(0.5, w.C())
+    gates = [oracle.decompose_gate_variant(W, K, nz, residual=residual, nz_u=nz_u) for W in draw_weights(w, 0)]
+    x = workload_inputs(w)
+    got, _ = run_gpu([gates], x, K, checkpoints=[8, 20])
+    ref = oracle_run([gates], x, K, checkpoints=[8, 20])
+    assert_parity(got, ref, FP32_TOL)
+
+
 @pytest.mark.parametrize("cs", [1, 2, 4, 8, 16])
 def test_every_cluster_size_agrees(cuda_device, cs):
     D, H, T, K = 96, 64, 5, 64
