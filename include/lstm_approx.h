@@ -200,7 +200,9 @@ enum lstm_approx_query_key {
   LSTM_APPROX_Q_LAUNCHES = 0,    /* kernels launched by this handle so far */
   LSTM_APPROX_Q_LAST_PATH = 1,   /* recurrence path of the last run (enum below) */
   LSTM_APPROX_Q_CLUSTER = 2,     /* CTAs per cluster of the last persistent run */
-  LSTM_APPROX_Q_DEVICE_BYTES = 3 /* device bytes currently held by the handle */
+  LSTM_APPROX_Q_DEVICE_BYTES = 3, /* device bytes currently held by the handle */
+  LSTM_APPROX_Q_PERSISTENT_VARIANT = 4 /* persistent kernel of the last persistent run
+                                          (1 or 2, see LSTM_APPROX_OPT_PERSISTENT_VARIANT) */
 };
 enum lstm_approx_path {
   LSTM_APPROX_PATH_NONE = 0,
@@ -215,8 +217,16 @@ enum lstm_approx_option_key {
   LSTM_APPROX_OPT_CLUSTER = 1,      /* 0 = automatic, else 1, 2, 4, 8 or 16 */
   LSTM_APPROX_OPT_TIMING = 2,       /* 1 = record CUDA events around each phase */
   LSTM_APPROX_OPT_WAIT_LIMIT = 3,   /* bounded-wait limit in polls (default 2^26) */
-  LSTM_APPROX_OPT_TEST_STALL = 4    /* 1 = next persistent run waits on a signal
+  LSTM_APPROX_OPT_TEST_STALL = 4,   /* 1 = next persistent run waits on a signal
                                        nobody sends (exercises ETIMEOUT) */
+  LSTM_APPROX_OPT_PERSISTENT_VARIANT = 5 /* persistent kernel: 0 = automatic (the
+                                       one-exchange kernel where it fits and
+                                       H x terms per CTA <= 16384, else the
+                                       per-unit-block one),
+                                       1 = per-unit-block kernel (two cluster
+                                       exchanges per timestep, any H <= 1024),
+                                       2 = one-exchange kernel (H <= 512,
+                                       K <= 256, cluster of 4, 8 or 16) */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 

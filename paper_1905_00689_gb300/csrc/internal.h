@@ -84,11 +84,11 @@ struct lstm_approx {
   char* stage = nullptr;
 
   // options and counters
-  int opt_force_path = 0, opt_cluster = 0;
+  int opt_force_path = 0, opt_cluster = 0, opt_persistent_variant = 0;
   long long opt_wait_limit_us = 2000000;
   int opt_test_stall = 0;
   long long launches = 0;
-  int last_path = 0, last_cluster = 0;
+  int last_path = 0, last_cluster = 0, last_variant = 0;
   long long device_bytes = 0;
   lstm_approx_impl::Timing timing;
   std::string last_error;
@@ -180,6 +180,36 @@ struct PersistentArgs {
   int test_stall;
 };
 cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s);
+
+// One-exchange variant (H <= 512, K <= 256): each CTA owns a range of one
+// gate's terms, and the CTAs swap partial gate sums once per timestep.
+struct PersistentAgPlan {
+  int CS = 0;       // CTAs per cluster (4, 8 or 16)
+  int RA = 0;       // terms per CTA (a multiple of 4, at most 64)
+  int Kp = 0;       // terms per gate rounded up to CS
+  int UB = 0;       // units per output block (a multiple of 4)
+  int nmask = 0;    // intermediate depths that cut a CTA's range
+  int tcols = 0;    // tensor-memory columns (V_h rows, then U)
+  int hq = 0;       // h quads per lane in the recurrent product (1, 2 or 4)
+  size_t smem = 0;  // dynamic shared memory bytes
+};
+bool plan_persistent_ag(int H, int K, const Checkpoints& ck, int want_cs, PersistentAgPlan* plan,
+                        std::string* why);
+cudaError_t launch_persistent_ag(const PersistentAgPlan& plan, const PersistentArgs& a, cudaStream_t s);
+
+// Either persistent kernel: variant 1 = per-unit-block kernel (two
+// exchanges per step), 2 = one-exchange kernel; 0 picks the one-exchange
+// kernel where it fits and a CTA's share (H x terms per CTA) is small, else
+// the per-unit-block one.
+struct PersistentChoice {
+  int variant = 0;
+  int CS = 0;
+  PersistentPlan ub;
+  PersistentAgPlan ag;
+};
+bool choose_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, int sm_count, int variant,
+                       PersistentChoice* c, std::string* why);
+cudaError_t launch_persistent_choice(const PersistentChoice& c, const PersistentArgs& a, cudaStream_t s);
 
 // ---- tensor-core path (bf16, tcgen05 / TMEM / TMA) -----------------------
 

@@ -333,17 +333,18 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     const Checkpoints& lck = top ? ck : none;
     // recurrence path
     int path = h->opt_force_path;
-    PersistentPlan plan;
+    PersistentChoice plan;
     std::string why;
     const bool tensor_ok = bf16 && tensor_path_fits(h, lck);
     if (path == 0) {
       path = LSTM_APPROX_PATH_SIMT;
       if (tensor_ok) path = LSTM_APPROX_PATH_TENSOR;
-      else if (!bf16 && B <= 8 && plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+      else if (!bf16 && B <= 8 &&
+               choose_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, h->opt_persistent_variant, &plan, &why))
         path = LSTM_APPROX_PATH_PERSISTENT;
     } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
       if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
-      if (!plan_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, &plan, &why))
+      if (!choose_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, h->opt_persistent_variant, &plan, &why))
         return fail(h, LSTM_APPROX_EINVAL, "persistent path unavailable: %s", why.c_str());
     } else if (path == LSTM_APPROX_PATH_TENSOR) {
       if (!tensor_ok)
@@ -409,9 +410,10 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
       a.wait_limit_ns = h->opt_wait_limit_us * 1000LL;
       a.test_stall = h->opt_test_stall;
       h->opt_test_stall = 0;
-      LA_CUDA(h, launch_persistent(plan, a, h->stream), "persistent kernel launch");
+      LA_CUDA(h, launch_persistent_choice(plan, a, h->stream), "persistent kernel launch");
       h->launches += 1;
       h->last_cluster = plan.CS;
+      h->last_variant = plan.variant;
     } else {
       float* hs = h->h_state + (size_t)l * h->max_batch * H;
       float* cs = h->c_state + (size_t)l * h->max_batch * H;
@@ -750,6 +752,7 @@ int lstm_approx_query(const lstm_approx_t* h, int key, long long* value) {
     case LSTM_APPROX_Q_LAST_PATH: *value = h->last_path; return LSTM_APPROX_OK;
     case LSTM_APPROX_Q_CLUSTER: *value = h->last_cluster; return LSTM_APPROX_OK;
     case LSTM_APPROX_Q_DEVICE_BYTES: *value = h->device_bytes; return LSTM_APPROX_OK;
+    case LSTM_APPROX_Q_PERSISTENT_VARIANT: *value = h->last_variant; return LSTM_APPROX_OK;
     default: return LSTM_APPROX_EINVAL;
   }
 }
@@ -775,6 +778,10 @@ int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_TEST_STALL:
       h->opt_test_stall = value != 0;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_PERSISTENT_VARIANT:
+      if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad persistent variant %lld", value);
+      h->opt_persistent_variant = (int)value;
       return LSTM_APPROX_OK;
     default: return fail(h, LSTM_APPROX_EINVAL, "unknown option %d", key);
   }

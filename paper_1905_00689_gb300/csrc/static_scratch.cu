@@ -98,9 +98,9 @@ extern "C" int lstm_approx_run_static(const float* Vx, const float* Vh, const fl
   if (major != 10 || minor != 3) return report(msg, msg_len, LSTM_APPROX_ECUDA, "needs an sm_103 device");
   if (dev < 0 || dev >= kMaxDevices) return report(msg, msg_len, LSTM_APPROX_ECUDA, "device index %d too large", dev);
 
-  PersistentPlan plan;
+  PersistentChoice plan;
   std::string why;
-  if (!plan_persistent(H, K, T, ck, 0, sms, &plan, &why))
+  if (!choose_persistent(H, K, T, ck, 0, sms, 0, &plan, &why))
     return report(msg, msg_len, LSTM_APPROX_EINVAL, "shape does not fit: %s", why.c_str());
 
   float* base = nullptr;
@@ -149,7 +149,7 @@ extern "C" int lstm_approx_run_static(const float* Vx, const float* Vh, const fl
   a.ck = ck;
   a.wait_limit_ns = 2000000000LL;
   a.test_stall = 0;
-  e = launch_persistent(plan, a, s);
+  e = launch_persistent_choice(plan, a, s);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "recurrence launch: %s", cudaGetErrorString(e));
   e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "synchronise: %s", cudaGetErrorString(e));

@@ -10,7 +10,8 @@ import numpy as np
 import pytest
 
 from parity_util import FP32_TOL, assert_parity, oracle_run, run_gpu
-from paper_1905_00689_gb300 import LSTMApproxError, OPT_TEST_STALL, OPT_WAIT_LIMIT, PATH_PERSISTENT, Q_LAUNCHES
+from paper_1905_00689_gb300 import (LSTMApproxError, OPT_TEST_STALL, OPT_WAIT_LIMIT, PATH_PERSISTENT, Q_LAUNCHES,
+                                    Q_PERSISTENT_VARIANT)
 from workloads import draw_factor_set, draw_inputs
 
 pytestmark = pytest.mark.gpu
@@ -23,10 +24,12 @@ def _small():
     return [gates], x, K
 
 
-def test_bounded_wait_reports_timeout_and_context_survives(cuda_device):
+@pytest.mark.parametrize("variant", [1, 2])
+def test_bounded_wait_reports_timeout_and_context_survives(cuda_device, variant):
     import torch
     layers, x, K = _small()
-    got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT)
+    got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=variant)
+    assert m.query(Q_PERSISTENT_VARIANT) == variant
     m.set_option(OPT_WAIT_LIMIT, 50_000)        # 50 ms
     m.set_option(OPT_TEST_STALL, 1)
     xt = torch.from_numpy(x.astype(np.float32)).cuda()

@@ -1,0 +1,103 @@
+"""Both persistent kernels against the fp64 oracle (fp32, max relative error <= 1e-4).
+
+Variant 1 splits the hidden units over the cluster and exchanges tau' and
+h every timestep; variant 2 gives each CTA a range of one gate's terms and
+exchanges partial gate sums once per timestep, with every CTA running all
+cells.  The cases below pin each variant explicitly (the automatic choice
+only ever runs one of them for a shape): the two batch-1 workloads, every
+cluster size of variant 2, intermediate depths on and inside the term
+ranges (several inside one range, one at K), and ragged shapes.
+"""
+import numpy as np
+import pytest
+
+from parity_util import (FP32_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run, run_gpu,
+                         synthetic_layer, workload_inputs)
+from paper_1905_00689_gb300 import PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_PERSISTENT_VARIANT
+from workloads import draw_factor_set, draw_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(layers, x, K, variant, cluster=0, **kw):
+    got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=variant, cluster=cluster, **kw)
+    assert m.query(Q_LAST_PATH) == PATH_PERSISTENT
+    assert m.query(Q_PERSISTENT_VARIANT) == variant
+    if cluster:
+        assert m.query(Q_CLUSTER) == cluster
+    ref = oracle_run(layers, x, K, **{k: v for k, v in kw.items() if k in ("h0", "c0", "checkpoints")})
+    assert_parity(got, ref, FP32_TOL)
+    return got
+
+
+@pytest.mark.parametrize("variant", [1, 2])
+@pytest.mark.parametrize("K", [1, 16, 64])
+def test_small_workload(cuda_device, variant, K):
+    layers = [list(decomposed_layer("c1", 0, 64, 0.5))]
+    x = workload_inputs(WORKLOADS["c1"])
+    cps = [c for c in (1, 4, 16, 64) if c <= K]
+    got = _check(layers, x, K, variant, checkpoints=cps)
+    assert np.array_equal(got["ckpt_h"][-1], got["h"])
+
+
+@pytest.mark.parametrize("variant", [1, 2])
+@pytest.mark.parametrize("K,cps", [(256, [16, 64]), (256, [16, 64, 100, 255]), (64, [3, 17, 40]), (16, [4, 8])])
+def test_latency_workload_full_size(cuda_device, variant, K, cps):
+    """D=1024, H=512, T=20, B=1, keep 25%: the benchmark's launch configuration."""
+    layers = [list(synthetic_layer("c2", 0, 256, 0.25))]
+    x = workload_inputs(WORKLOADS["c2"])
+    _check(layers, x, K, variant, checkpoints=cps, max_rank=256)
+
+
+@pytest.mark.parametrize("cs", [4, 8, 16])
+@pytest.mark.parametrize("cps", [[8, 33], [1, 2, 3, 61, 64], [16, 32, 48]])
+def test_one_exchange_every_cluster_size(cuda_device, cs, cps):
+    """Cuts on range boundaries, inside ranges, several inside one range, at K."""
+    D, H, T, K = 96, 64, 5, 64
+    layers = [[draw_factor_set(H, D + H, K, 40, 900 + g) for g in range(4)]]
+    x = draw_inputs(T, 1, D, "relu", 21)
+    _check(layers, x, K, 2, cluster=cs, checkpoints=cps)
+
+
+@pytest.mark.parametrize("D,H,T,B,K,nz,cps", [
+    (5, 12, 3, 3, 7, 9, [1, 3, 5]),        # ragged sizes, unaligned depths, several streams
+    (24, 36, 4, 2, 1, 60, [1]),            # K = 1, nothing pruned (nz = C)
+    (40, 100, 2, 1, 50, 1, [25, 49]),      # one kept entry per term
+    (3, 4, 1, 1, 3, 2, []),                # T = 1
+    (64, 44, 6, 5, 33, 17, [2, 32, 33]),
+    (16, 508, 3, 2, 255, 30, [1, 100, 254]),  # H and K just under the one-exchange limits
+])
+@pytest.mark.parametrize("variant", [1, 2])
+def test_ragged_shapes(cuda_device, D, H, T, B, K, nz, cps, variant):
+    C = D + H
+    gates = [draw_factor_set(H, C, K, nz, 7000 + 13 * D + g) for g in range(4)]
+    rng = np.random.default_rng(D * H)
+    for g in gates:
+        g["bias"] = 0.3 * rng.standard_normal(H)
+    x = draw_inputs(T, B, D, "uniform", 55 + D)
+    h0 = 0.5 * rng.standard_normal((1, B, H))
+    c0 = 0.5 * rng.standard_normal((1, B, H))
+    _check([gates], x, K, variant, h0=h0, c0=c0, checkpoints=cps)
+
+
+def test_variants_agree_on_two_layers(cuda_device):
+    D, H, T, B, K = 48, 32, 5, 2, 12
+    layers = [[draw_factor_set(H, (D if l == 0 else H) + H, K, 20, 800 + 10 * l + g) for g in range(4)]
+              for l in range(2)]
+    x = draw_inputs(T, B, D, "uniform", 3)
+    for variant in (1, 2):
+        _check(layers, x, K, variant, checkpoints=[3, 12])
+
+
+def test_one_exchange_rejects_what_it_cannot_hold(cuda_device):
+    """H above 512 or K above 256: forcing variant 2 is an error, the automatic
+    choice falls back to variant 1."""
+    from paper_1905_00689_gb300 import LSTMApproxError
+    D, H, T, K = 16, 520, 2, 8
+    layers = [[draw_factor_set(H, D + H, K, 30, 50 + g) for g in range(4)]]
+    x = draw_inputs(T, 1, D, "uniform", 5)
+    with pytest.raises(LSTMApproxError):
+        run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=2)
+    got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT)
+    assert m.query(Q_PERSISTENT_VARIANT) == 1
+    assert_parity(got, oracle_run(layers, x, K), FP32_TOL)
