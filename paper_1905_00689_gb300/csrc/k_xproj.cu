@@ -6,12 +6,14 @@
 // the whole packed V_x is read once, so the kernel is about latency: every
 // CTA owns 32 rows and one of S chunks of D (S CTAs of a cluster along D).
 // It stages up to 256 values of D of its 32 rows of V_x and of the x columns
-// in shared memory with one bulk copy (TMA engine) per row, all in flight at
-// once and completing on one mbarrier; its 8 warps then split the staged
-// range again, each lane accumulating a 4-row x NC-column register tile.
-// The 8 warp partials are summed in shared memory in warp order and the S
-// chunk partials through distributed shared memory in chunk order, so the
-// result does not depend on timing.
+// in shared memory with 16-byte asynchronous copies spread over all its
+// threads, in two commit groups of 128 values, so that its 8 warps start on
+// the first half while the second is in flight; each lane accumulates a
+// 4-row x NC-column register tile.  The 8 warp partials are summed in shared memory in warp
+// order; each CTA then pushes its chunk sums of the outputs another CTA
+// finishes to that CTA (16-byte st.async completing the owner's mbarrier),
+// and the owner adds the S chunk sums in chunk order, so the result does not
+// depend on timing.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -25,8 +27,11 @@ constexpr int kCols = 32;     // max columns (T*B)
 constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kSub = 256;     // values of D staged per round
+constexpr int kHalf = kSub / 2;  // values per staged half (one mbarrier each)
 constexpr int kPadF = 4;      // floats of padding after each staged row
 constexpr int kMaxSplit = 8;  // CTAs per cluster along D
+constexpr int kHdr = 32;      // mbarrier of the incoming chunk sums
+static_assert(kRows * kCols == 4 * kThreads, "each thread pushes one float4 of chunk sums");
 
 template <typename TF>
 constexpr int v_stride() {  // staged V_x row stride in elements (16-byte multiple)
@@ -34,11 +39,51 @@ constexpr int v_stride() {  // staged V_x row stride in elements (16-byte multip
 }
 constexpr int kXStride = kSub + kPadF;
 
+// header | staged tiles (later the warp partials) | red [32*32] | slot [32*32]
 template <typename TF>
 constexpr size_t smem_bytes() {
   const size_t tiles = (size_t)kRows * v_stride<TF>() * sizeof(TF) + (size_t)kCols * kXStride * 4;
   const size_t parts = (size_t)kWarps * kRows * kCols * 4;
-  return 16 + (tiles > parts ? tiles : parts) + (size_t)kRows * kCols * 4;
+  return kHdr + (tiles > parts ? tiles : parts) + 2 * (size_t)kRows * kCols * 4;
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Issues the 16-byte copies of values [h0, h0 + hl) of the round at d0: the
+// CTA's rows of V_x and the N x columns.
+template <typename TF>
+__device__ __forceinline__ void stage_half(const TF* A, int lda, int K, int Ks, int row0, int vrows,
+                                           const float* X, int ldxin, int N, int d0, int h0, int hl, TF* vs,
+                                           float* xs, int tid) {
+  constexpr int VS = v_stride<TF>();
+  constexpr int kPer = 16 / (int)sizeof(TF);  // values per copy
+  const int vq = hl / kPer;
+  for (int i = tid; i < vrows * vq; i += kThreads) {
+    const int rr = i / vq, c = i - rr * vq;
+    const int r = row0 + rr;
+    const TF* src = A + (long long)((r / K) * Ks + r % K) * lda + d0 + h0 + c * kPer;
+    cp_async16(smem_u32(vs + rr * VS + h0 + c * kPer), src);
+  }
+  const int xq = hl / 4;
+  for (int i = tid; i < N * xq; i += kThreads) {
+    const int n = i / xq, c = i - n * xq;
+    cp_async16(smem_u32(xs + n * kXStride + h0 + 4 * c), X + (long long)n * ldxin + d0 + h0 + 4 * c);
+  }
+  cp_async_commit();
+}
+
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ float4 lds4(const float* p) { return *reinterpret_cast<const float4*>(p); }
@@ -46,12 +91,6 @@ __device__ __forceinline__ float4 lds4(const __nv_bfloat16* p) {
   const uint2 u = *reinterpret_cast<const uint2*>(p);
   return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u), __uint_as_float(u.y << 16),
                      __uint_as_float(u.y & 0xFFFF0000u));
-}
-
-__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
 }
 
 // Lane (rg = lane >> 2, cg = lane & 3) of every warp owns rows 4*rg .. 4*rg+3
@@ -62,11 +101,12 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
                                                          int dchunk, float* __restrict__ out, int ldo, int S,
                                                          int* err, long long limit_ns) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
-  TF* vs = reinterpret_cast<TF*>(smem_raw + 16);  // [32][v_stride]
-  float* xs = reinterpret_cast<float*>(smem_raw + 16 + (size_t)kRows * v_stride<TF>() * sizeof(TF));  // [32][kXStride]
-  float* part = reinterpret_cast<float*>(smem_raw + 16);  // [warp][n * 32 + r], after the last round
-  float* red = reinterpret_cast<float*>(smem_raw + smem_bytes<TF>() - (size_t)kRows * kCols * 4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0]: incoming chunk sums
+  TF* vs = reinterpret_cast<TF*>(smem_raw + kHdr);         // [32][v_stride]
+  float* xs = reinterpret_cast<float*>(smem_raw + kHdr + (size_t)kRows * v_stride<TF>() * sizeof(TF));  // [32][kXStride]
+  float* part = reinterpret_cast<float*>(smem_raw + kHdr);  // [warp][n * 32 + r], after the last round
+  float* red = reinterpret_cast<float*>(smem_raw + smem_bytes<TF>() - 2 * (size_t)kRows * kCols * 4);
+  float* slot = red + kRows * kCols;  // [S][opc]: chunk c's sums of the outputs this CTA finishes
   constexpr int VS = v_stride<TF>();
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -74,20 +114,22 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
   const int rb = blockIdx.x;
   const uint32_t q = S > 1 ? cluster_ctarank() : 0u;  // chunk of D
   const int nrows = 4 * K;
+  const int vrows = min(kRows, nrows - rb * kRows);
   const int c_lo = min(D, (int)q * dchunk), c_hi = min(D, c_lo + dchunk);
-  const uint32_t mb = smem_u32(bar);
+  const int opc = kRows * kCols / S;  // outputs finished per CTA
+  const uint32_t bar_red = smem_u32(&bars[0]);
+  const uint64_t limit = static_cast<uint64_t>(limit_ns);
 
   griddep_launch_dependents();  // the recurrence kernel may start its set-up
   if (tid == 0) {
-    mbar_init(mb, 1);
+    mbar_init(bar_red, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (S > 1) mbar_arrive_expect_tx(bar_red, (uint32_t)((S - 1) * opc * 4));
   }
-  // rows and columns that are never loaded read as zero
-  for (int i = tid; i < kRows * VS; i += kThreads)
-    if (rb * kRows + i / VS >= nrows) vs[i] = TF(0.f);
-  for (int i = tid; i < kCols * kXStride; i += kThreads)
-    if (i / kXStride >= N) xs[i] = 0.f;
   __syncthreads();
+  // the peers push their chunk sums only after this CTA's barrier is armed
+  // (their cluster wait below); arriving now hides the barrier's latency
+  if (S > 1) cluster_arrive_release();
 
   float acc[4][NC];
 #pragma unroll
@@ -96,46 +138,50 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
     for (int j = 0; j < NC; ++j) acc[i][j] = 0.f;
 
   bool ok = true;
-  uint32_t phase = 0;
   for (int d0 = c_lo; d0 < c_hi; d0 += kSub) {
     const int len = min(kSub, c_hi - d0);
-    const int vrows = min(kRows, nrows - rb * kRows);
-    if (tid == 0) mbar_arrive_expect_tx(mb, (uint32_t)(len * (vrows * (int)sizeof(TF) + N * 4)));
-    if (tid < vrows) {
-      const int r = rb * kRows + tid;
-      bulk_copy_g2s(smem_u32(vs + tid * VS), A + (long long)((r / K) * Ks + r % K) * lda + d0,
-                    (uint32_t)(len * sizeof(TF)), mb);
-    } else if (tid >= kRows && tid < kRows + N) {
-      const int n = tid - kRows;
-      bulk_copy_g2s(smem_u32(xs + n * kXStride), X + (long long)n * ldxin + d0, (uint32_t)(len * 4), mb);
+    const int l0 = min(kHalf, len), l1 = len - l0;  // multiples of 8 (D % 8 == 0)
+    stage_half(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, d0, 0, l0, vs, xs, tid);
+    stage_half(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, d0, kHalf, l1, vs, xs, tid);
+    if (d0 == c_lo) {
+      // rows and columns that are never loaded read as zero (filled while
+      // the first copies are in flight; disjoint from what they write)
+      for (int i = tid; i < kRows * VS; i += kThreads)
+        if (i / VS >= vrows) vs[i] = TF(0.f);
+      for (int i = tid; i < 4 * NC * kXStride; i += kThreads)
+        if (i / kXStride >= N) xs[i] = 0.f;
     }
-    ok = __syncthreads_and(ok && mbar_wait_bounded<false>(mb, phase, static_cast<uint64_t>(limit_ns), err));
-    phase ^= 1u;
-    if (!ok) break;
-    // this warp's share of the staged range, in multiples of 4
-    const int wlen = ((len + kWarps - 1) / kWarps + 3) & ~3;
-    const int e_lo = min(len, warp * wlen), e_hi = min(len, e_lo + wlen);
-    for (int e = e_lo; e < e_hi; e += 4) {
-      float4 va[4], xb[NC];
+#pragma unroll 1
+    for (int hf = 0; hf < 2; ++hf) {
+      const int hl = hf == 0 ? l0 : l1;
+      if (hl == 0) break;
+      if (hf == 0) cp_async_wait<1>();
+      else cp_async_wait<0>();
+      __syncthreads();  // every thread's copies of this half (and the zero fill) are visible
+      // this warp's share of the half, in multiples of 4
+      const int wlen = ((hl + kWarps - 1) / kWarps + 3) & ~3;
+      const int e_lo = hf * kHalf + min(hl, warp * wlen), e_hi = hf * kHalf + min(hl, warp * wlen + wlen);
+      for (int e = e_lo; e < e_hi; e += 4) {
+        float4 va[4], xb[NC];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) va[i] = lds4(vs + (4 * rg + i) * VS + e);
+        for (int i = 0; i < 4; ++i) va[i] = lds4(vs + (4 * rg + i) * VS + e);
 #pragma unroll
-      for (int j = 0; j < NC; ++j) xb[j] = lds4(xs + (cg * NC + j) * kXStride + e);
+        for (int j = 0; j < NC; ++j) xb[j] = lds4(xs + (cg * NC + j) * kXStride + e);
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+        for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < NC; ++j) {
-          float s = acc[i][j];
-          s = fmaf(va[i].x, xb[j].x, s);
-          s = fmaf(va[i].y, xb[j].y, s);
-          s = fmaf(va[i].z, xb[j].z, s);
-          s = fmaf(va[i].w, xb[j].w, s);
-          acc[i][j] = s;
-        }
+          for (int j = 0; j < NC; ++j) {
+            float s = acc[i][j];
+            s = fmaf(va[i].x, xb[j].x, s);
+            s = fmaf(va[i].y, xb[j].y, s);
+            s = fmaf(va[i].z, xb[j].z, s);
+            s = fmaf(va[i].w, xb[j].w, s);
+            acc[i][j] = s;
+          }
+      }
     }
     __syncthreads();  // the staged tiles are free for the next round (and the partials)
   }
-  if (!ok && tid == 0) atomicCAS(err, 0, kErrTcTimeout);
 
   // warp partials, then their sum in warp order
 #pragma unroll
@@ -152,25 +198,42 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
     for (int w = 0; w < kWarps; ++w) s += part[w * kRows * kCols + o];
     red[o] = s;
   }
+  __syncthreads();
   if (S > 1) {
-    cluster_sync_all();
-    // this CTA finishes outputs [q*OPC, (q+1)*OPC) from the S chunk sums, in chunk order
-    const int opc = kRows * kCols / S;
-    for (int i = tid; i < opc; i += kThreads) {
-      const int o = (int)q * opc + i;
-      const uint32_t la = smem_u32(&red[o]);
-      float s = 0.f;
-      for (int c = 0; c < S; ++c) s += ld_cluster_f32(mapa_shared(la, c));
-      const int n = o / kRows, r = rb * kRows + o % kRows;
-      if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = s;
+    cluster_wait_acquire();  // every CTA of the cluster has armed its barrier
+    // thread tid hands outputs 4 tid .. 4 tid + 3 to the CTA that finishes them
+    const int o = 4 * tid, owner = o / opc;
+    const float4 v = *reinterpret_cast<const float4*>(red + o);
+    float* dst = slot + q * opc + (o - owner * opc);
+    if (owner == (int)q) {
+      *reinterpret_cast<float4*>(dst) = v;
+    } else {
+      st_async_v4(mapa_shared(smem_u32(dst), (uint32_t)owner), v.x, v.y, v.z, v.w,
+                  mapa_shared(bar_red, (uint32_t)owner));
     }
-    cluster_sync_all();  // chunk sums stay readable until every CTA has summed
-  } else {
-    __syncthreads();
+    const bool got = mbar_wait_bounded<true>(bar_red, 0, limit, err);
+    if (!got) atomicCAS(err, 0, kErrTcTimeout);
+    ok = __syncthreads_and(ok && got);  // also publishes the local slot writes
+    if (ok) {
+      for (int i = tid; i < opc; i += kThreads) {
+        float s = 0.f;
+        for (int c = 0; c < S; ++c) s += slot[c * opc + i];
+        const int oo = (int)q * opc + i;
+        const int n = oo / kRows, r = rb * kRows + oo % kRows;
+        if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = s;
+      }
+    }
+  } else if (ok) {
     for (int o = tid; o < kRows * kCols; o += kThreads) {
       const int n = o / kRows, r = rb * kRows + o % kRows;
       if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = red[o];
     }
+  }
+  if (!ok) {
+    // a wait ran out: copies or pushes issued before it may still be in
+    // flight towards this CTA; let them land before it exits
+    const uint64_t t0 = global_timer_ns();
+    while (global_timer_ns() - t0 < 50000ull) __nanosleep(1000);
   }
 }
 
