@@ -22,6 +22,7 @@ scaling, no data-path collective); rank 0 prints one JSON line.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -46,6 +47,24 @@ K_MAIN = 256
 CKPTS = (16, 64)
 K_SWEEP = (16, 64, 256)
 L2_FLUSH_BYTES = 256 << 20
+
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of
+# the recurrence kernel on this workload, from the ncu capture summarised in
+# profiles/persistent_kernel_lstm-d1024-h512-t20-b1-fp32.md.  The figure
+# holds only for the kernel sources it was taken on: `captured_traffic`
+# returns None once their SHA-256 differs.
+TRAFFIC_SOURCES = ("k_persistent.cu", "ptx.cuh")
+TRAFFIC_CAPTURE = {"sha256": "5fad44ade109d4b8e5e2a79bf61a1bddcba7dacf5f37bb09ad27353f268ae365",
+                   "bytes": 4338944}
+
+
+def captured_traffic():
+    csrc = os.path.join(HERE, "paper_1905_00689_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in TRAFFIC_SOURCES:
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    return TRAFFIC_CAPTURE["bytes"] if h.hexdigest() == TRAFFIC_CAPTURE["sha256"] else None
 
 
 def _config(n_gpus: int) -> dict:
@@ -221,7 +240,8 @@ def run_reference(args):
 
 def run_ours(args):
     import torch
-    from paper_1905_00689_gb300 import LSTMApprox, OPT_TIMING, Q_CLUSTER, Q_LAST_PATH, Q_LAUNCHES
+    from paper_1905_00689_gb300 import (LSTMApprox, OPT_TIMING, Q_CLUSTER, Q_LAST_PATH, Q_LAUNCHES,
+                                        Q_PERSISTENT_VARIANT)
 
     ws, rank, local = _dist_env()
     dist = None
@@ -283,6 +303,7 @@ def run_ours(args):
     p50_ms = statistics.median(step_ms)
     path = m.query(Q_LAST_PATH)
     cluster = m.query(Q_CLUSTER)
+    variant = m.query(Q_PERSISTENT_VARIANT)
 
     # ---- per-phase device times (CUDA events on the library's stream) ------
     m.set_option(OPT_TIMING, 1)
@@ -352,12 +373,12 @@ def run_ours(args):
                     "d2h_bytes_per_step": int(oh.numel() * 4 + kh.numel() * 4)},
             "roofline": {"kernel": "persistent recurrence kernel", "bound": "hbm", "achieved": achieved,
                          "peak": hbm_peak, "peak_source": peak_note, "unit": "GB/s", "frac": achieved / hbm_peak,
-                         "traffic": None,
+                         "traffic": captured_traffic() if (path == 2 and variant == 1) else None,
                          "algorithmic_bytes_per_launch": rec_bytes, "launch_ms": rec_ms},
             "path_effective_gbs": path_bytes / (ms_max / 1e3) / 1e9,
             "phase_ms": {"input_projection": xproj_ms, "recurrence": rec_ms},
             "recurrence_path": {1: "simt", 2: "persistent", 3: "tensor"}.get(path, str(path)),
-            "cluster_ctas": cluster,
+            "cluster_ctas": cluster, "persistent_kernel": {1: "per-unit-block", 2: "one-exchange"}.get(variant),
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
             "large_batch": large,
             "paper_case_study": paper_case,

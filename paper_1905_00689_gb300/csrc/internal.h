@@ -78,6 +78,7 @@ struct lstm_approx {
   void* seq_bf16 = nullptr;   // [T*B][ldh] bf16 sequence between layers (tensor path)
   void* h_bf16 = nullptr;     // [max_batch][ldh] bf16 h operand (tensor path)
   int* err = nullptr;         // device status word (0 = ok)
+  int* err_host = nullptr;    // pinned host copy of it, read after the stream synchronises
 
   // staging for lstm_approx_run_host
   size_t stage_bytes = 0;

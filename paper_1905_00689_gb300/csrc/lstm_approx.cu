@@ -517,6 +517,8 @@ int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dim
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->c_state), state, "state");
   if (!rc) rc = dmalloc(h, &h->tau, (size_t)max_batch * 4 * h->Ks * sizeof(float), "scratch tau");
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->err), sizeof(int), "status word");
+  if (!rc && cudaHostAlloc(reinterpret_cast<void**>(&h->err_host), sizeof(int), cudaHostAllocDefault) != cudaSuccess)
+    rc = fail(h, LSTM_APPROX_ENOMEM, "pinned status word");
   if (!rc && dtype == LSTM_APPROX_BF16)
     rc = dmalloc(h, &h->h_bf16, (size_t)max_batch * h->ldh * 2, "bf16 state");
   if (rc) {
@@ -677,11 +679,13 @@ int lstm_approx_run_host(lstm_approx_t* h, const float* x, int T, int B, int K, 
 int lstm_approx_sync(lstm_approx_t* h) {
   if (!h) return LSTM_APPROX_EINVAL;
   DeviceGuard dg(h->device);
+  // the status word rides on the stream into pinned memory: one synchronisation
+  LA_CUDA(h, cudaMemcpyAsync(h->err_host, h->err, sizeof(int), cudaMemcpyDeviceToHost, h->stream), "status read");
   LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
-  int code = 0;
-  LA_CUDA(h, cudaMemcpy(&code, h->err, sizeof(int), cudaMemcpyDeviceToHost), "status read");
+  const int code = *h->err_host;
   if (code != 0) {
-    LA_CUDA(h, cudaMemset(h->err, 0, sizeof(int)), "status clear");
+    LA_CUDA(h, cudaMemsetAsync(h->err, 0, sizeof(int), h->stream), "status clear");
+    LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
     return fail(h, LSTM_APPROX_ETIMEOUT, "a bounded in-kernel wait ran out (code %d); outputs are invalid", code);
   }
   return LSTM_APPROX_OK;
@@ -738,6 +742,7 @@ void lstm_approx_destroy(lstm_approx_t* h) {
   cudaFree(h->seq);
   cudaFree(h->tau);
   cudaFree(h->err);
+  if (h->err_host) cudaFreeHost(h->err_host);
   cudaFree(h->stage);
   cudaFree(h->x_bf16);
   cudaFree(h->seq_bf16);
