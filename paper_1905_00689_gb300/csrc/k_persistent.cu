@@ -56,7 +56,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kTauSlack = 384;          // padding rows of the last CTA and lane reads past gate 3
 constexpr int kMaxGroupsTmem = 2;       // groups of four V_h rows per warp, V_h in tensor memory
 constexpr int kMaxGroupsSmem = 8;       // the same, V_h in shared memory
-constexpr uint32_t kHeaderBytes = 128;  // 5 mbarriers, the TMEM address, the depths k_j
+constexpr uint32_t kHeaderBytes = 192;  // 11 mbarriers, the TMEM address, the depths k_j
 constexpr size_t kMinSmemBytes = 116 * 1024;
 
 struct DevPlan {
@@ -279,9 +279,10 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   constexpr int kMaxGroups = kTmem ? kMaxGroupsTmem : kMaxGroupsSmem;
   constexpr int PIECE = UW < 4 ? UW : 4;  // units per h message
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);          // [0,1] tau, [2,3] h, [4] set-up
-  uint32_t* taddr_s = reinterpret_cast<uint32_t*>(smem_raw + 40);  // TMEM base address
-  int* ck_s = reinterpret_cast<int*>(smem_raw + 48);                // the intermediate depths k_j
+  // mbarriers: [4 hb + g] tau' of gate g for parity hb, [8, 9] h, [10] set-up
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);
+  uint32_t* taddr_s = reinterpret_cast<uint32_t*>(smem_raw + 96);  // TMEM base address
+  int* ck_s = reinterpret_cast<int*>(smem_raw + 112);               // the intermediate depths k_j
   float* sm = reinterpret_cast<float*>(smem_raw + kHeaderBytes);
   const SmemLayout SL = smem_layout(p, a.H, HC, S4);
   float* vh_s = sm + SL.vh;  // V_h rows when they live in shared memory
@@ -296,16 +297,17 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const int H = a.H, K = a.K, J = a.ck.n;
   const int tau_len = 4 * tau_gate_len(p.Kp) + kTauSlack;
   const int h_len = h_buffer_len(p, HC);
-  const uint32_t bytes_tau = p.CS * p.RA * 4u;
+  const uint32_t bytes_tau = p.Kp * 4u;  // one gate's rows (zero rows k >= K included)
   const uint32_t bytes_h = p.CS * p.UBv * 4u;
   const uint64_t limit_ns = static_cast<uint64_t>(a.wait_limit_ns);
   const volatile int* err = a.err;
   const int ngroups = p.RA >> 2;
 
   // ---- set-up: barriers, tensor memory, resident factors, initial state ---
-  const uint32_t bar_setup = smem_u32(&bars[4]);
+  const uint32_t bar_setup = smem_u32(&bars[10]);
   if (tid == 0) {
-    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&bars[i]), kWarps);
+    for (int i = 0; i < 8; ++i) mbar_init(smem_u32(&bars[i]), 4);  // the four warps of the gate
+    for (int i = 8; i < 10; ++i) mbar_init(smem_u32(&bars[i]), kWarps);
     mbar_init(bar_setup, 1);
     if constexpr (!kTmem) {
       int nvalid = 0;  // V_h rows of this CTA that exist (the rest is padding)
@@ -328,11 +330,17 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   tc_fence_after();
   const uint32_t tmem_base = kTmem ? *taddr_s : 0u;
   if (lane == 0) {
-    // first use of each exchange barrier: every warp arrives once, warp 0 with the bytes
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t bytes = (i < 2 ? bytes_tau : bytes_h) + ((i == 0 && a.test_stall) ? 16u : 0u);
-      if (warp == 0) mbar_arrive_expect_tx(smem_u32(&bars[i]), bytes);
-      else mbar_arrive(smem_u32(&bars[i]));
+    // first use of each exchange barrier: every waiting warp arrives once,
+    // the first of them with the bytes (tau': the warps of the gate, warp g
+    // first; h: all warps, warp 0 first)
+    for (int hb = 0; hb < 2; ++hb) {
+      const uint32_t bt = smem_u32(&bars[4 * hb + (warp & 3)]);
+      const uint32_t bytes = bytes_tau + ((hb == 0 && (warp & 3) == 0 && a.test_stall) ? 16u : 0u);
+      if (warp < 4) mbar_arrive_expect_tx(bt, bytes);
+      else mbar_arrive(bt);
+      const uint32_t bh = smem_u32(&bars[8 + hb]);
+      if (warp == 0) mbar_arrive_expect_tx(bh, bytes_h);
+      else mbar_arrive(bh);
     }
   }
   for (int i = tid; i < 2 * tau_len; i += kThreads) tau_s[i] = 0.f;
@@ -517,7 +525,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   // remote addresses of the exchange buffers in CTA (lane mod CS)
   const uint32_t peer = static_cast<uint32_t>(lane) & static_cast<uint32_t>(p.CS - 1);
   const uint32_t bar_tau0 = smem_u32(&bars[0]);
-  const uint32_t bar_h0 = smem_u32(&bars[2]);
+  const uint32_t bar_h0 = smem_u32(&bars[8]);
   const uint32_t r_tau = mapa_shared(smem_u32(tau_s), peer);
   const uint32_t r_bar_tau = mapa_shared(bar_tau0, peer);
   const uint32_t r_h = mapa_shared(smem_u32(h_s), peer);
@@ -530,6 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   cluster_sync_all();  // every CTA's barriers are armed before any st.async
 
   const int t_end = *err == 0 ? a.T : 0;  // nothing to do after a failed set-up
+  bool failed = false;                     // a wait of this unit block ran out
   for (int t = 0; t < t_end; ++t) {
     const int hb = t & 1;
     int fail = 0;  // error code of a wait of this warp that ran out
@@ -583,9 +592,10 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
         const float t1 = __shfl_sync(0xffffffffu, tpr, 4 * q + 1);
         const float t2 = __shfl_sync(0xffffffffu, tpr, 4 * q + 2);
         const float t3 = __shfl_sync(0xffffffffu, tpr, 4 * q + 3);
-        if (lane < p.CS) {
-          const uint32_t off = 4u * (hb * tau_len + tau_pos(rank * p.RA + lr0, p.Kp));
-          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
+        const int gr = rank * p.RA + lr0, gg = gr / p.Kp;  // padding rows past gate 3 are not sent
+        if (lane < p.CS && gg < 4) {
+          const uint32_t off = 4u * (hb * tau_len + tau_pos(gr, p.Kp));
+          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * (4 * hb + gg));
         }
       }
     }
@@ -626,21 +636,24 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
         const float t1 = __shfl_sync(0xffffffffu, tpr, 8 + q);
         const float t2 = __shfl_sync(0xffffffffu, tpr, 16 + q);
         const float t3 = __shfl_sync(0xffffffffu, tpr, 24 + q);
-        if (lane < p.CS) {
-          const uint32_t off = 4u * (hb * tau_len + tau_pos(rank * p.RA + grp * 4, p.Kp));
-          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * hb);
+        const int gr = rank * p.RA + grp * 4, gg = gr / p.Kp;  // padding rows past gate 3 are not sent
+        if (lane < p.CS && gg < 4) {
+          const uint32_t off = 4u * (hb * tau_len + tau_pos(gr, p.Kp));
+          st_async_v4(r_tau + off, t0, t1, t2, t3, r_bar_tau + 8u * (4 * hb + gg));
         }
       }
     }
 
-    // ---- wait for every CTA's tau' ----------------------------------------
+    // ---- wait for this warp's gate of tau' --------------------------------
     if (fail == 0) {
-      const bool ok = mbar_wait_bounded<true>(bar_tau0 + 8u * hb, (t >> 1) & 1, limit_ns, err);
+      // only this warp's gate: the four CTAs that hold its rows
+      const uint32_t bt = bar_tau0 + 8u * (4 * hb + gw);
+      const bool ok = mbar_wait_bounded<true>(bt, (t >> 1) & 1, limit_ns, err);
       if (!__all_sync(0xffffffffu, ok)) {
         fail = kErrWaitTimeoutA;
       } else if (lane == 0) {
-        if (warp == 0) mbar_arrive_expect_tx(bar_tau0 + 8u * hb, bytes_tau);
-        else mbar_arrive(bar_tau0 + 8u * hb);
+        if (warp < 4) mbar_arrive_expect_tx(bt, bytes_tau);
+        else mbar_arrive(bt);
       }
     }
 
@@ -666,7 +679,10 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     if (fail != 0 && lane == 0) atomicCAS(a.err, 0, fail);
     // the four warps of the unit block meet; a wait that ran out in any of
     // them ends the time loop for the whole block here
-    if (block_barrier_or(1 + ub, 128, fail != 0)) break;
+    if (block_barrier_or(1 + ub, 128, fail != 0)) {
+      failed = true;
+      break;
+    }
 
     // ---- cell update (Sec. II) and h_t exchange, in the block's leader ----
     if (leader) {
@@ -721,6 +737,12 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     tmem_dealloc(tmem_base, p.tcols);
   }
   cluster_sync_all();  // no CTA leaves while others may still address its shared memory
+  if (__syncthreads_or(failed)) {
+    // after a wait ran out, copies and stores issued just before the peers
+    // stopped may still be in flight towards this CTA: let them land
+    const uint64_t t0 = global_timer_ns();
+    while (global_timer_ns() - t0 < 50000ull) __nanosleep(1000);
+  }
 }
 
 template <int UW, int KT, int HC>

@@ -74,17 +74,6 @@ __host__ __device__ inline AgLayout ag_layout(const AgPlan& p, int H) {
   return L;
 }
 
-__device__ __forceinline__ void bulk_copy_s2cluster(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
-                                                    uint32_t mb_cluster) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          dst_cluster),
-      "r"(src_cta), "r"(bytes), "r"(mb_cluster)
-      : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async_shared() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 
 // Sum of NV values over the 32 lanes, transposed (high lane bits first):
 // afterwards lane l holds in v[0] the total of value l >> (5 - log2 NV).

@@ -106,6 +106,25 @@ __device__ __forceinline__ void st_async_v4(uint32_t remote_addr, float a, float
       : "memory");
 }
 
+// Bulk copy (TMA engine) of `bytes` from this CTA's shared memory to shared
+// memory of a CTA of the cluster (dst and the mbarrier are cluster addresses
+// of that CTA, from mapa), completing `bytes` on that mbarrier.  Addresses
+// and size are multiples of 16 bytes.
+__device__ __forceinline__ void bulk_copy_s2cluster(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
+                                                    uint32_t mb_cluster) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst_cluster),
+      "r"(src_cta), "r"(bytes), "r"(mb_cluster)
+      : "memory");
+}
+
+// Orders this thread's generic-proxy shared-memory writes before later
+// async-proxy (bulk copy) reads of them.
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Bulk copy (TMA engine, no tensor map) of `bytes` from global to this CTA's
 // shared memory, completing `bytes` on the mbarrier at `mb`.  Addresses and
 // size must be multiples of 16 bytes.
