@@ -148,6 +148,27 @@ __device__ __forceinline__ void lane_partials(const float (&ureg)[UW][KT], const
   }
 }
 
+// The same from the warp's U values already loaded from tensor memory into
+// registers (NP pairs of 16-column loads, value i*KT + s in pre[c/2][16 (c%2) + j]
+// for column 16c + j).
+template <int UW, int KT, int NP>
+__device__ __forceinline__ void lane_partials_pre(const uint32_t (&pre)[2][32], const float* tau_lane,
+                                                  float (&v)[UW]) {
+  constexpr int NV = UW * KT;
+  static_assert(NV <= 32 * NP, "prefetched columns cover the slice");
+  float tv[KT];
+#pragma unroll
+  for (int q = 0; q < KT / 4; ++q) {
+    const float4 f = *reinterpret_cast<const float4*>(tau_lane + 4 * q);
+    tv[4 * q] = f.x; tv[4 * q + 1] = f.y; tv[4 * q + 2] = f.z; tv[4 * q + 3] = f.w;
+  }
+#pragma unroll
+  for (int i = 0; i < UW; ++i) v[i] = 0.f;
+#pragma unroll
+  for (int idx = 0; idx < NV; ++idx)
+    v[idx / KT] = fmaf(__uint_as_float(pre[idx / 32][idx % 32]), tv[idx % KT], v[idx / KT]);
+}
+
 // The same with the warp's slice of U in tensor memory at column u_col:
 // value i*KT + s of the lane (unit i, term s) in column u_col + i*KT + s.
 template <int UW, int KT>
@@ -275,6 +296,11 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   constexpr int HL = 16 * HC;             // h values per lane in a tensor-memory phase A
   constexpr bool kTmem = HC > 0;
   constexpr bool kUTmem = HC == 1;                     // U in tensor memory too
+  // U (one or two column pairs) is loaded from tensor memory before the
+  // tau' wait, so that the load latency hides behind the exchange (holding
+  // V_h's columns across the h wait as well would spill registers)
+  constexpr int kPreNP = (UW * KT + 31) / 32;
+  constexpr bool kPreB = kUTmem && KT >= 4 && (UW * KT == 32 || UW * KT == 64);
   constexpr int UKC = kUTmem ? (UW * KT + 15) / 16 * 16 : 0;  // its columns per warp
   constexpr int kMaxGroups = kTmem ? kMaxGroupsTmem : kMaxGroupsSmem;
   constexpr int PIECE = UW < 4 ? UW : 4;  // units per h message
@@ -644,6 +670,12 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       }
     }
 
+    // U slice of this warp, loaded while tau' is in flight
+    uint32_t upre[2][32];
+    if constexpr (kPreB) {
+      tmem_ld16x2_issue(u_col, u_col + 16, upre[0]);
+      if constexpr (kPreNP == 2) tmem_ld16x2_issue(u_col + 32, u_col + 48, upre[1]);
+    }
     // ---- wait for this warp's gate of tau' --------------------------------
     if (fail == 0) {
       // only this warp's gate: the four CTAs that hold its rows
@@ -657,13 +689,19 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       }
     }
 
+    if constexpr (kPreB) {  // also after a failed wait: no load stays outstanding
+      tmem_wait_ld_tie32(upre[0]);
+      if constexpr (kPreNP == 2) tmem_wait_ld_tie32(upre[1]);
+    }
+
     // ---- phase B: gate sums of this warp's (gate, unit block) -------------
     float* pb = part_s + hb * part_buf;
     if (fail == 0) {
       const float* tau_lane = tau_s + hb * tau_len + gw * tau_gate_len(p.Kp) + k_lane + 4 * (k_lane >> 5);
       float* dst = pb + gw * S4 + ub * UW;
       float v[UW];
-      if constexpr (kUTmem) lane_partials_tmem<UW, KT>(u_col, tau_lane, KT, v);
+      if constexpr (kPreB) lane_partials_pre<UW, KT, kPreNP>(upre, tau_lane, v);
+      else if constexpr (kUTmem) lane_partials_tmem<UW, KT>(u_col, tau_lane, KT, v);
       else lane_partials<UW, KT>(ureg, tau_lane, KT, v);
       butterfly_depths<UW>(v, lane, cap, dst, 4 * S4);
       for (uint32_t m = masked; m != 0u; m &= m - 1u) {  // depths of another form
