@@ -219,7 +219,7 @@ enum lstm_approx_option_key {
   LSTM_APPROX_OPT_WAIT_LIMIT = 3,   /* bounded-wait limit in polls (default 2^26) */
   LSTM_APPROX_OPT_TEST_STALL = 4,   /* 1 = next persistent run waits on a signal
                                        nobody sends (exercises ETIMEOUT) */
-  LSTM_APPROX_OPT_PERSISTENT_VARIANT = 5 /* persistent kernel: 0 = automatic (the
+  LSTM_APPROX_OPT_PERSISTENT_VARIANT = 5, /* persistent kernel: 0 = automatic (the
                                        one-exchange kernel where it fits and
                                        H x terms per CTA <= 16384, else the
                                        per-unit-block one),
@@ -227,6 +227,10 @@ enum lstm_approx_option_key {
                                        exchanges per timestep, any H <= 1024),
                                        2 = one-exchange kernel (H <= 512,
                                        K <= 256, cluster of 4, 8 or 16) */
+  LSTM_APPROX_OPT_XPROJ = 6 /* input projection of the small-batch fp32 path
+                               (T*B <= 32): 0 = automatic (compressed when v
+                               keeps at most 1/8 of the x columns), 1 =
+                               masked-dense rows, 2 = compressed rows */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 

@@ -21,7 +21,7 @@ OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, ESTATE = range(6)
 FP32, BF16 = 0, 1
 Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT = range(5)
 PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
-OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT = range(6)
+OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ = range(7)
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ETIMEOUT: "ETIMEOUT",
                 ESTATE: "ESTATE"}
 

@@ -86,6 +86,7 @@ struct lstm_approx {
 
   // options and counters
   int opt_force_path = 0, opt_cluster = 0, opt_persistent_variant = 0;
+  int opt_xproj = 0;  // 0 automatic, 1 masked-dense, 2 compressed (fp32, T*B <= 32)
   long long opt_wait_limit_us = 2000000;
   int opt_test_stall = 0;
   long long launches = 0;

@@ -180,13 +180,13 @@ void clear_timing(lstm_approx_t* h) {
 // The compressed x projection pays when v keeps at most 1/8 of the x columns
 // (fp32 factors, few columns).
 bool sparse_x_projection(const lstm_approx_t* h, const LayerStore& s, int K, int N) {
-  if (h->dtype != LSTM_APPROX_FP32 || N > 32) return false;
+  if (h->dtype != LSTM_APPROX_FP32 || N > 32 || h->opt_xproj == 1) return false;
   long long kept = 0;
   for (int g = 0; g < 4; ++g) {
     if (s.xoff[g] == nullptr || (int)s.xoff_h[g].size() <= K) return false;
     kept += s.xoff_h[g][K];
   }
-  return kept * 8 <= 4LL * K * s.D;
+  return h->opt_xproj == 2 || kept * 8 <= 4LL * K * s.D;
 }
 
 // The tensor path takes bf16 factors; its intermediate depths must fall on
@@ -783,6 +783,10 @@ int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_TEST_STALL:
       h->opt_test_stall = value != 0;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_XPROJ:
+      if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad projection choice %lld", value);
+      h->opt_xproj = (int)value;
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_PERSISTENT_VARIANT:
       if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad persistent variant %lld", value);

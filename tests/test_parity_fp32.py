@@ -174,3 +174,17 @@ def test_host_buffer_entry_point_matches_device_run(cuda_device):
     assert np.array_equal(out_h.astype(np.float64), got["h"])
     assert np.array_equal(out_c.astype(np.float64), got["c_last"])
     assert np.array_equal(ck_h.astype(np.float64), got["ckpt_h"])
+
+
+@pytest.mark.parametrize("xproj", [1, 2])
+@pytest.mark.parametrize("wl,keep,K,cps", [("c2", 0.25, 256, [16, 64]), ("c1", 0.5, 64, [4, 16]),
+                                           ("f1", 130 / 8320, 16, [5])])
+def test_both_input_projections(cuda_device, xproj, wl, keep, K, cps):
+    """The masked-dense and the compressed projection kernels, each forced, on
+    the batch-1 workloads (the automatic choice runs only one per shape)."""
+    w = WORKLOADS[wl]
+    layers = [list(synthetic_layer(wl, 0, K, keep))]
+    x = workload_inputs(w, T=min(w.T, 6))
+    got, m = run_gpu(layers, x, K, checkpoints=cps, max_rank=K, xproj=xproj)
+    ref = oracle_run(layers, x, K, checkpoints=cps)
+    assert_parity(got, ref, FP32_TOL)
