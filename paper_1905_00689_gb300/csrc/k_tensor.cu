@@ -349,17 +349,35 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
     const uint32_t trow = tmem + ((32u * q) << 16);
     griddep_wait();  // c_t-1 and the outputs are shared with the kernels before this one
+    // c_{t-1} of this thread's unit for its streams, loaded once while the
+    // MMAs run (up to 32 streams; wider tiles load it per chunk below)
+    constexpr bool kCpPre = kHalf <= 32;
+    float cpv[kCpPre ? kHalf : 1];
+    if constexpr (kCpPre) {
+#pragma unroll
+      for (int c = 0; c < kHalf; ++c) {
+        const int n = n0 + cbeg + c;
+        cpv[c] = (unit_ok && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+      }
+    }
     for (int step = 0; step <= J; ++step) {
       const bool final_sums = step == J;
       const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)(step & 1), limit, err);
       tc_fence_after();
       const bool write = ok && *err == 0 && unit_ok;
-      for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 16) {
+      constexpr int kUnroll = kCpPre ? kHalf / 16 : 1;  // registers for cpv, one chunk live otherwise
+#pragma unroll kUnroll
+      for (int ci = 0; ci < kHalf / 16; ++ci) {
+        const int c0 = cbeg + 16 * ci;
         float cp[16];  // c_{t-1}, loaded before any store of this chunk
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
-          const int n = n0 + c0 + c;
-          cp[c] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+          if constexpr (kCpPre) {
+            cp[c] = cpv[16 * ci + c];
+          } else {
+            const int n = n0 + c0 + c;
+            cp[c] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+          }
         }
         float y[4][16];
 #pragma unroll
