@@ -79,6 +79,12 @@ def _config(n_gpus: int) -> dict:
     }
 
 
+def p90(xs) -> float:
+    """90th percentile (nearest rank) of a non-empty sequence."""
+    ys = sorted(xs)
+    return ys[min(len(ys) - 1, max(0, math.ceil(0.9 * len(ys)) - 1))]
+
+
 def _dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -227,6 +233,7 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": _config(1),
         "p50_us_per_timestep": 1e3 * statistics.median(times) / WL.T * 1e3,
+        "p90_us_per_timestep": 1e3 * p90(times) / WL.T * 1e3,
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"{args.steps} full runs of the benchmark workload, fp64 NumPy, one thread"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -324,7 +331,7 @@ def run_ours(args):
         t = timed_loop(max(10, min(args.steps, 50)), lambda K=K: step(K, ()))
         med = statistics.median(t)
         sweep.append({"K": K, "value": T * B / (statistics.mean(t) / 1e3), "unit": UNIT,
-                      "p50_us_per_timestep": 1e3 * med / T,
+                      "p50_us_per_timestep": 1e3 * med / T, "p90_us_per_timestep": 1e3 * p90(t) / T,
                       "effective_factor_gbs": algorithmic_bytes_per_timestep(H, C, nz, K) * T / (med / 1e3) / 1e9})
 
     # ---- large-batch tensor-core path (bf16 factors) -------------------------
@@ -368,7 +375,7 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": _config(ws),
-            "p50_us_per_timestep": 1e3 * p50_ms / T,
+            "p50_us_per_timestep": 1e3 * p50_ms / T, "p90_us_per_timestep": 1e3 * p90(step_ms) / T,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(x_host.nbytes),
                     "d2h_bytes_per_step": int(oh.numel() * 4 + kh.numel() * 4)},
             "roofline": {"kernel": "persistent recurrence kernel", "bound": "hbm", "achieved": achieved,
