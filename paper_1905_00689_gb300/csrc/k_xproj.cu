@@ -5,11 +5,13 @@
 // With T*B this small the product is a skinny matrix times a thin one and
 // the whole packed V_x is read once, so the kernel is about latency: every
 // CTA owns 32 rows and one of S chunks of D (S CTAs of a cluster along D).
-// It stages up to 256 values of D of its 32 rows of V_x and of the x columns
-// in shared memory with 16-byte asynchronous copies spread over all its
-// threads, in two commit groups of 128 values, so that its 8 warps start on
-// the first half while the second is in flight; each lane accumulates a
-// 4-row x NC-column register tile.  The 8 warp partials are summed in shared memory in warp
+// It stages its chunk of D, 128 values of its 32 rows of V_x and of the x
+// columns at a time, with 16-byte asynchronous copies spread over all its
+// threads, through a ring of as many such groups as about 200 KB of shared
+// memory holds (one commit group each): all of them are in flight from the
+// start, the 8 warps consume them in order, and a freed slot is refilled
+// with the next group.  Each lane accumulates a 4-row x NC-column register
+// tile.  The 8 warp partials are summed in shared memory in warp
 // order; each CTA then pushes its chunk sums of the outputs another CTA
 // finishes to that CTA (16-byte st.async completing the owner's mbarrier),
 // and the owner adds the S chunk sums in chunk order, so the result does not
@@ -26,25 +28,35 @@ constexpr int kRows = 32;     // rows per CTA
 constexpr int kCols = 32;     // max columns (T*B)
 constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
-constexpr int kSub = 256;     // values of D staged per round
-constexpr int kHalf = kSub / 2;  // values per staged half (one mbarrier each)
+constexpr int kGrp = 128;     // values of D per staged group (one commit group)
 constexpr int kPadF = 4;      // floats of padding after each staged row
-constexpr int kMaxSplit = 8;  // CTAs per cluster along D
+constexpr int kMaxSplit = 8;  // CTAs per cluster along D (16-CTA clusters start too far apart)
 constexpr int kHdr = 32;      // mbarrier of the incoming chunk sums
+constexpr size_t kRingBudget = 200 * 1024;  // shared memory of the staging ring
 static_assert(kRows * kCols == 4 * kThreads, "each thread pushes one float4 of chunk sums");
 
 template <typename TF>
 constexpr int v_stride() {  // staged V_x row stride in elements (16-byte multiple)
-  return kSub + kPadF * 4 / (int)sizeof(TF);
+  return kGrp + kPadF * 4 / (int)sizeof(TF);
 }
-constexpr int kXStride = kSub + kPadF;
+constexpr int kXStride = kGrp + kPadF;
 
-// header | staged tiles (later the warp partials) | red [32*32] | slot [32*32]
-template <typename TF>
+// one ring slot: 32 rows of V_x and the 4 NC x columns of one group
+template <typename TF, int NC>
+constexpr size_t slot_bytes() {
+  return (size_t)kRows * v_stride<TF>() * sizeof(TF) + (size_t)4 * NC * kXStride * 4;
+}
+template <typename TF, int NC>
+constexpr int ring_slots() {
+  return kRingBudget / slot_bytes<TF, NC>() > 8 ? 8 : (int)(kRingBudget / slot_bytes<TF, NC>());
+}
+
+// header | staging ring (later the warp partials) | red [32*32] | slot [32*32]
+template <typename TF, int NC>
 constexpr size_t smem_bytes() {
-  const size_t tiles = (size_t)kRows * v_stride<TF>() * sizeof(TF) + (size_t)kCols * kXStride * 4;
+  const size_t ring = (size_t)ring_slots<TF, NC>() * slot_bytes<TF, NC>();
   const size_t parts = (size_t)kWarps * kRows * kCols * 4;
-  return kHdr + (tiles > parts ? tiles : parts) + 2 * (size_t)kRows * kCols * 4;
+  return kHdr + (ring > parts ? ring : parts) + 2 * (size_t)kRows * kCols * 4;
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
@@ -56,28 +68,64 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// Issues the 16-byte copies of values [h0, h0 + hl) of the round at d0: the
-// CTA's rows of V_x and the N x columns.
+// Issues the 16-byte copies of values [d0, d0 + len) of the CTA's rows of
+// V_x and of the N x columns into one ring slot, as one commit group.
 template <typename TF>
-__device__ __forceinline__ void stage_half(const TF* A, int lda, int K, int Ks, int row0, int vrows,
-                                           const float* X, int ldxin, int N, int d0, int h0, int hl, TF* vs,
-                                           float* xs, int tid) {
+__device__ __forceinline__ void stage_group(const TF* A, int lda, int K, int Ks, int row0, int vrows,
+                                            const float* X, int ldxin, int N, int d0, int len, TF* vs,
+                                            float* xs, int tid) {
   constexpr int VS = v_stride<TF>();
   constexpr int kPer = 16 / (int)sizeof(TF);  // values per copy
-  const int vq = hl / kPer;
+  const int vq = len / kPer;
   for (int i = tid; i < vrows * vq; i += kThreads) {
     const int rr = i / vq, c = i - rr * vq;
     const int r = row0 + rr;
-    const TF* src = A + (long long)((r / K) * Ks + r % K) * lda + d0 + h0 + c * kPer;
-    cp_async16(smem_u32(vs + rr * VS + h0 + c * kPer), src);
+    const TF* src = A + (long long)((r / K) * Ks + r % K) * lda + d0 + c * kPer;
+    cp_async16(smem_u32(vs + rr * VS + c * kPer), src);
   }
-  const int xq = hl / 4;
+  const int xq = len / 4;
   for (int i = tid; i < N * xq; i += kThreads) {
     const int n = i / xq, c = i - n * xq;
-    cp_async16(smem_u32(xs + n * kXStride + h0 + 4 * c), X + (long long)n * ldxin + d0 + h0 + 4 * c);
+    cp_async16(smem_u32(xs + n * kXStride + 4 * c), X + (long long)n * ldxin + d0 + 4 * c);
   }
   cp_async_commit();
 }
+
+// The same for a full group of kGrp values, from per-thread source pointers
+// computed once per kernel: thread tid copies piece tid % VQ of V_x rows
+// tid / VQ + RP j and of x columns tid / 32 + 8 j.
+template <typename TF>
+struct FullGroupCopies {
+  static constexpr int kPer = 16 / (int)sizeof(TF);  // values per copy
+  static constexpr int VQ = kGrp / kPer;              // copies per row
+  static constexpr int RP = kThreads / VQ;            // rows per pass
+  static constexpr int NP = kRows / RP;               // passes over the 32 rows
+  const TF* v[NP];     // source of this thread's piece of row tid / VQ + RP j at d = 0 (null: no row)
+  const float* x[4];   // source of its piece of x column tid / 32 + 8 j (null: no column)
+  __device__ FullGroupCopies(const TF* A, int lda, int K, int Ks, int row0, int vrows, const float* X, int ldxin,
+                             int N, int tid) {
+#pragma unroll
+    for (int j = 0; j < NP; ++j) {
+      const int rr = tid / VQ + RP * j, r = row0 + rr;
+      v[j] = rr < vrows ? A + (long long)((r / K) * Ks + r % K) * lda + (tid % VQ) * kPer : nullptr;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = tid / 32 + 8 * j;
+      x[j] = n < N ? X + (long long)n * ldxin + 4 * (tid % 32) : nullptr;
+    }
+  }
+  __device__ void issue(int d0, TF* vs, float* xs, int tid) const {
+    constexpr int VS = v_stride<TF>();
+#pragma unroll
+    for (int j = 0; j < NP; ++j)
+      if (v[j] != nullptr) cp_async16(smem_u32(vs + (tid / VQ + RP * j) * VS + (tid % VQ) * kPer), v[j] + d0);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (x[j] != nullptr) cp_async16(smem_u32(xs + (tid / 32 + 8 * j) * kXStride + 4 * (tid % 32)), x[j] + d0);
+    cp_async_commit();
+  }
+};
 
 __device__ __forceinline__ void cluster_arrive_release() {
   asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
@@ -102,10 +150,12 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
                                                          int* err, long long limit_ns) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0]: incoming chunk sums
-  TF* vs = reinterpret_cast<TF*>(smem_raw + kHdr);         // [32][v_stride]
-  float* xs = reinterpret_cast<float*>(smem_raw + kHdr + (size_t)kRows * v_stride<TF>() * sizeof(TF));  // [32][kXStride]
-  float* part = reinterpret_cast<float*>(smem_raw + kHdr);  // [warp][n * 32 + r], after the last round
-  float* red = reinterpret_cast<float*>(smem_raw + smem_bytes<TF>() - 2 * (size_t)kRows * kCols * 4);
+  // ring slot s: V_x rows [32][v_stride] then x columns [4 NC][kXStride]
+  unsigned char* ring = smem_raw + kHdr;
+  constexpr size_t kSlot = slot_bytes<TF, NC>();
+  constexpr int NG = ring_slots<TF, NC>();
+  float* part = reinterpret_cast<float*>(smem_raw + kHdr);  // [warp][n * 32 + r], after the last group
+  float* red = reinterpret_cast<float*>(smem_raw + smem_bytes<TF, NC>() - 2 * (size_t)kRows * kCols * 4);
   float* slot = red + kRows * kCols;  // [S][opc]: chunk c's sums of the outputs this CTA finishes
   constexpr int VS = v_stride<TF>();
 
@@ -138,49 +188,65 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
     for (int j = 0; j < NC; ++j) acc[i][j] = 0.f;
 
   bool ok = true;
-  for (int d0 = c_lo; d0 < c_hi; d0 += kSub) {
-    const int len = min(kSub, c_hi - d0);
-    const int l0 = min(kHalf, len), l1 = len - l0;  // multiples of 8 (D % 8 == 0)
-    stage_half(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, d0, 0, l0, vs, xs, tid);
-    stage_half(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, d0, kHalf, l1, vs, xs, tid);
-    if (d0 == c_lo) {
-      // rows and columns that are never loaded read as zero (filled while
-      // the first copies are in flight; disjoint from what they write)
-      for (int i = tid; i < kRows * VS; i += kThreads)
-        if (i / VS >= vrows) vs[i] = TF(0.f);
-      for (int i = tid; i < 4 * NC * kXStride; i += kThreads)
-        if (i / kXStride >= N) xs[i] = 0.f;
-    }
+  auto slot_v = [&](int sl) { return reinterpret_cast<TF*>(ring + sl * kSlot); };
+  auto slot_x = [&](int sl) {
+    return reinterpret_cast<float*>(ring + sl * kSlot + (size_t)kRows * VS * sizeof(TF));
+  };
+  const int ngrp = (c_hi - c_lo + kGrp - 1) / kGrp;
+  const FullGroupCopies<TF> full(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, tid);
+  auto stage = [&](int gi, int sl) {  // group gi of the chunk into ring slot sl
+    const int d0 = c_lo + gi * kGrp, len = min(kGrp, c_hi - d0);
+    if (len == kGrp) full.issue(d0, slot_v(sl), slot_x(sl), tid);
+    else stage_group(A, lda, K, Ks, rb * kRows, vrows, X, ldxin, N, d0, len, slot_v(sl), slot_x(sl), tid);
+  };
+  // the first NG groups all in flight (an empty commit group past the end
+  // keeps the count of groups behind the one consumed constant)
 #pragma unroll 1
-    for (int hf = 0; hf < 2; ++hf) {
-      const int hl = hf == 0 ? l0 : l1;
-      if (hl == 0) break;
-      if (hf == 0) cp_async_wait<1>();
-      else cp_async_wait<0>();
-      __syncthreads();  // every thread's copies of this half (and the zero fill) are visible
-      // this warp's share of the half, in multiples of 4
-      const int wlen = ((hl + kWarps - 1) / kWarps + 3) & ~3;
-      const int e_lo = hf * kHalf + min(hl, warp * wlen), e_hi = hf * kHalf + min(hl, warp * wlen + wlen);
-      for (int e = e_lo; e < e_hi; e += 4) {
-        float4 va[4], xb[NC];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) va[i] = lds4(vs + (4 * rg + i) * VS + e);
-#pragma unroll
-        for (int j = 0; j < NC; ++j) xb[j] = lds4(xs + (cg * NC + j) * kXStride + e);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-#pragma unroll
-          for (int j = 0; j < NC; ++j) {
-            float s = acc[i][j];
-            s = fmaf(va[i].x, xb[j].x, s);
-            s = fmaf(va[i].y, xb[j].y, s);
-            s = fmaf(va[i].z, xb[j].z, s);
-            s = fmaf(va[i].w, xb[j].w, s);
-            acc[i][j] = s;
-          }
-      }
+  for (int i = 0; i < NG; ++i) {
+    if (i < ngrp) stage(i, i);
+    else cp_async_commit();
+  }
+  // rows and columns that are never loaded read as zero (filled while the
+  // copies are in flight; disjoint from what they write)
+  if (vrows < kRows || N < 4 * NC) {
+    for (int sl = 0; sl < NG && sl < ngrp; ++sl) {
+      TF* vs = slot_v(sl);
+      float* xs = slot_x(sl);
+      for (int i = vrows * VS + tid; i < kRows * VS; i += kThreads) vs[i] = TF(0.f);
+      for (int i = N * kXStride + tid; i < 4 * NC * kXStride; i += kThreads) xs[i] = 0.f;
     }
-    __syncthreads();  // the staged tiles are free for the next round (and the partials)
+  }
+#pragma unroll 1
+  for (int i = 0; i < ngrp; ++i) {
+    const int sl = i % NG, len = min(kGrp, c_hi - (c_lo + i * kGrp));  // a multiple of 8 (D % 8 == 0)
+    cp_async_wait<NG - 1>();  // group i has landed (NG - 1 later groups may still be in flight)
+    __syncthreads();          // every thread's copies of it (and the zero fill) are visible
+    const TF* vs = slot_v(sl);
+    const float* xs = slot_x(sl);
+    // this warp's share of the group, in multiples of 4
+    const int wlen = ((len + kWarps - 1) / kWarps + 3) & ~3;
+    const int e_lo = min(len, warp * wlen), e_hi = min(len, warp * wlen + wlen);
+    for (int e = e_lo; e < e_hi; e += 4) {
+      float4 va[4], xb[NC];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) va[r] = lds4(vs + (4 * rg + r) * VS + e);
+#pragma unroll
+      for (int j = 0; j < NC; ++j) xb[j] = lds4(xs + (cg * NC + j) * kXStride + e);
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int j = 0; j < NC; ++j) {
+          float s = acc[r][j];
+          s = fmaf(va[r].x, xb[j].x, s);
+          s = fmaf(va[r].y, xb[j].y, s);
+          s = fmaf(va[r].z, xb[j].z, s);
+          s = fmaf(va[r].w, xb[j].w, s);
+          acc[r][j] = s;
+        }
+    }
+    __syncthreads();  // the slot is free: refill it with group i + NG
+    if (i + NG < ngrp) stage(i + NG, sl);
+    else cp_async_commit();
   }
 
   // warp partials, then their sum in warp order
@@ -241,7 +307,7 @@ template <typename TF, int NC>
 cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
                       int ldo, int* err, long long limit_ns, cudaStream_t s) {
   auto kern = xproj_kernel<TF, NC>;
-  constexpr size_t smem = smem_bytes<TF>();
+  constexpr size_t smem = smem_bytes<TF, NC>();
   static thread_local bool attr_set = false;
   if (!attr_set) {
     const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
