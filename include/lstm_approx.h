@@ -126,10 +126,11 @@ int lstm_approx_run(lstm_approx_t *h, const float *x, int T, int B, int K, const
 
 /*
  * lstm_approx_run with every tensor a HOST pointer (same shapes and
- * meaning).  Copies the inputs to device staging buffers owned by the
- * handle, runs, copies the outputs back and waits for the stream.  Host
- * buffers in page-locked memory copy fastest.  Returns what
- * lstm_approx_run or lstm_approx_sync would.
+ * meaning).  out_h, ckpt_h and ckpt_c in page-locked, mapped host memory
+ * (cudaHostAlloc / cudaHostRegister, 16-byte aligned) are written in place
+ * by the kernels; every other buffer is copied through device staging
+ * buffers owned by the handle.  Waits for the stream before it
+ * returns.  Returns what lstm_approx_run or lstm_approx_sync would.
  */
 int lstm_approx_run_host(lstm_approx_t *h, const float *x, int T, int B, int K, const float *h0,
                          const float *c0, float *out_h, float *out_c, const int *checkpoints, int J,

@@ -640,6 +640,20 @@ int lstm_approx_run(lstm_approx_t* h, const float* x, int T, int B, int K, const
   return run_device(h, x, T, B, K, h0, c0, out_h, out_c, ck, ckpt_h, ckpt_c);
 }
 
+// Device address of a page-locked, mapped host buffer that the kernels may
+// write in place (16-byte aligned), else null: pageable memory goes through
+// the staging copies.
+static float* mapped_view(const float* p) {
+  if (p == nullptr || (reinterpret_cast<uintptr_t>(p) & 15u) != 0) return nullptr;
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();  // an unknown pointer: clear the (non-sticky) error
+    return nullptr;
+  }
+  if (at.type != cudaMemoryTypeHost || at.devicePointer == nullptr) return nullptr;
+  return static_cast<float*>(at.devicePointer);
+}
+
 int lstm_approx_run_host(lstm_approx_t* h, const float* x, int T, int B, int K, const float* h0, const float* c0,
                          float* out_h, float* out_c, const int* checkpoints, int J, float* ckpt_h, float* ckpt_c) {
   if (!h) return LSTM_APPROX_EINVAL;
@@ -661,17 +675,40 @@ int lstm_approx_run_host(lstm_approx_t* h, const float* x, int T, int B, int K, 
     h->stage_bytes = total;
   }
   float* st = reinterpret_cast<float*>(h->stage);
-  LA_CUDA(h, cudaMemcpyAsync(st + off_x, x, nx * 4, cudaMemcpyHostToDevice, h->stream), "input copy");
-  if (h0) LA_CUDA(h, cudaMemcpyAsync(st + off_h0, h0, ns * 4, cudaMemcpyHostToDevice, h->stream), "h0 copy");
-  if (c0) LA_CUDA(h, cudaMemcpyAsync(st + off_c0, c0, ns * 4, cudaMemcpyHostToDevice, h->stream), "c0 copy");
-  rc = run_device(h, st + off_x, T, B, K, h0 ? st + off_h0 : nullptr, c0 ? st + off_c0 : nullptr, st + off_oh,
-                  out_c ? st + off_oc : nullptr, ck, ckpt_h ? st + off_kh : nullptr, ckpt_c ? st + off_kc : nullptr);
+  // page-locked out_h and checkpoint buffers are written in place by the
+  // kernels over the host link (the stores are posted; 3% off a batch-1
+  // call).  The inputs are staged: a kernel reading x from host memory waits
+  // on the link, which costs more than one copy.  The states, which the run
+  // copies between device buffers, are staged too.
+  const float* dx = nullptr;
+  const float* dh0 = nullptr;
+  const float* dc0 = nullptr;
+  float* doh = mapped_view(out_h);
+  float* doc = nullptr;
+  float* dkh = nk ? mapped_view(ckpt_h) : nullptr;
+  float* dkc = nk ? mapped_view(ckpt_c) : nullptr;
+  if (!dx) {
+    LA_CUDA(h, cudaMemcpyAsync(st + off_x, x, nx * 4, cudaMemcpyHostToDevice, h->stream), "input copy");
+    dx = st + off_x;
+  }
+  if (h0 && !dh0) {
+    LA_CUDA(h, cudaMemcpyAsync(st + off_h0, h0, ns * 4, cudaMemcpyHostToDevice, h->stream), "h0 copy");
+    dh0 = st + off_h0;
+  }
+  if (c0 && !dc0) {
+    LA_CUDA(h, cudaMemcpyAsync(st + off_c0, c0, ns * 4, cudaMemcpyHostToDevice, h->stream), "c0 copy");
+    dc0 = st + off_c0;
+  }
+  rc = run_device(h, dx, T, B, K, dh0, dc0, doh ? doh : st + off_oh, out_c ? (doc ? doc : st + off_oc) : nullptr, ck,
+                  (ckpt_h && nk) ? (dkh ? dkh : st + off_kh) : nullptr,
+                  (ckpt_c && nk) ? (dkc ? dkc : st + off_kc) : nullptr);
   if (rc) return rc;
-  LA_CUDA(h, cudaMemcpyAsync(out_h, st + off_oh, no * 4, cudaMemcpyDeviceToHost, h->stream), "output copy");
-  if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, st + off_oc, ns * 4, cudaMemcpyDeviceToHost, h->stream), "c copy");
-  if (ckpt_h && nk)
+  if (!doh) LA_CUDA(h, cudaMemcpyAsync(out_h, st + off_oh, no * 4, cudaMemcpyDeviceToHost, h->stream), "output copy");
+  if (out_c && !doc)
+    LA_CUDA(h, cudaMemcpyAsync(out_c, st + off_oc, ns * 4, cudaMemcpyDeviceToHost, h->stream), "c copy");
+  if (ckpt_h && nk && !dkh)
     LA_CUDA(h, cudaMemcpyAsync(ckpt_h, st + off_kh, nk * 4, cudaMemcpyDeviceToHost, h->stream), "ckpt copy");
-  if (ckpt_c && nk)
+  if (ckpt_c && nk && !dkc)
     LA_CUDA(h, cudaMemcpyAsync(ckpt_c, st + off_kc, nk * 4, cudaMemcpyDeviceToHost, h->stream), "ckpt copy");
   return lstm_approx_sync(h);
 }

@@ -188,3 +188,36 @@ def test_both_input_projections(cuda_device, xproj, wl, keep, K, cps):
     got, m = run_gpu(layers, x, K, checkpoints=cps, max_rank=K, xproj=xproj)
     ref = oracle_run(layers, x, K, checkpoints=cps)
     assert_parity(got, ref, FP32_TOL)
+
+
+@pytest.mark.parametrize("pinned", [False, True])
+def test_host_entry_pinned_and_pageable_buffers(cuda_device, pinned):
+    """lstm_approx_run_host writes out_h and the checkpoints in place when
+    they are page-locked, and stages them otherwise: both give the device
+    run's outputs bit for bit (with initial states and the final c, which
+    are always staged)."""
+    import torch
+    w = WORKLOADS["c2"]
+    layers = [list(synthetic_layer("c2", 0, 64, 0.25))]
+    x = workload_inputs(w, T=7).astype(np.float32)
+    rng = np.random.default_rng(5)
+    h0 = (0.3 * rng.standard_normal((1, 1, w.H))).astype(np.float32)
+    c0 = (0.3 * rng.standard_normal((1, 1, w.H))).astype(np.float32)
+    got, m = run_gpu(layers, x, 64, h0=h0, c0=c0, checkpoints=[16, 40])
+
+    def buf(shape, src=None):
+        t = torch.zeros(shape, dtype=torch.float32)
+        if pinned:
+            t = t.pin_memory()
+        if src is not None:
+            t.copy_(torch.from_numpy(src))
+        return t
+    xt, oh, oc = buf(x.shape, x), buf((7, 1, w.H)), buf((1, 1, w.H))
+    kh, kc = buf((2, 7, 1, w.H)), buf((2, 7, 1, w.H))
+    assert xt.is_pinned() == pinned
+    m.run_host(xt.numpy(), 64, oh.numpy(), h0=buf(h0.shape, h0).numpy(), c0=buf(c0.shape, c0).numpy(),
+               out_c=oc.numpy(), checkpoints=[16, 40], ckpt_h=kh.numpy(), ckpt_c=kc.numpy())
+    assert np.array_equal(oh.numpy().astype(np.float64), got["h"])
+    assert np.array_equal(oc.numpy().astype(np.float64), got["c_last"])
+    assert np.array_equal(kh.numpy().astype(np.float64), got["ckpt_h"])
+    assert np.array_equal(kc.numpy().astype(np.float64), got["ckpt_c"])
