@@ -339,7 +339,9 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     if (path == 0) {
       path = LSTM_APPROX_PATH_SIMT;
       if (tensor_ok) path = LSTM_APPROX_PATH_TENSOR;
-      else if (!bf16 && B <= 8 &&
+      // fp32 factors: a persistent launch whenever a plan fits, at any batch
+      // (one cluster per stream; clusters beyond one wave run in the next)
+      else if (!bf16 &&
                choose_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, h->opt_persistent_variant, &plan, &why))
         path = LSTM_APPROX_PATH_PERSISTENT;
     } else if (path == LSTM_APPROX_PATH_PERSISTENT) {

@@ -101,3 +101,15 @@ def test_one_exchange_rejects_what_it_cannot_hold(cuda_device):
     got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT)
     assert m.query(Q_PERSISTENT_VARIANT) == 1
     assert_parity(got, oracle_run(layers, x, K), FP32_TOL)
+
+
+@pytest.mark.parametrize("D,H,T,B,K", [(64, 64, 4, 16, 64), (96, 512, 3, 12, 64), (40, 128, 2, 40, 16)])
+def test_many_streams_take_the_persistent_path(cuda_device, D, H, T, B, K):
+    """fp32 runs with more streams than one wave of clusters holds still take
+    a persistent kernel (the later clusters run in the next wave)."""
+    gates = [draw_factor_set(H, D + H, K, (D + H) // 3, 60 + D + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 7 + B)
+    got, m = run_gpu([gates], x, K, checkpoints=[8])
+    assert m.query(Q_LAST_PATH) == PATH_PERSISTENT
+    ref = oracle_run([gates], x, K, checkpoints=[8])
+    assert_parity(got, ref, FP32_TOL)
