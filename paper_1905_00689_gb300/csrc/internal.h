@@ -107,10 +107,11 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
                              int N, int Kdim, float* out, int ldo, int mode, const float* sigma,
                              const float* P, int ldp, cudaStream_t s);
 
-// Same product for few columns (N = T*B <= 32): clusters split the D axis,
-// rows are staged by bulk copies and reduced through distributed shared
-// memory (deterministic).  Needs D % 8 == 0 and 16-byte aligned rows; a
-// staged load that does not complete within limit_ns sets *err.
+// Same product for few columns (N = T*B <= 256, in chunks of 32): clusters
+// split the D axis, rows are staged by asynchronous copies and the chunk
+// sums pushed to their owner CTA (deterministic).  Needs D % 8 == 0 and
+// 16-byte aligned rows; a push that does not arrive within limit_ns sets
+// *err.
 bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16);
 
 // Compressed x part of the pruned v (fp32 factors): per gate, the kept x

@@ -1,4 +1,5 @@
-// Hoisted input projection for few columns (T*B <= 32): P[n][(g,k)] =
+// Hoisted input projection for few columns (T*B <= 256, 32 columns per
+// launch chunk along grid z): P[n][(g,k)] =
 // prune(v_{g,k})[0:D]^T x_n for every timestep and stream at once (the x
 // columns of x~ = [x_t; h_{t-1}], Sec. III, split off Eq. 1's dot products).
 //
@@ -162,6 +163,10 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rg = lane >> 2, cg = lane & 3;
   const int rb = blockIdx.x;
+  // column chunk blockIdx.z of 32 (launches with more than 32 columns)
+  X += (long long)blockIdx.z * kCols * ldxin;
+  out += (long long)blockIdx.z * kCols * ldo;
+  N = min(kCols, N - (int)blockIdx.z * kCols);
   const uint32_t q = S > 1 ? cluster_ctarank() : 0u;  // chunk of D
   const int nrows = 4 * K;
   const int vrows = min(kRows, nrows - rb * kRows);
@@ -315,11 +320,12 @@ cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int l
     attr_set = true;
   }
   const int row_tiles = (4 * K + kRows - 1) / kRows;
+  const int col_chunks = (N + kCols - 1) / kCols;
   int S = 1;  // chunks of D: about one CTA per SM in total, at least 128 values of D each
-  while (S < kMaxSplit && row_tiles * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
+  while (S < kMaxSplit && row_tiles * col_chunks * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
   const int dchunk = (((D + S - 1) / S) + 7) & ~7;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(row_tiles, S, 1);
+  cfg.gridDim = dim3(row_tiles, S, col_chunks);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
@@ -336,7 +342,7 @@ cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int l
 template <typename TF>
 cudaError_t launch_typed(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
                          int ldo, int* err, long long limit_ns, cudaStream_t s) {
-  switch ((N + 3) / 4) {  // columns per lane
+  switch ((min(N, kCols) + 3) / 4) {  // columns per lane (more than 32: chunks of 32)
     case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
     case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
     case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
@@ -422,7 +428,9 @@ cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const floa
 bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16) {
   // bulk copies need 16-byte aligned rows and lengths
   const int a_align = a_bf16 ? 8 : 4;
-  return N >= 1 && N <= kCols && D % 8 == 0 && lda % a_align == 0 && ldxin % 4 == 0;
+  // up to 8 chunks of 32 columns: beyond that every chunk re-reading the
+  // CTA's rows costs more than a tiled GEMM
+  return N >= 1 && N <= 8 * kCols && D % 8 == 0 && lda % a_align == 0 && ldxin % 4 == 0;
 }
 
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
