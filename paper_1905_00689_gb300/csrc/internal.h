@@ -82,6 +82,8 @@ struct lstm_approx {
 
   // staging for lstm_approx_run_host
   size_t stage_bytes = 0;
+  float* gpart = nullptr;     // raw gate sums of a term-split gate GEMM (tensor path), grown on demand
+  size_t gpart_bytes = 0;
   char* stage = nullptr;
 
   // options and counters
@@ -255,9 +257,20 @@ struct TcGatesArgs {
   long long ck_stride;
   int* err;
   long long limit_ns;
+  // split over the term axis (ks > 1, grid z = ks): CTA z accumulates the
+  // 64-term chunks [z nkb_per, (z+1) nkb_per) and writes its raw gate sums,
+  // element (slot, g, n, unit) at ((slot*4 + g)*B + n)*H + unit of `part`:
+  // slot z for its whole range, slot ks + j at an intermediate depth k_j that
+  // ends inside it.  launch_tc_gates then runs the sum over the splits and
+  // the cell update of Sec. II in a second kernel.
+  int ks, nkb_per;
+  float* part;
 };
 // `nt` (32, 64 or 128) must match the box rows of Tau's map.
 cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s);
+// Term-axis splits for a gate GEMM of `tiles` CTAs over nkb 64-term chunks
+// (1: no split); *nkb_per receives the chunks per split.
+int tc_gates_splits(int tiles, int nkb, int* nkb_per);
 
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s);
 cudaError_t launch_tc_init_state(const float* h0, const float* c0, int B, int H, __nv_bfloat16* h_bf16, int ldh,

@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // ---------------------------------------------------------------------------
 // four gate sums for 128 units x NT streams, cell update in the epilogue
 // ---------------------------------------------------------------------------
-template <int NT, int S>
+template <int NT, int S, bool SPLIT>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_gates_kernel(const __grid_constant__ CUtensorMap tmu, const __grid_constant__ CUtensorMap tmt, TcGatesArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -239,8 +239,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int j0 = blockIdx.x * kTileM;
   const int n0 = blockIdx.y * NT;
-  const int nkb = a.nkb;
+  // this CTA's 64-term chunks [kb0, kb1) (all of them without a split), and
+  // the intermediate depths that end inside them, [jj_lo, jj_hi)
+  constexpr bool split = SPLIT;
+  const int kb0 = split ? (int)blockIdx.z * a.nkb_per : 0;
+  const int kb1 = split ? min(a.nkb, kb0 + a.nkb_per) : a.nkb;
+  const int nkb = kb1 - kb0;
   const int J = a.ck.n;
+  int jj_lo = 0, jj_hi = J;
+  if constexpr (SPLIT) {
+    jj_hi = 0;
+    for (int j = 0; j < J; ++j) {
+      jj_lo += a.ck.k[j] <= kb0 * kTileK ? 1 : 0;
+      jj_hi += a.ck.k[j] <= kb1 * kTileK ? 1 : 0;
+    }
+  }
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
 
@@ -275,11 +288,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int npre = nst < S ? nst : S;
     for (int i = 0; i < npre; ++i) {
       mbar_arrive_expect_tx(bar0 + 8u * i, kABytes + kBBytes);
-      tma_load_2d(sA + i * kABytes, &tmu, bar0 + 8u * i, (i >> 2) * kTileK, (i & 3) * a.H + j0);
+      tma_load_2d(sA + i * kABytes, &tmu, bar0 + 8u * i, (kb0 + (i >> 2)) * kTileK, (i & 3) * a.H + j0);
     }
     griddep_wait();
     for (int i = 0; i < nst; ++i) {
-      const int s = i % S, kb = i >> 2, g = i & 3;
+      const int s = i % S, kb = kb0 + (i >> 2), g = i & 3;
       if (i >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((i / S) - 1) & 1, limit, err))) break;
       if (i >= npre) {
         mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
@@ -296,8 +309,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, NT);
     bool ok = true;
-    int jj = 0;
-    for (int kb = 0; kb < nkb && ok; ++kb) {
+    int jj = jj_lo;
+    for (int kl = 0; kl < nkb && ok; ++kl) {
+      const int kb = kb0 + kl;
       uint64_t da[4], db[4];
       // 16-term slices of this chunk, cut where an intermediate depth ends;
       // each gate's stage is used as soon as it lands and freed as soon as
@@ -305,10 +319,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       int kk0 = 0;
       while (kk0 < 4 && ok) {
         int kk1 = 4;
-        const bool cut_here = jj < J && a.ck.k[jj] <= (kb + 1) * kTileK;
+        const bool cut_here = jj < jj_hi && a.ck.k[jj] <= (kb + 1) * kTileK;
         if (cut_here) kk1 = (a.ck.k[jj] - kb * kTileK) / 16;
         for (int g = 0; g < 4 && ok; ++g) {
-          const int i = 4 * kb + g, s = i % S;
+          const int i = 4 * kl + g, s = i % S;
           if (kk0 == 0) {
             if (!(ok = wait_cta(bar0 + 8u * s, (i / S) & 1, limit, err))) break;
             tc_fence_after();
@@ -316,12 +330,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             db[g] = umma_desc_sw128(sB + s * kBBytes);
           }
           for (int kk = kk0; kk < kk1; ++kk)
-            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, db[g] + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, db[g] + 2ull * kk, idesc, (kl | kk) != 0 ? 1u : 0u);
           if (kk1 == 4) umma_commit(bar0 + 8u * (S + s));  // frees this gate's stage
         }
         if (ok && cut_here) {  // partial sums up to depth k_jj are complete: hand them to the epilogue
           umma_commit(ckpt_bar);
-          ok = wait_cta(ckpt_done, jj & 1, limit, err);
+          ok = wait_cta(ckpt_done, (jj - jj_lo) & 1, limit, err);
           tc_fence_after();
           ++jj;
         }
@@ -329,9 +343,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
-    while (jj < J) {  // release epilogue warps still waiting for a depth (abort only)
+    while (jj < jj_hi) {  // release epilogue warps still waiting for a depth (abort only)
       umma_commit(ckpt_bar);
-      wait_cta(ckpt_done, jj & 1, limit, err);
+      wait_cta(ckpt_done, (jj - jj_lo) & 1, limit, err);
       ++jj;
     }
     umma_commit(accum_bar);
@@ -357,14 +371,39 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
       for (int c = 0; c < kHalf; ++c) {
         const int n = n0 + cbeg + c;
-        cpv[c] = (unit_ok && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+        cpv[c] = (!split && unit_ok && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
       }
     }
-    for (int step = 0; step <= J; ++step) {
-      const bool final_sums = step == J;
-      const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)(step & 1), limit, err);
+    for (int step = jj_lo; step <= jj_hi; ++step) {
+      const bool final_sums = step == jj_hi;
+      const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)((step - jj_lo) & 1),
+                               limit, err);
       tc_fence_after();
       const bool write = ok && *err == 0 && unit_ok;
+      if constexpr (SPLIT) {
+        // raw gate sums of this CTA's terms: slot z for its whole range, slot
+        // ks + step at a depth that ends inside it
+        const long long slot = final_sums ? (long long)blockIdx.z : (long long)(a.ks + step);
+        for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 16) {
+          float y[4][16];
+#pragma unroll
+          for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
+          tmem_wait_ld();
+          if (!write) continue;
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const int n = n0 + c0 + c;
+            if (n >= a.B) break;
+#pragma unroll
+            for (int g = 0; g < 4; ++g) a.part[((slot * 4 + g) * a.B + n) * a.H + j] = y[g][c];
+          }
+        }
+        if (!final_sums) {
+          tc_fence_before();
+          mbar_arrive(ckpt_done);
+        }
+        continue;
+      }
       constexpr int kUnroll = kCpPre ? kHalf / 16 : 1;  // registers for cpv, one chunk live otherwise
 #pragma unroll kUnroll
       for (int ci = 0; ci < kHalf / 16; ++ci) {
@@ -392,7 +431,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           float hh, cc;
           lstm_cell_hw(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
           if (!final_sums) {
-            const long long o = (long long)step * a.ck_stride + sj;
+            const long long o = (long long)step * a.ck_stride + sj;  // (no split: jj_lo = 0)
             if (a.ckpt_h) a.ckpt_h[o] = hh;
             if (a.ckpt_c) a.ckpt_c[o] = cc;
           } else {
@@ -416,6 +455,54 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kCols);
   }
+}
+
+// After a term-axis split of the gate GEMM: one thread per (stream n, unit
+// j) adds the splits' raw gate sums in split order and runs the cell update
+// of Sec. II, at full depth and at each intermediate depth k_j (the splits
+// before the one k_j ends in, then that split's sums up to k_j).
+__global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
+  griddep_launch_dependents();  // the next step's tau' kernel may start its set-up
+  const long long total = (long long)a.B * a.H;
+  const long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  griddep_wait();  // the partial sums of the gate GEMM before this kernel
+  if (i >= total || *reinterpret_cast<volatile int*>(a.err) != 0) return;
+  const int n = (int)(i / a.H), j = (int)(i - (long long)n * a.H);
+  const long long gs = (long long)a.B * a.H;  // gate stride within a slot
+  const float* part = a.part + (long long)n * a.H + j;
+  float bias[4];
+#pragma unroll
+  for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
+  const float cp = a.c_state[i];
+  for (int jj = 0; jj < a.ck.n; ++jj) {
+    const int sj = ((a.ck.k[jj] + kTileK - 1) / kTileK - 1) / a.nkb_per;  // split the depth ends in
+    float y[4];
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      float v = 0.f;
+      for (int z = 0; z < sj; ++z) v += part[(z * 4 + g) * gs];
+      y[g] = v + part[((a.ks + jj) * 4 + g) * gs] + bias[g];
+    }
+    float hh, cc;
+    lstm_cell_hw(y[0], y[1], y[2], y[3], cp, hh, cc);
+    const long long o = (long long)jj * a.ck_stride + i;
+    if (a.ckpt_h) a.ckpt_h[o] = hh;
+    if (a.ckpt_c) a.ckpt_c[o] = cc;
+  }
+  float y[4];
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    float v = 0.f;
+    for (int z = 0; z < a.ks; ++z) v += part[(z * 4 + g) * gs];
+    y[g] = v + bias[g];
+  }
+  float hh, cc;
+  lstm_cell_hw(y[0], y[1], y[2], y[3], cp, hh, cc);
+  a.c_state[i] = cc;
+  if (a.out_h) a.out_h[i] = hh;
+  const __nv_bfloat16 hb = __float2bfloat16_rn(hh);
+  a.h_bf16[(long long)n * a.ldh + j] = hb;
+  if (a.seq_bf16) a.seq_bf16[(long long)n * a.ldh + j] = hb;
 }
 
 // x (fp32 [N][D]) -> bf16 [N][ld] with zero columns D..ld-1: one thread per
@@ -484,10 +571,10 @@ EncodeTiled encoder() {
 // the one before it in the stream finishes, and waits on it (griddep_wait)
 // only where it reads that kernel's results or writes what it reads.
 template <typename Kern, typename... Args>
-cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args... args) {
+cudaError_t launch_pdl_block(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(kTcThreads);
+  cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -496,6 +583,10 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args..
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+template <typename Kern, typename... Args>
+cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args... args) {
+  return launch_pdl_block(kern, grid, dim3(kTcThreads), smem, s, args...);
 }
 
 template <int BN, int S>
@@ -522,9 +613,9 @@ cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, 
                     a);
 }
 
-template <int NT, int S>
+template <int NT, int S, bool SPLIT>
 cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, cudaStream_t s) {
-  auto kern = tc_gates_kernel<NT, S>;
+  auto kern = tc_gates_kernel<NT, S, SPLIT>;
   static thread_local bool attr = false;
   const size_t smem = gates_smem<NT, S>();
   if (!attr) {
@@ -532,9 +623,12 @@ cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& 
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  return launch_pdl(kern, dim3((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT), smem, s,
-                    *reinterpret_cast<const CUtensorMap*>(U.bytes), *reinterpret_cast<const CUtensorMap*>(Tau.bytes),
-                    a);
+  const cudaError_t e =
+      launch_pdl(kern, dim3((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT, a.ks > 1 ? a.ks : 1), smem, s,
+                 *reinterpret_cast<const CUtensorMap*>(U.bytes), *reinterpret_cast<const CUtensorMap*>(Tau.bytes), a);
+  if (e != cudaSuccess || a.ks <= 1) return e;
+  const long long total = (long long)a.B * a.H;
+  return launch_pdl_block(tc_gates_reduce_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, s, a);
 }
 
 }  // namespace
@@ -562,6 +656,19 @@ int tc_rows_tile_n(int n_cols, int row_tiles) {
     if ((long long)row_tiles * ((n_cols + bn - 1) / bn) <= 148) return bn;
   return 256;
 }
+int tc_gates_splits(int tiles, int nkb, int* nkb_per) {
+  // about one wave: as many splits as the GPU holds grids of `tiles` CTAs
+  int ks = 148 / (tiles > 0 ? tiles : 1);
+  if (ks > 8) ks = 8;
+  if (ks > nkb) ks = nkb;
+  if (ks < 2) {
+    *nkb_per = nkb;
+    return 1;
+  }
+  *nkb_per = (nkb + ks - 1) / ks;
+  return (nkb + *nkb_per - 1) / *nkb_per;  // no empty split
+}
+
 int tc_gates_tile_n(int H, int B) {
   const int unit_tiles = (H + kTileM - 1) / kTileM;
   for (int nt : {32, 64, 128})
@@ -579,9 +686,9 @@ cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a,
 
 cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s) {
   switch (nt) {
-    case 128: return launch_gates_t<128, 6>(U, Tau, a, s);
-    case 64: return launch_gates_t<64, 8>(U, Tau, a, s);
-    default: return launch_gates_t<32, 8>(U, Tau, a, s);
+    case 128: return a.ks > 1 ? launch_gates_t<128, 6, true>(U, Tau, a, s) : launch_gates_t<128, 6, false>(U, Tau, a, s);
+    case 64: return a.ks > 1 ? launch_gates_t<64, 8, true>(U, Tau, a, s) : launch_gates_t<64, 8, false>(U, Tau, a, s);
+    default: return a.ks > 1 ? launch_gates_t<32, 8, true>(U, Tau, a, s) : launch_gates_t<32, 8, false>(U, Tau, a, s);
   }
 }
 

@@ -263,6 +263,22 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   h->launches += 1;
   const int bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
   const int nt = tc_gates_tile_n(H, B);
+  // small grids (few streams) split the gate GEMM's terms over more CTAs
+  int nkb_per = 0;
+  const int gate_tiles = ((H + 127) / 128) * ((B + nt - 1) / nt);
+  const int ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &nkb_per);
+  if (ks > 1) {
+    const size_t need = (size_t)(ks + ck.n) * 4 * B * H * sizeof(float);
+    if (need > h->gpart_bytes) {
+      LA_CUDA(h, cudaStreamSynchronize(h->stream), "synchronising before growing the split buffer");
+      dfree(h, h->gpart, h->gpart_bytes);
+      h->gpart = nullptr;
+      h->gpart_bytes = 0;
+      rc = dmalloc(h, reinterpret_cast<void**>(&h->gpart), need, "split gate sums");
+      if (rc) return rc;
+      h->gpart_bytes = need;
+    }
+  }
   TcMap mh, mt;
   if (!tc_make_map(&mh, hb, H, B, (uint64_t)h->ldh * 2, bnh) ||
       !tc_make_map(&mt, tau, ldp, B, (uint64_t)ldp * 2, nt))
@@ -301,8 +317,11 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ga.ck_stride = (long long)T * B * H;
     ga.err = h->err;
     ga.limit_ns = limit_ns;
+    ga.ks = ks;
+    ga.nkb_per = nkb_per;
+    ga.part = h->gpart;
     LA_CUDA(h, launch_tc_gates(s.map_u, mt, ga, nt, h->stream), "gate GEMM launch");
-    h->launches += 2;
+    h->launches += ks > 1 ? 3 : 2;
   }
   if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, cs, (size_t)B * H * sizeof(float), cudaMemcpyDeviceToDevice, h->stream),
                      "c copy");
@@ -783,6 +802,7 @@ void lstm_approx_destroy(lstm_approx_t* h) {
   cudaFree(h->err);
   if (h->err_host) cudaFreeHost(h->err_host);
   cudaFree(h->stage);
+  cudaFree(h->gpart);
   cudaFree(h->x_bf16);
   cudaFree(h->seq_bf16);
   cudaFree(h->h_bf16);
