@@ -117,8 +117,10 @@ int lstm_approx_set_factors(lstm_approx_t *h, int layer, int gate, int K, int nz
  * Errors: EINVAL, ESTATE (a gate's factors missing or shallower than K),
  * ENOMEM (growing the T-dependent scratch), ECUDA (launch failure).
  * Kernel-side failures (a bounded wait that ran out) are reported by the
- * next lstm_approx_sync().  The first run at a new largest T*B may allocate
- * scratch (synchronising the stream).
+ * next lstm_approx_sync().  The first run at a new largest T*B (and, on
+ * the bf16 tensor-core path with few streams, at a new largest B * H with
+ * intermediate depths) may allocate scratch, synchronising the stream;
+ * lstm_approx_run_static never allocates.
  */
 int lstm_approx_run(lstm_approx_t *h, const float *x, int T, int B, int K, const float *h0,
                     const float *c0, float *out_h, float *out_c, const int *checkpoints, int J,
