@@ -113,7 +113,8 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
 // split the D axis, rows are staged by asynchronous copies and the chunk
 // sums pushed to their owner CTA (deterministic).  Needs D % 8 == 0 and
 // 16-byte aligned rows; a push that does not arrive within limit_ns sets
-// *err.
+// *err.  max_split caps the CTAs per cluster along D (1: one CTA per row
+// tile and column chunk).
 bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16);
 
 // Compressed x part of the pruned v (fp32 factors): per gate, the kept x
@@ -127,7 +128,8 @@ struct SparseXRows {
 cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const float* X, int ldxin, int N, float* out,
                                 int ldo, cudaStream_t s);
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
-                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s);
+                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s,
+                                 int max_split);
 
 // One timestep of the refinement sums over u (a3), the intermediate outputs
 // (a6) and the cell update (a4) for B streams.

@@ -310,7 +310,7 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
 
 template <typename TF, int NC>
 cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
-                      int ldo, int* err, long long limit_ns, cudaStream_t s) {
+                      int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split) {
   auto kern = xproj_kernel<TF, NC>;
   constexpr size_t smem = smem_bytes<TF, NC>();
   static thread_local bool attr_set = false;
@@ -321,8 +321,10 @@ cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int l
   }
   const int row_tiles = (4 * K + kRows - 1) / kRows;
   const int col_chunks = (N + kCols - 1) / kCols;
-  int S = 1;  // chunks of D: about one CTA per SM in total, at least 128 values of D each
-  while (S < kMaxSplit && row_tiles * col_chunks * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
+  // chunks of D: about one CTA per SM in total, at least 128 values of D
+  // each, and at most max_split (the caller's choice: see run_device)
+  int S = 1;
+  while (S < kMaxSplit && S < max_split && row_tiles * col_chunks * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
   const int dchunk = (((D + S - 1) / S) + 7) & ~7;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(row_tiles, S, col_chunks);
@@ -341,16 +343,16 @@ cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int l
 
 template <typename TF>
 cudaError_t launch_typed(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
-                         int ldo, int* err, long long limit_ns, cudaStream_t s) {
+                         int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split) {
   switch ((min(N, kCols) + 3) / 4) {  // columns per lane (more than 32: chunks of 32)
-    case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 4: return launch_nc<TF, 4>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 5: return launch_nc<TF, 5>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 6: return launch_nc<TF, 6>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 7: return launch_nc<TF, 7>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
-    case 8: return launch_nc<TF, 8>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+    case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 4: return launch_nc<TF, 4>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 5: return launch_nc<TF, 5>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 6: return launch_nc<TF, 6>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 7: return launch_nc<TF, 7>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 8: return launch_nc<TF, 8>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -434,11 +436,12 @@ bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16) {
 }
 
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
-                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s) {
+                                 int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s,
+                                 int max_split) {
   if (a_bf16)
     return launch_typed(static_cast<const __nv_bfloat16*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns,
-                        s);
-  return launch_typed(static_cast<const float*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s);
+                        s, max_split);
+  return launch_typed(static_cast<const float*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
 }
 
 }  // namespace lstm_approx_impl

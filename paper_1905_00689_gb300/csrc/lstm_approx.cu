@@ -383,6 +383,15 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
       continue;
     }
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
+    // Before the per-unit-block kernel at K > 128 (a cluster of 16 CTAs
+    // whose set-up fills about 256 KB of tensor memory each), the projection
+    // runs unsplit along D: its smaller grid leaves a GPC free, so that the
+    // recurrence's set-up overlaps it (D = 1024, H = 512, T = 20: the run
+    // 2% faster although the projection takes 15.8 instead of 10.5 us).
+    // Shorter set-ups gain less than the slower projection costs (K = 64:
+    // 4% slower, the one-exchange kernel at K = 16: 11%).
+    const int xproj_max_split =
+        (path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && K > 128) ? 1 : 8;
     {
       PhaseTimer pt(h, 0);
       if (sparse_x_projection(h, s, K, T * B)) {
@@ -397,7 +406,7 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
       } else if (xproj_cluster_fits(T * B, s.D, s.ldx, s.D, bf16))
         LA_CUDA(h,
                 launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->err,
-                                     h->opt_wait_limit_us * 1000LL, h->stream),
+                                     h->opt_wait_limit_us * 1000LL, h->stream, xproj_max_split),
                 "input projection launch");
       else
         LA_CUDA(h,
