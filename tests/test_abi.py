@@ -81,3 +81,41 @@ def test_product_path_does_not_import_the_oracle():
                 text = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(from|import)\s+oracle", text, flags=re.M), f
                 assert "oracle/" not in text, f
+
+
+def _header_enum(prefix):
+    """name -> value of the header's enumerators starting with `prefix`."""
+    text = open(os.path.join(ROOT, "include", "lstm_approx.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return {m.group(1): int(m.group(2)) for m in re.finditer(r"\b(" + prefix + r"\w+)\s*=\s*(\d+)", text)}
+
+
+def test_binding_constants_match_the_header():
+    """The Python binding's option, query, path and status numbers are the
+    header's, so a key added on one side cannot drift from the other."""
+    from paper_1905_00689_gb300 import _binding as b
+    for prefix, strip in (("LSTM_APPROX_OPT_", "LSTM_APPROX_"), ("LSTM_APPROX_Q_", "LSTM_APPROX_"),
+                          ("LSTM_APPROX_PATH_", "LSTM_APPROX_")):
+        enum = _header_enum(prefix)
+        assert enum, prefix
+        for name, value in enum.items():
+            py = name[len(strip):]
+            assert getattr(b, py) == value, (py, getattr(b, py, None), value)
+
+
+def test_bench_helpers():
+    """p90 is the nearest-rank 90th percentile; the captured DRAM traffic is
+    reported only while the recurrence kernel's sources match the capture."""
+    import sys
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.p90([5.0]) == 5.0
+    assert bench.p90(list(range(1, 11))) == 9
+    assert bench.p90(list(range(100))) == 89
+    assert bench.captured_traffic() in (None, bench.TRAFFIC_CAPTURE["bytes"])
+    saved = dict(bench.TRAFFIC_CAPTURE)
+    try:
+        bench.TRAFFIC_CAPTURE["sha256"] = "0" * 64  # sources that no longer match the capture
+        assert bench.captured_traffic() is None
+    finally:
+        bench.TRAFFIC_CAPTURE.update(saved)
