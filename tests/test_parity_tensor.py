@@ -30,6 +30,10 @@ def _sample(got, streams, T=None):
     (64, 128, 3, 16, 64, 96, []),            # one tile of everything
     (40, 200, 4, 3, 80, 70, [16, 48, 80]),    # ragged H, B, K; depths inside and at the end of chunks
     (300, 136, 2, 130, 128, 150, [64]),       # two stream tiles, ragged tail
+    # one output tile: the gate GEMM's terms split 4 and 8 ways, depths on
+    # split boundaries, inside splits and at K
+    (48, 128, 3, 8, 256, 100, [64, 96, 128, 192, 256]),
+    (32, 128, 2, 4, 512, 60, [16, 320, 512]),
 ])
 def test_tensor_path_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     gates = [draw_factor_set(H, D + H, K, nz, 5100 + 7 * D + g) for g in range(4)]
