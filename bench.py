@@ -338,6 +338,7 @@ def run_ours(args):
     large = [] if (args.quick or args.no_large) else large_batch_sweep(dev, stream, peaks_bf16())
     paper_case = None if (args.quick or args.no_large) else paper_case_sweep(dev, stream)
     dense = None if args.quick else dense_comparator(dev, stream, x)
+    k_sweeps = [] if (args.quick or args.no_large) else workload_k_sweeps(dev, flush)
 
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
@@ -388,6 +389,7 @@ def run_ours(args):
             "cluster_ctas": cluster, "persistent_kernel": {1: "per-unit-block", 2: "one-exchange"}.get(variant),
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
             "large_batch": large,
+            "k_sweeps": k_sweeps,
             "paper_case_study": paper_case,
             "dense_lstm_comparator": dense,
         }
@@ -401,6 +403,74 @@ def run_ours(args):
 
 LARGE_BATCH = (("c3", 0.5, 512, ()), ("c4", 0.5, 512, ()), ("c4", 0.1, 128, ()),
                ("c5", 0.3, 1024, (16, 64, 256, 1024)))
+
+
+# throughput against K on the other workloads: (workload, dtype, keep, K values);
+# one model per row holds the largest K, and each smaller K runs its prefix
+K_SWEEPS = (("c1", "fp32", 0.5, (1, 4, 16, 64)),
+            ("c3", "bf16", 0.5, (32, 128, 512)),
+            ("c4", "bf16", 0.5, (8, 32, 128, 512)),
+            ("c4", "bf16", 0.1, (8, 32, 128, 512)))
+
+
+def workload_k_sweeps(dev, flush):
+    """Timesteps·streams/s and p50 per-timestep latency against K for each
+    row of K_SWEEPS (no intermediate outputs, L2 flushed before every run),
+    eager and replayed as a CUDA graph.  Runs on a stream of its own (the
+    default stream cannot be captured)."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, Q_LAST_PATH
+    torch.cuda.synchronize(dev)  # the flush buffer was last written on another stream
+    stream = torch.cuda.Stream(dev)
+    out = []
+    with torch.cuda.stream(stream):
+        for name, dtype, keep, Ks in K_SWEEPS:
+            out.append(_k_sweep_row(dev, stream, flush, WORKLOADS[name], dtype, keep, Ks, LSTMApprox, Q_LAST_PATH))
+            torch.cuda.empty_cache()
+    torch.cuda.synchronize(dev)
+    return out
+
+
+def _k_sweep_row(dev, stream, flush, w, dtype, keep, Ks, LSTMApprox, Q_LAST_PATH):
+    import torch
+    km = max(Ks)
+    m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, km, w.B, dtype, stream=stream)
+    for l in range(w.L):
+        m.set_layer(l, synthetic_layer_factors(w, l, km, keep))
+    x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+    oh = torch.empty((w.T, w.B, w.H), device=dev)
+    row = {"workload": w.name, "dtype": dtype, "keep": keep, "points": []}
+    n = 50 if w.B == 1 else 10
+
+    def timed(fn):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for i, (a, b) in enumerate(evs):
+            flush.fill_(float(i))
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        return [a.elapsed_time(b) for a, b in evs]
+
+    for K in Ks:
+        for _ in range(3):
+            m.run(x, K, oh)
+        t = timed(lambda: m.run(x, K, oh))
+        path = m.query(Q_LAST_PATH)
+        # the same call captured once as a CUDA graph: the device time of its
+        # launches without the host's enqueue between them
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            m.run(x, K, oh)
+        g.replay()
+        tg = timed(g.replay)
+        del g
+        row["points"].append({
+            "K": K, "value": w.T * w.B / (statistics.mean(t) / 1e3), "unit": UNIT,
+            "p50_us_per_timestep": 1e3 * statistics.median(t) / w.T,
+            "p50_us_per_timestep_graph": 1e3 * statistics.median(tg) / w.T,
+            "path": {1: "simt", 2: "persistent", 3: "tensor"}.get(path)})
+    return row
 
 
 def peaks_bf16():
@@ -556,6 +626,11 @@ def run_profile(args):
     cps = list(w.checkpoints)
     if w.name == WL.name:  # the configuration of the main timed loop
         keep, K, cps = KEEP, K_MAIN, list(CKPTS)
+    if args.profile_k:
+        K = args.profile_k
+        cps = [c for c in cps if c < K] + [K] if cps else []
+    if args.profile_keep:
+        keep = args.profile_keep
     dev = torch.device("cuda", 0)
     m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, K, w.B, w.dtype)
     for l in range(w.L):
@@ -580,6 +655,8 @@ def main():
     ap.add_argument("--no-large", action="store_true", help="skip the large-batch tensor-core measurements")
     ap.add_argument("--profile", choices=sorted(WORKLOADS), default=None,
                     help="only run one workload's path (warmup + steps runs), for profilers")
+    ap.add_argument("--profile-k", type=int, default=0, help="with --profile: this K instead of the workload's largest")
+    ap.add_argument("--profile-keep", type=float, default=0.0, help="with --profile: this keep fraction")
     ap.add_argument("--quick", action="store_true",
                     help="main timed loop only (short side measurements, no K sweep, no CPU baseline)")
     args = ap.parse_args()

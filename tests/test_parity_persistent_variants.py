@@ -31,7 +31,7 @@ def _check(layers, x, K, variant, cluster=0, **kw):
 
 
 @pytest.mark.parametrize("variant", [1, 2])
-@pytest.mark.parametrize("K", [1, 16, 64])
+@pytest.mark.parametrize("K", [1, 4, 16, 64])
 def test_small_workload(cuda_device, variant, K):
     layers = [list(decomposed_layer("c1", 0, 64, 0.5))]
     x = workload_inputs(WORKLOADS["c1"])

@@ -72,6 +72,19 @@ def test_throughput_workload_full_size(cuda_device, K):
     assert_parity(_sample(got, streams), ref, BF16_TOL)
 
 
+@pytest.mark.parametrize("K,cps", [(8, []), (24, [16]), (40, [16, 32])])
+def test_prefix_of_stored_terms(cuda_device, K, cps):
+    """Runs at K below the stored rank, with K not a multiple of the MMA's 16
+    terms: the terms past K in the last slice must contribute nothing."""
+    D, H, T, B, KS = 72, 128, 3, 24, 96
+    gates = [draw_factor_set(H, D + H, KS, 60, 6100 + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 8)
+    got, m = run_gpu([gates], x, K, dtype="bf16", checkpoints=cps, force_path=PATH_TENSOR, max_rank=KS)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    ref = oracle_run([gates], x, K, dtype="bf16", checkpoints=cps)
+    assert_parity(got, ref, BF16_TOL)
+
+
 def test_throughput_workload_decomposed_factors(cuda_device):
     w = WORKLOADS["c3"]
     layers = [list(decomposed_layer("c3", 0, 32, 0.5))]
