@@ -113,3 +113,21 @@ def test_many_streams_take_the_persistent_path(cuda_device, D, H, T, B, K):
     assert m.query(Q_LAST_PATH) == PATH_PERSISTENT
     ref = oracle_run([gates], x, K, checkpoints=[8])
     assert_parity(got, ref, FP32_TOL)
+
+
+@pytest.mark.parametrize("D,H,T,K,nz,cps,cs,variant", [
+    (256, 1024, 3, 128, 380, [16, 100], 0, 1),  # V_h in tensor memory, 32 h values per lane
+    (200, 768, 4, 40, 290, [7, 40], 0, 1),      # the same with lanes past H reading zeros
+    (128, 384, 3, 256, 150, [64, 130], 0, 1),   # V_h and U in tensor memory, 8 units per warp
+    (128, 384, 3, 100, 150, [33], 8, 1),        # 16 units per warp
+    (128, 384, 3, 100, 150, [33, 64], 0, 2),    # one-exchange kernel, four h quarters per thread
+])
+def test_wider_hidden_sizes(cuda_device, D, H, T, K, nz, cps, cs, variant):
+    """Hidden sizes other than the workloads': each selects another
+    instantiation of the kernel's on-chip layout."""
+    layers = [[draw_factor_set(H, D + H, K, nz, 4400 + H + g) for g in range(4)]]
+    x = draw_inputs(T, 1, D, "relu", H)
+    rng = np.random.default_rng(H)
+    h0 = 0.5 * rng.standard_normal((1, 1, H))
+    c0 = 0.5 * rng.standard_normal((1, 1, H))
+    _check(layers, x, K, variant, cluster=cs, checkpoints=cps, h0=h0, c0=c0)
