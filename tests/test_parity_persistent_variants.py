@@ -131,3 +131,46 @@ def test_wider_hidden_sizes(cuda_device, D, H, T, K, nz, cps, cs, variant):
     h0 = 0.5 * rng.standard_normal((1, 1, H))
     c0 = 0.5 * rng.standard_normal((1, 1, H))
     _check(layers, x, K, variant, cluster=cs, checkpoints=cps, h0=h0, c0=c0)
+
+
+# The per-unit-block kernel is compiled for each combination of units per
+# warp (the smallest power of two with 4 * UW >= the CTA's units, about
+# H / CS), terms per lane (the smallest power of two with 32 * KT >= K) and
+# where V_h lives (shared memory up to H = 256, tensor memory with U up to
+# 512, tensor memory with 32 h values per lane up to 1024).  One case per
+# compiled combination, ragged hidden sizes, two intermediate depths.
+_UB_LAYOUTS = [  # (H, cluster size) for UW = 1, 2, 4, 8, 16 with V_h in shared memory
+    (36, 16), (100, 16), (196, 16), (196, 8), (196, 4)]
+_KT = {1: 23, 2: 50, 4: 100, 8: 200}  # a K for each number of terms per lane
+
+
+def _layout_cases():
+    cases = []
+    for i, (H, cs) in enumerate(_UB_LAYOUTS):
+        for kt in (1, 2, 4, 8) if i < 4 else (1, 2, 4):
+            cases.append((H, _KT[kt], cs))
+    for kt in (1, 2, 4, 8):
+        cases.append((388, _KT[kt], 16))  # UW = 8, V_h and U in tensor memory
+    for kt in (1, 2, 4):
+        cases.append((388, _KT[kt], 8))   # UW = 16, V_h and U in tensor memory
+        cases.append((772, _KT[kt], 16))  # UW = 16, V_h in tensor memory, 32 values per lane
+    return cases
+
+
+@pytest.mark.parametrize("H,K,cs", _layout_cases())
+def test_per_unit_block_kernel_every_layout(cuda_device, H, K, cs):
+    D, T = 40, 3
+    layers = [[draw_factor_set(H, D + H, K, 30, 5100 + H + K + g) for g in range(4)]]
+    x = draw_inputs(T, 1, D, "uniform", H + K)
+    _check(layers, x, K, 1, cluster=cs, checkpoints=[K // 3, K - 7])
+
+
+# The one-exchange kernel: each thread keeps HQ quarters of h (1 up to H = 128,
+# 2 up to 256, 4 up to 512), at each cluster size.
+@pytest.mark.parametrize("H", [100, 200, 340])
+@pytest.mark.parametrize("cs,K", [(4, 60), (8, 120), (16, 250)])
+def test_one_exchange_kernel_every_layout(cuda_device, H, cs, K):
+    D, T = 40, 3
+    layers = [[draw_factor_set(H, D + H, K, 30, 5300 + H + K + g) for g in range(4)]]
+    x = draw_inputs(T, 1, D, "relu", H + K)
+    _check(layers, x, K, 2, cluster=cs, checkpoints=[K // 3, K - 7])
