@@ -85,6 +85,20 @@ def test_prefix_of_stored_terms(cuda_device, K, cps):
     assert_parity(got, ref, BF16_TOL)
 
 
+def test_widest_stream_tile(cuda_device):
+    """Enough gate tiles that the gate GEMM takes 128 streams per tile
+    (10 unit tiles x 16 tiles of 64 streams would exceed one wave); ragged
+    last tile, checked on sampled streams."""
+    D, H, T, B, K = 64, 1280, 2, 1000, 48
+    gates = [draw_factor_set(H, D + H, K, 200, 6300 + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 31)
+    got, m = run_gpu([gates], x, K, dtype="bf16", checkpoints=[16, 32], force_path=PATH_TENSOR)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    streams = [0, 517, 895, 999]
+    ref = oracle_run([gates], x[:, streams], K, dtype="bf16", checkpoints=[16, 32])
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
 def test_throughput_workload_decomposed_factors(cuda_device):
     w = WORKLOADS["c3"]
     layers = [list(decomposed_layer("c3", 0, 32, 0.5))]
