@@ -245,6 +245,53 @@ int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
  */
 int lstm_approx_phase_times(lstm_approx_t *h, float *ms_out);
 
+/*
+ * Which kernels lstm_approx_run takes for one layer of this shape, by the
+ * same rules as the run: the path, the persistent kernel with its cluster
+ * size and on-chip layout, and the tensor-core tiles and term splits.  Host
+ * only: no handle, no device, nothing launched.
+ *
+ *   dtype        enum lstm_approx_dtype of the factors
+ *   hidden       H >= 1;  T, B, K >= 1: timesteps, streams, refinement depth
+ *   checkpoints  host array [J] of the layer's intermediate depths k_j
+ *                (strictly increasing, in [1, K]); NULL when J = 0
+ *   force_path, cluster, persistent_variant
+ *                the values of LSTM_APPROX_OPT_FORCE_PATH, _CLUSTER and
+ *                _PERSISTENT_VARIANT (0 = automatic)
+ *   out          host array [n_out]; out[i] receives item i of enum
+ *                lstm_approx_plan_item (0 where an item does not apply to
+ *                the chosen path, and for i >= LSTM_APPROX_PLAN_ITEMS)
+ *   msg          optional host buffer of msg_len bytes for an error text
+ *
+ * Returns OK, or EINVAL for invalid arguments and for a forced path or
+ * kernel that cannot take the shape (where lstm_approx_run returns EINVAL).
+ * The input projection's kernel, which also depends on the factors' masks,
+ * is not reported.
+ */
+enum lstm_approx_plan_item {
+  LSTM_APPROX_PLAN_PATH = 0,               /* enum lstm_approx_path */
+  LSTM_APPROX_PLAN_PERSISTENT_VARIANT = 1, /* 1 per-unit-block, 2 one-exchange kernel */
+  LSTM_APPROX_PLAN_CLUSTER = 2,            /* CTAs per stream */
+  LSTM_APPROX_PLAN_TERMS_PER_CTA = 3,      /* coefficient rows a CTA owns (per-unit-block:
+                                              gate-major rows of all four gates; one-exchange:
+                                              terms of one gate) */
+  LSTM_APPROX_PLAN_UNITS_PER_WARP = 4,     /* per-unit-block: hidden units per warp, 1..16 */
+  LSTM_APPROX_PLAN_TERMS_PER_LANE = 5,     /* per-unit-block: terms per lane, 1..8 */
+  LSTM_APPROX_PLAN_VH_LAYOUT = 6,          /* per-unit-block: 0 V_h in shared memory, 1 V_h and
+                                              U in tensor memory, 2 V_h in tensor memory at 32
+                                              values per lane */
+  LSTM_APPROX_PLAN_H_QUADS = 7,            /* one-exchange: h quads per lane, 1, 2 or 4 */
+  LSTM_APPROX_PLAN_SMEM_BYTES = 8,         /* persistent: dynamic shared memory per CTA */
+  LSTM_APPROX_PLAN_TMEM_COLUMNS = 9,       /* persistent: tensor-memory columns per CTA */
+  LSTM_APPROX_PLAN_TAU_TILE_STREAMS = 10,  /* tensor path: streams per tile of the tau' GEMM */
+  LSTM_APPROX_PLAN_GATE_TILE_STREAMS = 11, /* tensor path: streams per tile of the gate GEMM */
+  LSTM_APPROX_PLAN_GATE_SPLITS = 12,       /* tensor path: term-axis splits of the gate GEMM */
+  LSTM_APPROX_PLAN_ITEMS = 13
+};
+int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int *checkpoints, int J,
+                     int force_path, int cluster, int persistent_variant, int *out, int n_out,
+                     char *msg, int msg_len);
+
 #ifdef __cplusplus
 }
 #endif

@@ -22,6 +22,12 @@ FP32, BF16 = 0, 1
 Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT = range(5)
 PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
 OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ = range(7)
+(PLAN_PATH, PLAN_PERSISTENT_VARIANT, PLAN_CLUSTER, PLAN_TERMS_PER_CTA, PLAN_UNITS_PER_WARP, PLAN_TERMS_PER_LANE,
+ PLAN_VH_LAYOUT, PLAN_H_QUADS, PLAN_SMEM_BYTES, PLAN_TMEM_COLUMNS, PLAN_TAU_TILE_STREAMS, PLAN_GATE_TILE_STREAMS,
+ PLAN_GATE_SPLITS, PLAN_ITEMS) = range(14)
+PLAN_KEYS = ("path", "persistent_variant", "cluster", "terms_per_cta", "units_per_warp", "terms_per_lane",
+             "vh_layout", "h_quads", "smem_bytes", "tmem_columns", "tau_tile_streams", "gate_tile_streams",
+             "gate_splits")
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ETIMEOUT: "ETIMEOUT",
                 ESTATE: "ESTATE"}
 
@@ -29,6 +35,7 @@ EXPORTS = (
     "lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_run_host",
     "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
     "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times", "lstm_approx_run_static",
+    "lstm_approx_plan",
 )
 
 _lib = None
@@ -66,6 +73,7 @@ def load(path: str = LIB_PATH):
     lib.lstm_approx_phase_times.argtypes = [P, ctypes.POINTER(ctypes.c_float)]
     lib.lstm_approx_run_static.argtypes = [P, P, P, P, P, I, I, I, P, I, I, P, P, P, P, P, I, P, P, P,
                                            ctypes.c_char_p, I]
+    lib.lstm_approx_plan.argtypes = [I, I, I, I, I, P, I, I, I, I, P, I, ctypes.c_char_p, I]
     for name in EXPORTS:
         if name not in ("lstm_approx_last_error", "lstm_approx_destroy"):
             getattr(lib, name).restype = ctypes.c_int
@@ -108,6 +116,21 @@ def run_static(Vx, Vh, U, sigma, bias, x, K, out_h, h0=None, c0=None, out_c=None
                                     _ptr(ckpt_h), _ptr(ckpt_c), ctypes.c_void_p(stream.cuda_stream), msg, 512)
     if rc != OK:
         raise LSTMApproxError(rc, msg.value.decode())
+
+
+def plan(dtype: int, hidden: int, T: int, B: int, K: int, checkpoints: Sequence[int] = (), force_path: int = 0,
+         cluster: int = 0, variant: int = 0) -> dict:
+    """lstm_approx_plan: the kernels a run of one layer of this shape takes,
+    as a dict keyed by PLAN_KEYS (host only, no device needed)."""
+    lib = load()
+    cps = (ctypes.c_int * max(1, len(checkpoints)))(*checkpoints)
+    out = (ctypes.c_int * PLAN_ITEMS)()
+    msg = ctypes.create_string_buffer(512)
+    rc = lib.lstm_approx_plan(dtype, hidden, T, B, K, cps, len(checkpoints), force_path, cluster, variant, out,
+                              PLAN_ITEMS, msg, 512)
+    if rc != OK:
+        raise LSTMApproxError(rc, msg.value.decode())
+    return dict(zip(PLAN_KEYS, list(out)))
 
 
 class LSTMApprox:

@@ -191,11 +191,61 @@ bool sparse_x_projection(const lstm_approx_t* h, const LayerStore& s, int K, int
 
 // The tensor path takes bf16 factors; its intermediate depths must fall on
 // the 16-term slices of one MMA instruction.
-bool tensor_path_fits(const lstm_approx_t* h, const Checkpoints& ck) {
-  if (h->dtype != LSTM_APPROX_BF16) return false;
+bool tensor_path_fits(int dtype, const Checkpoints& ck) {
+  if (dtype != LSTM_APPROX_BF16) return false;
   for (int j = 0; j < ck.n; ++j)
     if (ck.k[j] % 16 != 0) return false;
   return true;
+}
+
+// Recurrence path of one layer.  Automatic: bf16 factors take the
+// tensor-core path when the depths allow it; fp32 factors take a persistent
+// launch whenever a plan fits, at any batch (one cluster per stream;
+// clusters beyond one wave run in the next); everything else takes the
+// CUDA-core kernels.  A forced path that cannot take the shape returns 0
+// with the reason in *why.  *plan is filled for the persistent path.
+int select_path(int dtype, int H, int K, int T, const Checkpoints& ck, int force_path, int want_cs, int sm_count,
+                int variant, PersistentChoice* plan, std::string* why) {
+  const bool bf16 = dtype == LSTM_APPROX_BF16;
+  const bool tensor_ok = tensor_path_fits(dtype, ck);
+  if (force_path == 0) {
+    if (tensor_ok) return LSTM_APPROX_PATH_TENSOR;
+    if (!bf16 && choose_persistent(H, K, T, ck, want_cs, sm_count, variant, plan, why))
+      return LSTM_APPROX_PATH_PERSISTENT;
+    return LSTM_APPROX_PATH_SIMT;
+  }
+  if (force_path == LSTM_APPROX_PATH_PERSISTENT) {
+    if (bf16) {
+      *why = "the persistent path runs fp32 factors only";
+      return 0;
+    }
+    std::string r;
+    if (!choose_persistent(H, K, T, ck, want_cs, sm_count, variant, plan, &r)) {
+      *why = "persistent path unavailable: " + r;
+      return 0;
+    }
+  } else if (force_path == LSTM_APPROX_PATH_TENSOR && !tensor_ok) {
+    *why = "tensor path needs bf16 factors and intermediate depths that are multiples of 16";
+    return 0;
+  }
+  return force_path;
+}
+
+struct TensorTiles {
+  int bnh = 0, nt = 0, ks = 1, nkb_per = 0;
+};
+
+// Tiles of the tensor-core path for one layer: streams per tile of the tau'
+// GEMM (bnh) and of the gate GEMM (nt), and the gate GEMM's term-axis
+// splits (ks, of nkb_per 64-term chunks each; small grids split the terms
+// over more CTAs).
+TensorTiles tensor_tiles(int H, int B, int K) {
+  TensorTiles t;
+  t.bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
+  t.nt = tc_gates_tile_n(H, B);
+  const int gate_tiles = ((H + 127) / 128) * ((B + t.nt - 1) / t.nt);
+  t.ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &t.nkb_per);
+  return t;
 }
 
 int ensure_factor_maps(lstm_approx_t* h, int l) {
@@ -261,12 +311,8 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
   LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
   h->launches += 1;
-  const int bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
-  const int nt = tc_gates_tile_n(H, B);
-  // small grids (few streams) split the gate GEMM's terms over more CTAs
-  int nkb_per = 0;
-  const int gate_tiles = ((H + 127) / 128) * ((B + nt - 1) / nt);
-  const int ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &nkb_per);
+  const TensorTiles tt = tensor_tiles(H, B, K);
+  const int bnh = tt.bnh, nt = tt.nt, ks = tt.ks, nkb_per = tt.nkb_per;
   if (ks > 1) {
     const size_t need = (size_t)(ks + ck.n) * 4 * B * H * sizeof(float);
     if (need > h->gpart_bytes) {
@@ -351,27 +397,11 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     const Checkpoints none = {0, {0}};
     const Checkpoints& lck = top ? ck : none;
     // recurrence path
-    int path = h->opt_force_path;
     PersistentChoice plan;
     std::string why;
-    const bool tensor_ok = bf16 && tensor_path_fits(h, lck);
-    if (path == 0) {
-      path = LSTM_APPROX_PATH_SIMT;
-      if (tensor_ok) path = LSTM_APPROX_PATH_TENSOR;
-      // fp32 factors: a persistent launch whenever a plan fits, at any batch
-      // (one cluster per stream; clusters beyond one wave run in the next)
-      else if (!bf16 &&
-               choose_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, h->opt_persistent_variant, &plan, &why))
-        path = LSTM_APPROX_PATH_PERSISTENT;
-    } else if (path == LSTM_APPROX_PATH_PERSISTENT) {
-      if (bf16) return fail(h, LSTM_APPROX_EINVAL, "the persistent path runs fp32 factors only");
-      if (!choose_persistent(H, K, T, lck, h->opt_cluster, h->sm_count, h->opt_persistent_variant, &plan, &why))
-        return fail(h, LSTM_APPROX_EINVAL, "persistent path unavailable: %s", why.c_str());
-    } else if (path == LSTM_APPROX_PATH_TENSOR) {
-      if (!tensor_ok)
-        return fail(h, LSTM_APPROX_EINVAL,
-                    "tensor path needs bf16 factors and intermediate depths that are multiples of 16");
-    }
+    const int path = select_path(h->dtype, H, K, T, lck, h->opt_force_path, h->opt_cluster, h->sm_count,
+                                 h->opt_persistent_variant, &plan, &why);
+    if (path == 0) return fail(h, LSTM_APPROX_EINVAL, "%s", why.c_str());
     const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
     const float* l_c0 = c0 ? c0 + (size_t)l * B * H : nullptr;
     float* l_cout = out_c ? out_c + (size_t)l * B * H : nullptr;
@@ -489,6 +519,17 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
   }
   if (h->timing.on) cudaEventRecord(h->timing.run1, h->stream);
   return LSTM_APPROX_OK;
+}
+
+// Error text into a caller's buffer (entry points without a handle).
+int report(char* msg, int msg_len, int code, const char* fmt, ...) {
+  if (msg && msg_len > 0) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(msg, (size_t)msg_len, fmt, ap);
+    va_end(ap);
+  }
+  return code;
 }
 
 }  // namespace
@@ -876,6 +917,62 @@ int lstm_approx_phase_times(lstm_approx_t* h, float* ms_out) {
     ms_out[h->timing.phase[i / 2]] += ms;
   }
   LA_CUDA(h, cudaEventElapsedTime(&ms_out[2], h->timing.run0, h->timing.run1), "event time");
+  return LSTM_APPROX_OK;
+}
+
+int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int* checkpoints, int J, int force_path,
+                     int cluster, int persistent_variant, int* out, int n_out, char* msg, int msg_len) {
+  if (msg && msg_len > 0) msg[0] = '\0';
+  const int E = LSTM_APPROX_EINVAL;
+  if (dtype != LSTM_APPROX_FP32 && dtype != LSTM_APPROX_BF16) return report(msg, msg_len, E, "bad dtype %d", dtype);
+  if (hidden < 1 || T < 1 || B < 1 || K < 1)
+    return report(msg, msg_len, E, "hidden=%d, T=%d, B=%d and K=%d must be >= 1", hidden, T, B, K);
+  if (J < 0 || J > kMaxCheckpoints) return report(msg, msg_len, E, "J=%d outside [0, %d]", J, kMaxCheckpoints);
+  if (J > 0 && !checkpoints) return report(msg, msg_len, E, "checkpoints is NULL with J=%d", J);
+  Checkpoints ck;
+  ck.n = J;
+  for (int j = 0; j < kMaxCheckpoints; ++j) ck.k[j] = 0;
+  for (int j = 0; j < J; ++j) {
+    const int k = checkpoints[j];
+    if (k < 1 || k > K) return report(msg, msg_len, E, "checkpoint %d = %d outside [1, K=%d]", j, k, K);
+    if (j > 0 && k <= checkpoints[j - 1]) return report(msg, msg_len, E, "checkpoints must be strictly increasing");
+    ck.k[j] = k;
+  }
+  if (force_path < 0 || force_path > 3) return report(msg, msg_len, E, "bad path %d", force_path);
+  if (cluster != 0 && cluster != 1 && cluster != 2 && cluster != 4 && cluster != 8 && cluster != 16)
+    return report(msg, msg_len, E, "bad cluster size %d", cluster);
+  if (persistent_variant < 0 || persistent_variant > 2)
+    return report(msg, msg_len, E, "bad persistent variant %d", persistent_variant);
+  if (n_out < 0 || (n_out > 0 && !out)) return report(msg, msg_len, E, "out is NULL with n_out=%d", n_out);
+  PersistentChoice pc;
+  std::string why;
+  const int path = select_path(dtype, hidden, K, T, ck, force_path, cluster, 0, persistent_variant, &pc, &why);
+  if (path == 0) return report(msg, msg_len, E, "%s", why.c_str());
+  int v[LSTM_APPROX_PLAN_ITEMS] = {};
+  v[LSTM_APPROX_PLAN_PATH] = path;
+  if (path == LSTM_APPROX_PATH_PERSISTENT) {
+    v[LSTM_APPROX_PLAN_PERSISTENT_VARIANT] = pc.variant;
+    v[LSTM_APPROX_PLAN_CLUSTER] = pc.CS;
+    if (pc.variant == 1) {
+      v[LSTM_APPROX_PLAN_TERMS_PER_CTA] = pc.ub.RA;
+      v[LSTM_APPROX_PLAN_UNITS_PER_WARP] = pc.ub.upl;
+      v[LSTM_APPROX_PLAN_TERMS_PER_LANE] = pc.ub.kpw;
+      v[LSTM_APPROX_PLAN_VH_LAYOUT] = pc.ub.hc;
+      v[LSTM_APPROX_PLAN_SMEM_BYTES] = (int)pc.ub.smem;
+      v[LSTM_APPROX_PLAN_TMEM_COLUMNS] = pc.ub.tcols;
+    } else {
+      v[LSTM_APPROX_PLAN_TERMS_PER_CTA] = pc.ag.RA;
+      v[LSTM_APPROX_PLAN_H_QUADS] = pc.ag.hq;
+      v[LSTM_APPROX_PLAN_SMEM_BYTES] = (int)pc.ag.smem;
+      v[LSTM_APPROX_PLAN_TMEM_COLUMNS] = pc.ag.tcols;
+    }
+  } else if (path == LSTM_APPROX_PATH_TENSOR) {
+    const TensorTiles tt = tensor_tiles(hidden, B, K);
+    v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = tt.bnh;
+    v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = tt.nt;
+    v[LSTM_APPROX_PLAN_GATE_SPLITS] = tt.ks;
+  }
+  for (int i = 0; i < n_out; ++i) out[i] = i < LSTM_APPROX_PLAN_ITEMS ? v[i] : 0;
   return LSTM_APPROX_OK;
 }
 

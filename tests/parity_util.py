@@ -119,4 +119,29 @@ def assert_parity(got, ref, tol, keys=("h", "c_last", "ckpt_h", "ckpt_c"), metri
 
 
 __all__ = ["FP32_TOL", "BF16_TOL", "max_rel_err", "max_rel_err_vec", "decomposed_layer", "synthetic_layer", "run_gpu",
-           "oracle_run", "assert_parity", "workload_inputs", "WORKLOADS"]
+           "oracle_run", "assert_parity", "workload_inputs", "WORKLOADS", "persistent_layout_cases"]
+
+
+# The per-unit-block kernel is compiled for each combination of units per
+# warp (the smallest power of two with 4 * UW >= the CTA's units, about
+# H / CS), terms per lane (the smallest power of two with 32 * KT >= K) and
+# where V_h lives (shared memory up to H = 256, tensor memory with U up to
+# 512, tensor memory with 32 h values per lane up to 1024).
+# persistent_layout_cases() gives one (H, K, cluster size) for each compiled
+# combination, with ragged hidden sizes.
+UB_LAYOUTS = [  # (H, cluster size) for UW = 1, 2, 4, 8, 16 with V_h in shared memory
+    (36, 16), (100, 16), (196, 16), (196, 8), (196, 4)]
+LAYOUT_K = {1: 23, 2: 50, 4: 100, 8: 200}  # a K for each number of terms per lane
+
+
+def persistent_layout_cases():
+    cases = []
+    for i, (H, cs) in enumerate(UB_LAYOUTS):
+        for kt in (1, 2, 4, 8) if i < 4 else (1, 2, 4):
+            cases.append((H, LAYOUT_K[kt], cs))
+    for kt in (1, 2, 4, 8):
+        cases.append((388, LAYOUT_K[kt], 16))  # UW = 8, V_h and U in tensor memory
+    for kt in (1, 2, 4):
+        cases.append((388, LAYOUT_K[kt], 8))   # UW = 16, V_h and U in tensor memory
+        cases.append((772, LAYOUT_K[kt], 16))  # UW = 16, V_h in tensor memory, 32 values per lane
+    return cases

@@ -95,7 +95,7 @@ def test_binding_constants_match_the_header():
     header's, so a key added on one side cannot drift from the other."""
     from paper_1905_00689_gb300 import _binding as b
     for prefix, strip in (("LSTM_APPROX_OPT_", "LSTM_APPROX_"), ("LSTM_APPROX_Q_", "LSTM_APPROX_"),
-                          ("LSTM_APPROX_PATH_", "LSTM_APPROX_")):
+                          ("LSTM_APPROX_PATH_", "LSTM_APPROX_"), ("LSTM_APPROX_PLAN_", "LSTM_APPROX_")):
         enum = _header_enum(prefix)
         assert enum, prefix
         for name, value in enum.items():

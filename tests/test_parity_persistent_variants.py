@@ -11,9 +11,9 @@ ranges (several inside one range, one at K), and ragged shapes.
 import numpy as np
 import pytest
 
-from parity_util import (FP32_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run, run_gpu,
-                         synthetic_layer, workload_inputs)
-from paper_1905_00689_gb300 import PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_PERSISTENT_VARIANT
+from parity_util import (FP32_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run,
+                         persistent_layout_cases, run_gpu, synthetic_layer, workload_inputs)
+from paper_1905_00689_gb300 import FP32, PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_PERSISTENT_VARIANT, plan
 from workloads import draw_factor_set, draw_inputs
 
 pytestmark = pytest.mark.gpu
@@ -25,6 +25,10 @@ def _check(layers, x, K, variant, cluster=0, **kw):
     assert m.query(Q_PERSISTENT_VARIANT) == variant
     if cluster:
         assert m.query(Q_CLUSTER) == cluster
+    # the host-side plan of the same shape names the kernel that ran
+    T, B = x.shape[:2]
+    p = plan(FP32, layers[0][0]["u"].shape[1], T, B, K, kw.get("checkpoints", ()), PATH_PERSISTENT, cluster, variant)
+    assert (m.query(Q_CLUSTER), m.query(Q_PERSISTENT_VARIANT)) == (p["cluster"], p["persistent_variant"])
     ref = oracle_run(layers, x, K, **{k: v for k, v in kw.items() if k in ("h0", "c0", "checkpoints")})
     assert_parity(got, ref, FP32_TOL)
     return got
@@ -133,31 +137,9 @@ def test_wider_hidden_sizes(cuda_device, D, H, T, K, nz, cps, cs, variant):
     _check(layers, x, K, variant, cluster=cs, checkpoints=cps, h0=h0, c0=c0)
 
 
-# The per-unit-block kernel is compiled for each combination of units per
-# warp (the smallest power of two with 4 * UW >= the CTA's units, about
-# H / CS), terms per lane (the smallest power of two with 32 * KT >= K) and
-# where V_h lives (shared memory up to H = 256, tensor memory with U up to
-# 512, tensor memory with 32 h values per lane up to 1024).  One case per
-# compiled combination, ragged hidden sizes, two intermediate depths.
-_UB_LAYOUTS = [  # (H, cluster size) for UW = 1, 2, 4, 8, 16 with V_h in shared memory
-    (36, 16), (100, 16), (196, 16), (196, 8), (196, 4)]
-_KT = {1: 23, 2: 50, 4: 100, 8: 200}  # a K for each number of terms per lane
-
-
-def _layout_cases():
-    cases = []
-    for i, (H, cs) in enumerate(_UB_LAYOUTS):
-        for kt in (1, 2, 4, 8) if i < 4 else (1, 2, 4):
-            cases.append((H, _KT[kt], cs))
-    for kt in (1, 2, 4, 8):
-        cases.append((388, _KT[kt], 16))  # UW = 8, V_h and U in tensor memory
-    for kt in (1, 2, 4):
-        cases.append((388, _KT[kt], 8))   # UW = 16, V_h and U in tensor memory
-        cases.append((772, _KT[kt], 16))  # UW = 16, V_h in tensor memory, 32 values per lane
-    return cases
-
-
-@pytest.mark.parametrize("H,K,cs", _layout_cases())
+# One case per compiled layout of the per-unit-block kernel (see
+# parity_util.persistent_layout_cases), ragged hidden sizes, two depths.
+@pytest.mark.parametrize("H,K,cs", persistent_layout_cases())
 def test_per_unit_block_kernel_every_layout(cuda_device, H, K, cs):
     D, T = 40, 3
     layers = [[draw_factor_set(H, D + H, K, 30, 5100 + H + K + g) for g in range(4)]]
