@@ -73,6 +73,28 @@ def test_no_cpu_fallback_without_a_device(built_lib):
     assert h.value is None
 
 
+def test_header_is_c_and_a_c_client_links(built_lib, tmp_path):
+    """tests/c_client.c, compiled as strict C99 against the header and linked
+    to the library, gets the documented answers from the device-free calls."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    pkg = os.path.join(ROOT, "paper_1905_00689_gb300")
+    exe = str(tmp_path / "c_client")
+    subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
+                    os.path.join(ROOT, "tests", "c_client.c"), "-L", pkg, "-llstm_approx", "-Wl,-rpath," + pkg,
+                    "-o", exe], check=True, capture_output=True, text=True)
+    lines = subprocess.run([exe], check=True, capture_output=True, text=True).stdout.splitlines()
+    assert lines[0] == "plan 0 path 2 variant 1 cluster 16"
+    assert lines[1].startswith("forced 1 ") and "fp32 factors only" in lines[1]
+    import torch
+    if not torch.cuda.is_available():
+        assert lines[2] == "create 3 null"  # ECUDA: no CPU fallback
+    assert lines[3] == "error invalid handle (NULL)"
+
+
 def test_product_path_does_not_import_the_oracle():
     pkg = os.path.join(ROOT, "paper_1905_00689_gb300")
     for dirpath, _, files in os.walk(pkg):
