@@ -15,7 +15,7 @@ Follows Sec. III of the paper:
   takes the top singular triplet of the residual R^(n) = W - W~^(n-1), prunes
   its v, and adds sigma u prune(v)^T to the running approximation W~.
 
-Readings where the paper is silent (stated again in the design doc):
+Readings where the paper is silent:
 * ties in the magnitude ranking go to the lower column index; the kept index
   list is stored in ascending order;
 * the triplet's sign is fixed so that v's largest-magnitude entry (lowest

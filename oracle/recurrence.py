@@ -15,7 +15,7 @@ Per timestep t and stream b (Sec. II, Fig. 2; Sec. III):
    forget and output gates use the logistic sigmoid, the cell gate tanh;
    c_t = f * c_{t-1} + i * g,  h_t = o * tanh(c_t).
 
-Readings (stated again in the design doc): gates are ordered (i, f, g, o); the
+Readings: gates are ordered (i, f, g, o); the
 paper writes no bias, so the optional per-gate bias defaults to zero and is
 exact (not approximated); the carried state h_t, c_t always uses the full
 depth K, and the output at depth k_j applies step 3 to the k_j-prefix sums
