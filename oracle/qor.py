@@ -14,7 +14,16 @@ Eq. 1 at each pruning level, and for every (NZ, K) it reports
   seeded random linear head A (classes x H, N(0, 1/sqrt(H))) standing in
   for the model's output layer;
 * the operations per timestep of Sec. III, 4 gates x K (2R + 2NZ + 1),
-  against the dense 4 x 2RC.
+  against the dense 4 x 2RC;
+* the relative Frobenius error of the gate matrices themselves,
+  ||W - W~^(K)|| / ||W|| over the four gates.
+
+Two schemes are compared: the residual refinement of Eq. 1, where each
+term is the top triplet of what the pruned terms before it left over, and
+the non-residual scheme Sec. III contrasts it with, where the terms are the
+first K singular triplets of W itself, each pruned afterwards.  Without
+pruning the two coincide (deflation by exact triplets leaves the remaining
+ones).
 
 ``python -m oracle.qor`` prints the tables for the small workload and the
 paper's case-study shape.
@@ -26,7 +35,7 @@ from typing import Dict, List, Sequence
 
 import numpy as np
 
-from .factors import decompose_gate
+from .factors import decompose_gate, decompose_gate_variant
 from .recurrence import lstm_cell, op_count, run_lstm
 
 
@@ -51,32 +60,61 @@ def softmax(z: np.ndarray) -> np.ndarray:
     return e / e.sum(axis=-1, keepdims=True)
 
 
+def reconstruct(f: dict, K: int, C: int) -> np.ndarray:
+    """W~^(K) = sum_{n<K} sigma_n u_n prune(v_n)^T of one gate's factors."""
+    V = np.zeros((K, C))
+    for n in range(K):
+        V[n, f["idx"][n]] = f["val"][n]
+    return (f["u"][:K].T * f["sigma"][:K]) @ V
+
+
 def qor_table(weights: Sequence[np.ndarray], x: np.ndarray, nzs: Sequence[int], Ks: Sequence[int],
-              classes: int = 10, seed: int = 1905) -> List[Dict]:
-    """One row per (NZ, K): relative h error, head KL, ops per timestep."""
+              classes: int = 10, seed: int = 1905, scheme: str = "residual") -> List[Dict]:
+    """One row per (NZ, K): relative h error, head KL, ops per timestep,
+    relative gate-matrix error.  scheme: "residual" (Eq. 1) or "truncated"
+    (the first K triplets of W, each pruned)."""
+    if scheme not in ("residual", "truncated"):
+        raise ValueError(scheme)
     H, C = weights[0].shape
     h_ref = dense_lstm(weights, x)
     A = np.random.Generator(np.random.PCG64(seed)).normal(0.0, 1.0 / np.sqrt(H), (classes, H))
     p_ref = softmax(h_ref @ A.T)
+    w_norm = np.sqrt(sum(float(np.sum(W * W)) for W in weights))
     rows = []
     for nz in nzs:
-        layer = [decompose_gate(W, max(Ks), nz) for W in weights]
+        if scheme == "residual":
+            layer = [decompose_gate(W, max(Ks), nz) for W in weights]
+        else:
+            layer = [decompose_gate_variant(W, max(Ks), nz, residual=False) for W in weights]
         for K in Ks:
             h = run_lstm([layer], x, K)["h"]
             p = softmax(h @ A.T)
             kl = float(np.mean(np.sum(p_ref * (np.log(p_ref) - np.log(p)), axis=-1)))
-            rows.append({"NZ": nz, "K": K,
+            w_err = np.sqrt(sum(float(np.sum((W - reconstruct(f, K, C)) ** 2)) for W, f in zip(weights, layer)))
+            rows.append({"NZ": nz, "K": K, "scheme": scheme,
                          "rel_h_error": float(np.linalg.norm(h - h_ref) / np.linalg.norm(h_ref)),
                          "head_kl": kl,
+                         "rel_w_error": w_err / w_norm,
                          "ops": 4 * op_count(H, nz, K), "dense_ops": 4 * 2 * H * C})
     return rows
 
 
 def markdown(rows: List[Dict]) -> str:
-    lines = ["| NZ | K | rel. h error | head KL | ops / step | fraction of dense ops |", "|---|---|---|---|---|---|"]
+    lines = ["| NZ | K | rel. h error | head KL | rel. W error | ops / step | fraction of dense ops |",
+             "|---|---|---|---|---|---|---|"]
     for r in rows:
-        lines.append(f"| {r['NZ']} | {r['K']} | {r['rel_h_error']:.3g} | {r['head_kl']:.3g} | {r['ops']} | "
-                     f"{r['ops'] / r['dense_ops']:.3g} |")
+        lines.append(f"| {r['NZ']} | {r['K']} | {r['rel_h_error']:.3g} | {r['head_kl']:.3g} | "
+                     f"{r['rel_w_error']:.3g} | {r['ops']} | {r['ops'] / r['dense_ops']:.3g} |")
+    return "\n".join(lines)
+
+
+def markdown_schemes(res: List[Dict], trunc: List[Dict]) -> str:
+    """The two schemes side by side, row for row."""
+    lines = ["| NZ | K | rel. W error, residual | rel. W error, truncated | rel. h error, residual | "
+             "rel. h error, truncated |", "|---|---|---|---|---|---|"]
+    for a, b in zip(res, trunc):
+        lines.append(f"| {a['NZ']} | {a['K']} | {a['rel_w_error']:.3g} | {b['rel_w_error']:.3g} | "
+                     f"{a['rel_h_error']:.3g} | {b['rel_h_error']:.3g} |")
     return "\n".join(lines)
 
 
@@ -89,7 +127,13 @@ def main(argv: Sequence[str]) -> None:
         nzs = [nz_from_keep(k, w.C()) for k in w.keeps] if name == "f1" else [w.C(), nz_from_keep(0.5, w.C()),
                                                                               nz_from_keep(0.125, w.C())]
         print(f"## {w.name} (H={w.H}, C={w.C()}, T={T})\n")
-        print(markdown(qor_table(weights, x, nzs, w.Ks)))
+        res = qor_table(weights, x, nzs, w.Ks)
+        print(markdown(res))
+        print()
+        pruned = [nz for nz in nzs if nz < w.C()]
+        res_p = [r for r in res if r["NZ"] in pruned]
+        print(f"### residual refinement against truncated SVD then pruning ({w.name})\n")
+        print(markdown_schemes(res_p, qor_table(weights, x, pruned, w.Ks, scheme="truncated")))
         print()
 
 

@@ -36,6 +36,7 @@ def test_full_rank_unpruned_has_zero_error_and_kl():
     rows = qor.qor_table(W, x, nzs=[C], Ks=[H])
     assert rows[0]["rel_h_error"] < 1e-12
     assert abs(rows[0]["head_kl"]) < 1e-12
+    assert rows[0]["rel_w_error"] < 1e-12
 
 
 def test_truncation_and_pruning_raise_the_error():
@@ -50,3 +51,40 @@ def test_truncation_and_pruning_raise_the_error():
     for r in rows.values():
         assert r["head_kl"] >= -1e-15
         assert r["ops"] == 4 * r["K"] * (2 * H + 2 * r["NZ"] + 1)
+
+
+def test_schemes_coincide_without_pruning():
+    """Deflating W by exact singular triplets leaves the remaining ones, so
+    without pruning the residual refinement and the truncated SVD are the
+    same approximation at every K (Eckart-Young)."""
+    D, H, T = 10, 6, 4
+    C = D + H
+    W = _weights(H, C, 600)
+    x = draw_inputs(T, 1, D, "uniform", 6)
+    res = qor.qor_table(W, x, nzs=[C], Ks=[1, 2, 4, 6])
+    trunc = qor.qor_table(W, x, nzs=[C], Ks=[1, 2, 4, 6], scheme="truncated")
+    for a, b in zip(res, trunc):
+        for key in ("rel_h_error", "head_kl", "rel_w_error"):
+            assert abs(a[key] - b[key]) < 1e-9, (a["K"], key, a[key], b[key])
+
+
+def test_residual_matrix_error_never_increases():
+    """||W - W~^(n+1)||^2 = ||W - W~^(n)||^2 - sigma_n^2 ||prune(v_n)||^2:
+    with any pruning the residual scheme's error falls or stays with K, and
+    the law holds term by term."""
+    D, H, T = 12, 8, 3
+    C = D + H
+    W = _weights(H, C, 700)
+    x = draw_inputs(T, 1, D, "uniform", 7)
+    for nz in (3, 9):
+        rows = qor.qor_table(W, x, nzs=[nz], Ks=list(range(1, 13)))
+        errs = [r["rel_w_error"] for r in rows]
+        assert all(b <= a + 1e-12 for a, b in zip(errs, errs[1:])), errs
+    from oracle import decompose_gate
+    f = decompose_gate(W[0], 6, 5)
+    prev = float(np.sum(W[0] ** 2))
+    for K in range(1, 7):
+        cur = float(np.sum((W[0] - qor.reconstruct(f, K, C)) ** 2))
+        drop = f["sigma"][K - 1] ** 2 * float(np.sum(f["val"][K - 1] ** 2))
+        assert abs(prev - cur - drop) < 1e-10 * max(1.0, prev)
+        prev = cur
