@@ -99,6 +99,26 @@ def qor_table(weights: Sequence[np.ndarray], x: np.ndarray, nzs: Sequence[int], 
     return rows
 
 
+def pareto(rows: List[Dict], cost: str = "ops", err: str = "rel_h_error") -> List[Dict]:
+    """The candidate designs (NZ, K) of Sec. III that no other candidate
+    beats: a row stays unless another has cost <= and error <= with one of
+    them strictly lower.  Sorted by cost."""
+    keep = []
+    for r in rows:
+        dominated = any(o[cost] <= r[cost] and o[err] <= r[err] and (o[cost] < r[cost] or o[err] < r[err])
+                        for o in rows)
+        if not dominated:
+            keep.append(r)
+    return sorted(keep, key=lambda r: (r[cost], r[err]))
+
+
+def best_within(rows: List[Dict], budget: float, cost: str = "ops", err: str = "rel_h_error"):
+    """The candidate with the lowest error among those whose cost fits the
+    budget (the cheaper one on a tie), or None if none fits."""
+    fit = [r for r in rows if r[cost] <= budget]
+    return min(fit, key=lambda r: (r[err], r[cost])) if fit else None
+
+
 def markdown(rows: List[Dict]) -> str:
     lines = ["| NZ | K | rel. h error | head KL | rel. W error | ops / step | fraction of dense ops |",
              "|---|---|---|---|---|---|---|"]
@@ -134,6 +154,9 @@ def main(argv: Sequence[str]) -> None:
         res_p = [r for r in res if r["NZ"] in pruned]
         print(f"### residual refinement against truncated SVD then pruning ({w.name})\n")
         print(markdown_schemes(res_p, qor_table(weights, x, pruned, w.Ks, scheme="truncated")))
+        print()
+        print(f"### candidate designs (NZ, K) no other beats on ops and h error ({w.name})\n")
+        print(markdown(pareto(res)))
         print()
 
 

@@ -88,3 +88,30 @@ def test_residual_matrix_error_never_increases():
         drop = f["sigma"][K - 1] ** 2 * float(np.sum(f["val"][K - 1] ** 2))
         assert abs(prev - cur - drop) < 1e-10 * max(1.0, prev)
         prev = cur
+
+
+def test_design_selection_by_definition():
+    """A hand-checked set: (ops, error) pairs where b and d are beaten by a
+    and c respectively, e ties a on error at a higher cost, and f is the
+    most accurate."""
+    rows = [{"name": n, "ops": o, "rel_h_error": e} for n, o, e in
+            [("a", 10, 0.5), ("b", 12, 0.6), ("c", 20, 0.3), ("d", 20, 0.4), ("e", 15, 0.5), ("f", 40, 0.1)]]
+    assert [r["name"] for r in qor.pareto(rows)] == ["a", "c", "f"]
+    assert qor.best_within(rows, 9) is None
+    assert qor.best_within(rows, 15)["name"] == "a"   # e has the same error at a higher cost
+    assert qor.best_within(rows, 39)["name"] == "c"
+    assert qor.best_within(rows, 40)["name"] == "f"
+
+
+def test_every_front_design_is_the_best_at_its_own_cost():
+    D, H, T = 12, 8, 3
+    C = D + H
+    W = _weights(H, C, 800)
+    x = draw_inputs(T, 1, D, "uniform", 8)
+    rows = qor.qor_table(W, x, nzs=[C, 10, 4], Ks=[1, 2, 4, 8])
+    front = qor.pareto(rows)
+    assert front and all(r in rows for r in front)
+    for r in front:
+        assert qor.best_within(rows, r["ops"]) is r
+    errs = [r["rel_h_error"] for r in front]
+    assert all(b < a for a, b in zip(errs, errs[1:]))   # more cost buys strictly less error along the front
