@@ -151,7 +151,7 @@ struct CellArgs {
 };
 cudaError_t launch_cell_step(const CellArgs& a, cudaStream_t s);
 
-// ---- persistent cluster kernel (fp32 factors, small batch) ---------------
+// ---- persistent cluster kernels (fp32 factors, one cluster per stream) -----
 
 struct PersistentPlan {
   int CS = 0;        // CTAs per cluster

@@ -23,6 +23,13 @@
 // thread commits, the epilogue warps compute the cell from the partial sums
 // and hand the accumulators back -- no prefix is recomputed.
 //
+// When the stream tiles are too few to fill the GPU (small B), the gate
+// GEMM's term axis is split over up to 8 CTAs per tile (grid z, 64-term
+// chunks [kb0, kb1) each).  Such a CTA stores its raw gate sums, and at a
+// depth that ends inside its range the sums up to that depth, to a scratch
+// array; tc_gates_reduce_kernel then adds the splits in split order and runs
+// the cell update at full depth and at every intermediate depth.
+//
 // Every mbarrier wait is bounded in wall time; a wait that runs out writes
 // the device status word, the CTA stops issuing work, waits (bounded) for
 // its copies and MMAs in flight, frees its tensor memory and returns.

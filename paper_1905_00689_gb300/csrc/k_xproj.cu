@@ -26,7 +26,7 @@ namespace {
 using namespace lstm_approx_dev;
 
 constexpr int kRows = 32;     // rows per CTA
-constexpr int kCols = 32;     // max columns (T*B)
+constexpr int kCols = 32;     // columns per launch chunk (grid z covers T*B <= 256)
 constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kGrp = 128;     // values of D per staged group (one commit group)
