@@ -191,6 +191,22 @@ int lstm_approx_sync(lstm_approx_t *h);
  */
 int lstm_approx_get_mask(lstm_approx_t *h, int layer, int gate, int k, int32_t *idx_out, int *nz_out);
 
+/*
+ * Read back term k (0 <= k < K set) of (layer, gate) as the device storage
+ * holds it, i.e. after the rounding of lstm_approx_set_factors: sigma, u
+ * and prune(v) of Eq. 1 (Sec. III), each stored value widened exactly to
+ * fp32 (a bf16 value is the upper half of its fp32 pattern).
+ *
+ *   sigma_out  host [1]
+ *   u_out      host [H]
+ *   v_out      host [C] (C = D_layer + H): dense, zero at pruned columns
+ *
+ * Synchronises the handle's stream.  Errors: EINVAL (range, NULL), ECUDA.
+ * Used to check the stored values bit for bit against the rounding rule.
+ */
+int lstm_approx_get_term(lstm_approx_t *h, int layer, int gate, int k, float *sigma_out, float *u_out,
+                         float *v_out);
+
 /* Text of the handle's last error ("" if none).  Static text for NULL. */
 const char *lstm_approx_last_error(const lstm_approx_t *h);
 

@@ -35,7 +35,7 @@ EXPORTS = (
     "lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_run_host",
     "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
     "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times", "lstm_approx_run_static",
-    "lstm_approx_plan",
+    "lstm_approx_plan", "lstm_approx_get_term",
 )
 
 _lib = None
@@ -64,6 +64,7 @@ def load(path: str = LIB_PATH):
     lib.lstm_approx_run_host.argtypes = run_args
     lib.lstm_approx_sync.argtypes = [P]
     lib.lstm_approx_get_mask.argtypes = [P, I, I, I, P, ctypes.POINTER(I)]
+    lib.lstm_approx_get_term.argtypes = [P, I, I, I, P, P, P]
     lib.lstm_approx_last_error.argtypes = [P]
     lib.lstm_approx_last_error.restype = ctypes.c_char_p
     lib.lstm_approx_destroy.argtypes = [P]
@@ -220,6 +221,15 @@ class LSTMApprox:
         n = ctypes.c_int(0)
         self._check(self.lib.lstm_approx_get_mask(self.h, layer, gate, k, _np_ptr(out), ctypes.byref(n)))
         return out[: n.value].copy()
+
+    def get_term(self, layer: int, gate: int, k: int):
+        """(sigma, u [H], dense v [C]) of one stored term, as fp32 numpy arrays."""
+        C = self.input_dims[layer] + self.H
+        sigma = np.zeros(1, dtype=np.float32)
+        u = np.zeros(self.H, dtype=np.float32)
+        v = np.zeros(C, dtype=np.float32)
+        self._check(self.lib.lstm_approx_get_term(self.h, layer, gate, k, _np_ptr(sigma), _np_ptr(u), _np_ptr(v)))
+        return float(sigma[0]), u, v
 
     def query(self, key: int) -> int:
         v = ctypes.c_longlong(0)

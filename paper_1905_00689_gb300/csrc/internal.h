@@ -73,10 +73,11 @@ struct lstm_approx {
   size_t cap_TB = 0;          // capacity (T*B) of the T-dependent scratch
   float* Px = nullptr;        // [T*B][4*Ks] hoisted input projection
   float* seq = nullptr;       // [T*B][H] output sequence of a lower layer
-  void* tau = nullptr;        // [max_batch][4*Ks] refinement coefficients (fp32, or bf16 on the tensor path)
-  void* x_bf16 = nullptr;     // [T*B][ldx of layer 0] bf16 input (tensor path)
-  void* seq_bf16 = nullptr;   // [T*B][ldh] bf16 sequence between layers (tensor path)
-  void* h_bf16 = nullptr;     // [max_batch][ldh] bf16 h operand (tensor path)
+  void* tau = nullptr;        // [max_batch][4*Ks] refinement coefficients (fp32; on the tensor path
+                              // the bf16 pair planes [2][B][4*Ks], the same bytes)
+  void* x_bf16 = nullptr;     // [2][T*B][ldx of layer 0] bf16 pair of the input (tensor path)
+  void* seq_bf16 = nullptr;   // [2][T*B][ldh] bf16 pair of the sequence between layers (tensor path)
+  void* h_bf16 = nullptr;     // [2][B][ldh] bf16 pair of the h operand (tensor path)
   int* err = nullptr;         // device status word (0 = ok)
   int* err_host = nullptr;    // pinned host copy of it, read after the stream synchronises
 
@@ -112,10 +113,10 @@ cudaError_t launch_rows_gemm(const void* A, bool a_bf16, int lda, int K, int Ks,
 // Same product for few columns (N = T*B <= 256, in chunks of 32): clusters
 // split the D axis, rows are staged by asynchronous copies and the chunk
 // sums pushed to their owner CTA (deterministic).  Needs D % 8 == 0 and
-// 16-byte aligned rows; a push that does not arrive within limit_ns sets
-// *err.  max_split caps the CTAs per cluster along D (1: one CTA per row
-// tile and column chunk).
-bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16);
+// 16-byte aligned base pointers and rows; a push that does not arrive
+// within limit_ns sets *err.  max_split caps the CTAs per cluster along D
+// (1: one CTA per row tile and column chunk).
+bool xproj_cluster_fits(int N, int D, const void* A, int lda, const float* X, int ldxin, bool a_bf16);
 
 // Compressed x part of the pruned v (fp32 factors): per gate, the kept x
 // columns of row k are entries off[g][k] .. off[g][k+1] of idx[g] / val[g].
@@ -219,6 +220,9 @@ bool choose_persistent(int H, int K, int T, const Checkpoints& ck, int want_cs, 
 cudaError_t launch_persistent_choice(const PersistentChoice& c, const PersistentArgs& a, cudaStream_t s);
 
 // ---- tensor-core path (bf16, tcgen05 / TMEM / TMA) -----------------------
+// Activations (x, h, tau') enter the MMAs as bf16 pairs hi = bf16(a),
+// lo = bf16(a - hi), stored as two planes: the hi plane of R rows, then the
+// lo plane of R rows, so one tensor map of 2R rows covers both.
 
 // 2-D K-major bf16 tensor [rows][inner] with `pitch_bytes` between rows, as
 // TMA tiles of 64 inner elements x box_rows rows, 128-byte swizzled.
@@ -232,12 +236,14 @@ struct TcRowsArgs {
   int K, Ks;         // refinement depth of the run; gate stride of the packed rows
   int kt_per_gate;   // 128-row tiles per gate: ceil(K / 128)
   int N;             // valid columns (T*B for the projection, B for tau')
-  int mode;          // 0: P[n][row] = sum; 1: tau[n][row] = bf16(sigma[row] (sum + P[n][row])), 0 for k >= K
+  int b_plane;       // rows of one plane of the activation's map (its lo plane starts there)
+  int mode;          // 0: P[n][row] = sum; 1: tau[n][row] = pair of sigma[row] (sum + P[n][row]), 0 for k >= K
   float* P;          // [N][ldp]
   int ldp;
   const float* sigma;
-  __nv_bfloat16* tau;  // [N][ldt]
+  __nv_bfloat16* tau;  // planes [2][N][ldt]: hi, then lo at tau + tau_plane
   int ldt;
+  long long tau_plane;
   int* err;
   long long limit_ns;
 };
@@ -247,13 +253,20 @@ cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a,
 struct TcGatesArgs {
   int H, K, Ks, B;
   int nkb;                  // 64-term chunks: ceil(K / 64)
+  int tau_rows;             // rows of one plane of tau's map (B: the lo plane starts there)
+  const __nv_bfloat16* U;   // factor U [4][H][Ks] and the stored tau' pair [2][B][ldt]: the terms of an
+  const __nv_bfloat16* tau; // intermediate depth that is not a multiple of 16 past the last 16-term slice
+  int ldt;                  // are added from these on the CUDA cores
+  long long tau_plane;
   const float* bias;        // [4][H]
   float* c_state;           // [B][H] fp32, c_{t-1} in, c_t out
-  __nv_bfloat16* h_bf16;    // [B][ldh] h_t out (next step's operand)
+  __nv_bfloat16* h_bf16;    // planes [2][B][ldh]: h_t out (next step's operand), lo at h_bf16 + h_plane
   int ldh;
+  long long h_plane;
   float* out_h;             // [B][H] fp32 h_t (this timestep) or null
-  __nv_bfloat16* seq_bf16;  // [B][ldh] h_t for the next layer (this timestep) or null
-  Checkpoints ck;           // depths, multiples of 16
+  __nv_bfloat16* seq_bf16;  // [B][ldh] h_t for the next layer (this timestep; lo at seq_bf16 + seq_plane) or null
+  long long seq_plane;
+  Checkpoints ck;           // intermediate depths
   float* ckpt_h;            // element (j, n, unit) at j*ck_stride + n*H + unit (this timestep) or null
   float* ckpt_c;
   long long ck_stride;

@@ -1,4 +1,13 @@
-// Large-batch tensor-core path (bf16 factors and operands, fp32 accumulate).
+// Large-batch tensor-core path (bf16 factors, fp32 accumulate).
+//
+// The factors u, v are stored in bf16.  The activations x, h and tau' are
+// fp32 values; each enters the MMAs as a pair of bf16 planes, hi = bf16(a)
+// and lo = bf16(a - hi), so that hi + lo equals a to about 2^-17 relative
+// and every product is issued twice (factor tile x hi, factor tile x lo)
+// into the same fp32 accumulator.  Rounding the activations to one bf16
+// (unit roundoff 2^-9) instead gives elementwise errors of 0.03-0.2 on h
+// and c; with the pair the kernels differ from fp64 arithmetic on the same
+// bf16 factors by a few 1e-4.
 //
 // The two products of one timestep are dense contractions over B streams:
 //   (a2) tau'[n][(g,k)] = sigma_{g,k} (P_t[n][(g,k)] + sum_j Vh[(g,k)][j] h_{t-1}[n][j])
@@ -7,18 +16,19 @@
 // h over all T*B columns (Eq. 1 with the augmentation of Sec. III).
 //
 // tc_rows_kernel computes one 128-row x BN-column tile of the first kind:
-// warp 0 streams K-major tiles of both operands with TMA (128-byte swizzle)
-// through an S-stage mbarrier ring, one thread of warp 1 issues
-// tcgen05.mma (M = 128, N = BN, K = 16 per instruction) into a tensor-memory
-// accumulator, and warps 4..11 (two per 32-lane quarter of tensor memory)
-// read it back with tcgen05.ld for the epilogue: store P, or form tau' in
-// bf16.  For tau' the epilogue warps load their P_t values while the
-// mainloop streams: into registers for tiles up to 128 columns, otherwise
-// into the accumulator with tcgen05.st so that the MMAs accumulate on top.
+// warp 0 streams K-major tiles of the factor and of both planes of the
+// activation with TMA (128-byte swizzle) through an S-stage mbarrier ring,
+// one thread of warp 1 issues tcgen05.mma (M = 128, N = BN, K = 16 per
+// instruction, once per plane) into a tensor-memory accumulator, and warps
+// 4..11 (two per 32-lane quarter of tensor memory) read it back with
+// tcgen05.ld for the epilogue: store P, or form tau' and store it as its
+// bf16 pair.  For tau' the epilogue warps load their P_t values into
+// registers while the mainloop streams.
 //
 // tc_gates_kernel computes, for 128 hidden units x NT streams, the four gate
 // sums at once in four tensor-memory accumulators and runs the cell update
-// of Sec. II in the epilogue.  Intermediate depths k_j (multiples of 16) are
+// of Sec. II in the epilogue (fp32 sigmoid and tanh, relative error a few
+// 1e-7), storing h_t as its bf16 pair for the next step.  Intermediate depths k_j (multiples of 16) are
 // read from the same accumulators when the MMA stream reaches them: the MMA
 // thread commits, the epilogue warps compute the cell from the partial sums
 // and hand the accumulators back -- no prefix is recomputed.
@@ -55,6 +65,56 @@ __device__ __forceinline__ bool wait_cta(uint32_t mb, uint32_t parity, uint64_t 
   return mbar_wait_bounded<false>(mb, parity, limit, err);
 }
 
+// The bf16 pair of an fp32 value: hi = bf16(v), lo = bf16(v - hi), both
+// round-to-nearest-even (v - hi is exact in fp32).
+__device__ __forceinline__ void bf16_pair(float v, __nv_bfloat16& hi, __nv_bfloat16& lo) {
+  hi = __float2bfloat16_rn(v);
+  lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& w, float* f) {
+  const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    f[2 * e] = __uint_as_float(v[e] << 16);
+    f[2 * e + 1] = __uint_as_float(v[e] & 0xFFFF0000u);
+  }
+}
+
+// Gate sums at an intermediate depth k_j that is not a multiple of 16: the
+// MMA stream stopped at the slice boundary k0 = k_j - r (0 < r < 16), and
+// this adds the r terms [k0, k_j) for unit j and the 16 streams from nbeg,
+// y[g][c] += sum_{k0 <= k < k_j} u_{g,k}[j] (tau'_hi + tau'_lo)[n][(g, k)],
+// from the factor U and the stored tau' pair, on the CUDA cores.
+__device__ __noinline__ void add_remainder_terms(const TcGatesArgs& a, int j, int nbeg, int k0, int r,
+                                                 float (&y)[4][16]) {
+#pragma unroll 1
+  for (int g = 0; g < 4; ++g) {
+    float u[16];
+    const uint4* up = reinterpret_cast<const uint4*>(a.U + ((long long)g * a.H + j) * a.Ks + k0);
+    bf16x8_to_f32(__ldg(up), u);
+    bf16x8_to_f32(__ldg(up + 1), u + 8);
+#pragma unroll 1
+    for (int c = 0; c < 16; ++c) {
+      const int n = nbeg + c;
+      if (n >= a.B) break;
+      const long long o = (long long)n * a.ldt + (long long)g * a.Ks + k0;
+      const uint4* th = reinterpret_cast<const uint4*>(a.tau + o);
+      const uint4* tl = reinterpret_cast<const uint4*>(a.tau + a.tau_plane + o);
+      float hi[16], lo[16];
+      bf16x8_to_f32(th[0], hi);
+      bf16x8_to_f32(th[1], hi + 8);
+      bf16x8_to_f32(tl[0], lo);
+      bf16x8_to_f32(tl[1], lo + 8);
+      float acc = 0.f;
+#pragma unroll
+      for (int k = 0; k < 16; ++k)
+        if (k < r) acc = fmaf(u[k], hi[k] + lo[k], acc);
+      y[g][c] += acc;
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
 // tile of tau' / P: rows of the packed factor matrix x columns (streams)
 // ---------------------------------------------------------------------------
@@ -62,14 +122,15 @@ template <int BN, int S>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_rows_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, TcRowsArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  constexpr uint32_t kBBytes = BN * kTileK * 2;
+  static_assert(BN <= 128, "the epilogue holds P_t of its columns in registers");
+  constexpr uint32_t kBBytes = BN * kTileK * 2;        // one plane of the activation tile
+  constexpr uint32_t kStage = kABytes + 2 * kBBytes;   // factor tile, hi plane, lo plane
   constexpr uint32_t kCols = BN < 32 ? 32 : BN;
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t sA = base, sB = base + S * kABytes;
-  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | pinit | tmem slot
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 3));
-  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u, pinit_bar = accum_bar + 16u;
+  const uint32_t bar0 = base + S * kStage;  // full[S] | empty[S] | accum | drain | tmem slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 2));
+  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.x / a.kt_per_gate, kt = blockIdx.x % a.kt_per_gate;
@@ -79,10 +140,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
   const bool add_p = a.mode == 1;  // tau' = sigma * (accumulator + P_t)
-  // BN <= 128: the epilogue threads hold their P_t values in registers; wider
-  // tiles store P_t into the accumulator before the MMAs start
-  constexpr bool kPReg = BN <= 128;
-  const bool p_tmem = add_p && !kPReg;
 
   griddep_launch_dependents();  // the next kernel may start its own set-up
   if (threadIdx.x == 0) {
@@ -92,7 +149,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
-    mbar_init(pinit_bar, 8 * 32);
     fence_mbarrier_init_cluster();
   }
   if (warp == 2) {
@@ -113,18 +169,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // before this one: issue them before waiting for it
     const int npre = nkb < S ? nkb : S;
     for (int kb = 0; kb < npre; ++kb) {
-      mbar_arrive_expect_tx(bar0 + 8u * kb, kABytes + kBBytes);
-      tma_load_2d(sA + kb * kABytes, &tma, bar0 + 8u * kb, kb * kTileK, row0);
+      mbar_arrive_expect_tx(bar0 + 8u * kb, kStage);
+      tma_load_2d(base + kb * kStage, &tma, bar0 + 8u * kb, kb * kTileK, row0);
     }
     griddep_wait();
     for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % S;
       if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
+      const uint32_t st = base + s * kStage;
       if (kb >= npre) {
-        mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
-        tma_load_2d(sA + s * kABytes, &tma, bar0 + 8u * s, kb * kTileK, row0);
+        mbar_arrive_expect_tx(bar0 + 8u * s, kStage);
+        tma_load_2d(st, &tma, bar0 + 8u * s, kb * kTileK, row0);
       }
-      tma_load_2d(sB + s * kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
+      tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);                      // hi plane
+      tma_load_2d(st + kABytes + kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, a.b_plane + col0);  // lo plane
       ++issued;
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
@@ -136,19 +194,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, BN);
     bool ok = true;
-    if (p_tmem) {  // the accumulator starts from P_t
-      ok = wait_cta(pinit_bar, 0, limit, err);
-      tc_fence_after();
-    }
     for (int kb = 0; kb < nkb && ok; ++kb) {
       const int s = kb % S;
       if (!(ok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
       tc_fence_after();
-      const uint64_t da = umma_desc_sw128(sA + s * kABytes);
-      const uint64_t db = umma_desc_sw128(sB + s * kBBytes);
+      const uint32_t st = base + s * kStage;
+      const uint64_t da = umma_desc_sw128(st);
+      const uint64_t dhi = umma_desc_sw128(st + kABytes), dlo = umma_desc_sw128(st + kABytes + kBBytes);
 #pragma unroll
-      for (int kk = 0; kk < kTileK / 16; ++kk)
-        umma_bf16(tmem, da + 2ull * kk, db + 2ull * kk, idesc, (p_tmem || (kb | kk) != 0) ? 1u : 0u);
+      for (int kk = 0; kk < kTileK / 16; ++kk) {
+        umma_bf16(tmem, da + 2ull * kk, dhi + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        umma_bf16(tmem, da + 2ull * kk, dlo + 2ull * kk, idesc, 1u);
+      }
       umma_commit(bar0 + 8u * (S + s));  // frees the stage once these MMAs are done
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
@@ -164,35 +221,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int row = row0 + lrow;
     const bool row_ok = k < a.K;
     const uint32_t trow = tmem + ((32u * q) << 16);
-    float preg[kPReg ? kHalf : 1];  // P_t of this thread's row and columns
-    if (add_p && kPReg) {  // loaded while the mainloop runs
+    float preg[kHalf];  // P_t of this thread's row and columns, loaded while the mainloop runs
+    if (add_p) {
 #pragma unroll
-      for (int c = 0; c < (kPReg ? kHalf : 1); ++c) {
+      for (int c = 0; c < kHalf; ++c) {
         const int n = col0 + cbeg + c;
         preg[c] = (row_ok && n < a.N) ? __ldg(a.P + (long long)n * a.ldp + row) : 0.f;
       }
     }
     griddep_wait();  // the outputs below may still be read by the kernel before this one
-    if (p_tmem) {  // P_t of this tile -> tensor memory, while the mainloop runs
-      const float* __restrict__ P = a.P;
-#pragma unroll 1
-      for (int c0 = cbeg; c0 < cbeg + kHalf; c0 += 64) {
-        float pv[4][16];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int n = col0 + c0 + 16 * u + j;
-            pv[u][j] = (row_ok && n < a.N && c0 + 16 * u < cbeg + kHalf) ? __ldg(P + (long long)n * a.ldp + row) : 0.f;
-          }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (c0 + 16 * u < cbeg + kHalf) tmem_st16(trow + c0 + 16 * u, pv[u]);
-      }
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(pinit_bar);
-    }
     const bool ok = wait_cta(accum_bar, 0, limit, err);
     tc_fence_after();
     const float sig = (add_p && row_ok) ? a.sigma[row] : 0.f;
@@ -211,8 +248,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (!add_p) {
           if (row_ok) a.P[(long long)n * a.ldp + row] = v[j];
         } else {
-          const float acc = kPReg ? v[j] + preg[kPReg ? cc + j : 0] : v[j];
-          a.tau[(long long)n * a.ldt + row] = __float2bfloat16_rn(row_ok ? sig * acc : 0.f);
+          __nv_bfloat16 hi, lo;
+          bf16_pair(row_ok ? sig * (v[j] + preg[cc + j]) : 0.f, hi, lo);
+          a.tau[(long long)n * a.ldt + row] = hi;
+          a.tau[a.tau_plane + (long long)n * a.ldt + row] = lo;
         }
       }
     }
@@ -232,13 +271,13 @@ template <int NT, int S, bool SPLIT>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_gates_kernel(const __grid_constant__ CUtensorMap tmu, const __grid_constant__ CUtensorMap tmt, TcGatesArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  constexpr uint32_t kBBytes = NT * kTileK * 2;
+  constexpr uint32_t kBBytes = NT * kTileK * 2;       // one plane of the tau' tile
+  constexpr uint32_t kStage = kABytes + 2 * kBBytes;  // U tile, hi plane, lo plane
   constexpr uint32_t kCols = 4 * NT < 32 ? 32 : 4 * NT;
   static_assert(S >= 4, "a chunk of all four gates must be resident");
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t sA = base, sB = base + S * kABytes;
-  const uint32_t bar0 = sB + S * kBBytes;  // full[S] | empty[S] | accum | drain | ckpt | ckpt_done | slot
+  const uint32_t bar0 = base + S * kStage;  // full[S] | empty[S] | accum | drain | ckpt | ckpt_done | slot
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 4));
   const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
   const uint32_t ckpt_bar = accum_bar + 16u, ckpt_done = accum_bar + 24u;
@@ -294,18 +333,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // U tiles of the first S stages first: they do not depend on the kernel before this one
     const int npre = nst < S ? nst : S;
     for (int i = 0; i < npre; ++i) {
-      mbar_arrive_expect_tx(bar0 + 8u * i, kABytes + kBBytes);
-      tma_load_2d(sA + i * kABytes, &tmu, bar0 + 8u * i, (kb0 + (i >> 2)) * kTileK, (i & 3) * a.H + j0);
+      mbar_arrive_expect_tx(bar0 + 8u * i, kStage);
+      tma_load_2d(base + i * kStage, &tmu, bar0 + 8u * i, (kb0 + (i >> 2)) * kTileK, (i & 3) * a.H + j0);
     }
     griddep_wait();
     for (int i = 0; i < nst; ++i) {
       const int s = i % S, kb = kb0 + (i >> 2), g = i & 3;
       if (i >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((i / S) - 1) & 1, limit, err))) break;
+      const uint32_t st = base + s * kStage;
       if (i >= npre) {
-        mbar_arrive_expect_tx(bar0 + 8u * s, kABytes + kBBytes);
-        tma_load_2d(sA + s * kABytes, &tmu, bar0 + 8u * s, kb * kTileK, g * a.H + j0);
+        mbar_arrive_expect_tx(bar0 + 8u * s, kStage);
+        tma_load_2d(st, &tmu, bar0 + 8u * s, kb * kTileK, g * a.H + j0);
       }
-      tma_load_2d(sB + s * kBBytes, &tmt, bar0 + 8u * s, g * a.Ks + kb * kTileK, n0);
+      tma_load_2d(st + kABytes, &tmt, bar0 + 8u * s, g * a.Ks + kb * kTileK, n0);                         // hi
+      tma_load_2d(st + kABytes + kBBytes, &tmt, bar0 + 8u * s, g * a.Ks + kb * kTileK, a.tau_rows + n0);  // lo
       ++issued;
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
@@ -319,10 +360,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     int jj = jj_lo;
     for (int kl = 0; kl < nkb && ok; ++kl) {
       const int kb = kb0 + kl;
-      uint64_t da[4], db[4];
-      // 16-term slices of this chunk, cut where an intermediate depth ends;
-      // each gate's stage is used as soon as it lands and freed as soon as
-      // its last slice is issued
+      uint64_t da[4], dhi[4], dlo[4];
+      // 16-term slices of this chunk, cut at the last slice boundary at or
+      // below an intermediate depth (the epilogue adds the terms between the
+      // boundary and the depth); each gate's stage is used as soon as it
+      // lands and freed as soon as its last slice is issued
       int kk0 = 0;
       while (kk0 < 4 && ok) {
         int kk1 = 4;
@@ -333,11 +375,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           if (kk0 == 0) {
             if (!(ok = wait_cta(bar0 + 8u * s, (i / S) & 1, limit, err))) break;
             tc_fence_after();
-            da[g] = umma_desc_sw128(sA + s * kABytes);
-            db[g] = umma_desc_sw128(sB + s * kBBytes);
+            const uint32_t st = base + s * kStage;
+            da[g] = umma_desc_sw128(st);
+            dhi[g] = umma_desc_sw128(st + kABytes);
+            dlo[g] = umma_desc_sw128(st + kABytes + kBBytes);
           }
-          for (int kk = kk0; kk < kk1; ++kk)
-            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, db[g] + 2ull * kk, idesc, (kl | kk) != 0 ? 1u : 0u);
+          for (int kk = kk0; kk < kk1; ++kk) {
+            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, dhi[g] + 2ull * kk, idesc, (kl | kk) != 0 ? 1u : 0u);
+            umma_bf16(tmem + g * NT, da[g] + 2ull * kk, dlo[g] + 2ull * kk, idesc, 1u);
+          }
           if (kk1 == 4) umma_commit(bar0 + 8u * (S + s));  // frees this gate's stage
         }
         if (ok && cut_here) {  // partial sums up to depth k_jj are complete: hand them to the epilogue
@@ -387,6 +433,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                                limit, err);
       tc_fence_after();
       const bool write = ok && *err == 0 && unit_ok;
+      // an intermediate depth off the 16-term slices: the MMAs stopped at
+      // rem_k0, the last rem_r terms are added on the CUDA cores; when this
+      // CTA issued no MMA before rem_k0 the accumulator holds nothing yet
+      const int kj = final_sums ? 0 : a.ck.k[step];
+      const int rem_r = kj & 15, rem_k0 = kj - rem_r;
+      const bool acc_valid = final_sums || rem_k0 > kb0 * kTileK;
       if constexpr (SPLIT) {
         // raw gate sums of this CTA's terms: slot z for its whole range, slot
         // ks + step at a depth that ends inside it
@@ -397,6 +449,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
           tmem_wait_ld();
           if (!write) continue;
+          if (!acc_valid)
+#pragma unroll
+            for (int g = 0; g < 4; ++g)
+#pragma unroll
+              for (int c = 0; c < 16; ++c) y[g][c] = 0.f;
+          if (rem_r) add_remainder_terms(a, j, n0 + c0, rem_k0, rem_r, y);
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
             const int n = n0 + c0 + c;
@@ -430,13 +488,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
         tmem_wait_ld();
         if (!write) continue;
+        if (!acc_valid)
+#pragma unroll
+          for (int g = 0; g < 4; ++g)
+#pragma unroll
+            for (int c = 0; c < 16; ++c) y[g][c] = 0.f;
+        if (rem_r) add_remainder_terms(a, j, n0 + c0, rem_k0, rem_r, y);
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
           const int n = n0 + c0 + c;
           if (n >= a.B) break;
           const long long sj = (long long)n * a.H + j;
           float hh, cc;
-          lstm_cell_hw(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
+          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
           if (!final_sums) {
             const long long o = (long long)step * a.ck_stride + sj;  // (no split: jj_lo = 0)
             if (a.ckpt_h) a.ckpt_h[o] = hh;
@@ -444,9 +508,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           } else {
             a.c_state[sj] = cc;
             if (a.out_h) a.out_h[sj] = hh;
-            const __nv_bfloat16 hb = __float2bfloat16_rn(hh);
-            a.h_bf16[(long long)n * a.ldh + j] = hb;
-            if (a.seq_bf16) a.seq_bf16[(long long)n * a.ldh + j] = hb;
+            __nv_bfloat16 hi, lo;
+            bf16_pair(hh, hi, lo);
+            const long long hj = (long long)n * a.ldh + j;
+            a.h_bf16[hj] = hi;
+            a.h_bf16[a.h_plane + hj] = lo;
+            if (a.seq_bf16) {
+              a.seq_bf16[hj] = hi;
+              a.seq_bf16[a.seq_plane + hj] = lo;
+            }
           }
         }
       }
@@ -491,7 +561,7 @@ __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
       y[g] = v + part[((a.ks + jj) * 4 + g) * gs] + bias[g];
     }
     float hh, cc;
-    lstm_cell_hw(y[0], y[1], y[2], y[3], cp, hh, cc);
+    lstm_cell_f(y[0], y[1], y[2], y[3], cp, hh, cc);
     const long long o = (long long)jj * a.ck_stride + i;
     if (a.ckpt_h) a.ckpt_h[o] = hh;
     if (a.ckpt_c) a.ckpt_c[o] = cc;
@@ -504,20 +574,27 @@ __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
     y[g] = v + bias[g];
   }
   float hh, cc;
-  lstm_cell_hw(y[0], y[1], y[2], y[3], cp, hh, cc);
+  lstm_cell_f(y[0], y[1], y[2], y[3], cp, hh, cc);
   a.c_state[i] = cc;
   if (a.out_h) a.out_h[i] = hh;
-  const __nv_bfloat16 hb = __float2bfloat16_rn(hh);
-  a.h_bf16[(long long)n * a.ldh + j] = hb;
-  if (a.seq_bf16) a.seq_bf16[(long long)n * a.ldh + j] = hb;
+  __nv_bfloat16 hi, lo;
+  bf16_pair(hh, hi, lo);
+  const long long hj = (long long)n * a.ldh + j;
+  a.h_bf16[hj] = hi;
+  a.h_bf16[a.h_plane + hj] = lo;
+  if (a.seq_bf16) {
+    a.seq_bf16[hj] = hi;
+    a.seq_bf16[a.seq_plane + hj] = lo;
+  }
 }
 
-// x (fp32 [N][D]) -> bf16 [N][ld] with zero columns D..ld-1: one thread per
-// 8 output elements (one 16-byte store), vector loads when D is a multiple of 8
-__global__ void to_bf16_kernel(const float* __restrict__ x, int N, int D, __nv_bfloat16* __restrict__ out, int ld) {
+// x (fp32 [N][D]) -> its bf16 pair, hi plane [N][ld] then lo plane [N][ld],
+// with zero columns D..ld-1: one thread per 8 elements (one 16-byte store
+// per plane), vector loads when x is 16-byte aligned and D is a multiple of 8
+__global__ void to_bf16_kernel(const float* __restrict__ x, int N, int D, __nv_bfloat16* __restrict__ out, int ld,
+                               bool vec) {
   const int c8 = ld >> 3;  // 8-element chunks per output row (ld is a multiple of 8)
   const long long total = (long long)N * c8;
-  const bool vec = (D & 7) == 0;
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
        i += (long long)gridDim.x * blockDim.x) {
     const int n = (int)(i / c8), d0 = (int)(i % c8) * 8;
@@ -530,18 +607,22 @@ __global__ void to_bf16_kernel(const float* __restrict__ x, int N, int D, __nv_b
 #pragma unroll
       for (int e = 0; e < 8; ++e) v[e] = d0 + e < D ? __ldg(x + (long long)n * D + d0 + e) : 0.f;
     }
-    uint4 o;
-    __nv_bfloat162 p0 = __floats2bfloat162_rn(v[0], v[1]), p1 = __floats2bfloat162_rn(v[2], v[3]),
-                    p2 = __floats2bfloat162_rn(v[4], v[5]), p3 = __floats2bfloat162_rn(v[6], v[7]);
-    o.x = *reinterpret_cast<uint32_t*>(&p0);
-    o.y = *reinterpret_cast<uint32_t*>(&p1);
-    o.z = *reinterpret_cast<uint32_t*>(&p2);
-    o.w = *reinterpret_cast<uint32_t*>(&p3);
-    reinterpret_cast<uint4*>(out)[i] = o;
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      __nv_bfloat16 h0, l0, h1, l1;
+      bf16_pair(v[2 * e], h0, l0);
+      bf16_pair(v[2 * e + 1], h1, l1);
+      hw[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+      lw[e] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+    }
+    reinterpret_cast<uint4*>(out)[i] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    reinterpret_cast<uint4*>(out)[total + i] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
 }
 
-// initial state of the tensor path: h0 -> bf16 operand, c0 -> fp32 state
+// initial state of the tensor path: h0 -> the bf16 pair planes of the
+// operand ([B][ldh] each), c0 -> fp32 state
 __global__ void tc_init_state_kernel(const float* __restrict__ h0, const float* __restrict__ c0, int B, int H,
                                      __nv_bfloat16* __restrict__ h_bf16, int ldh, float* __restrict__ c_state) {
   const long long total = (long long)B * ldh;
@@ -549,7 +630,10 @@ __global__ void tc_init_state_kernel(const float* __restrict__ h0, const float* 
        i += (long long)gridDim.x * blockDim.x) {
     const long long n = i / ldh;
     const int j = (int)(i % ldh);
-    h_bf16[i] = __float2bfloat16_rn((h0 != nullptr && j < H) ? h0[n * H + j] : 0.f);
+    __nv_bfloat16 hi, lo;
+    bf16_pair((h0 != nullptr && j < H) ? h0[n * H + j] : 0.f, hi, lo);
+    h_bf16[i] = hi;
+    h_bf16[total + i] = lo;
     if (j < H) c_state[n * H + j] = c0 != nullptr ? c0[n * H + j] : 0.f;
   }
 }
@@ -598,11 +682,11 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args..
 
 template <int BN, int S>
 size_t rows_smem() {
-  return 1024 + S * (kABytes + BN * kTileK * 2) + 8 * (2 * S + 3) + 16;
+  return 1024 + S * (kABytes + 2 * BN * kTileK * 2) + 8 * (2 * S + 2) + 16;
 }
 template <int NT, int S>
 size_t gates_smem() {
-  return 1024 + S * (kABytes + NT * kTileK * 2) + 8 * (2 * S + 4) + 16;
+  return 1024 + S * (kABytes + 2 * NT * kTileK * 2) + 8 * (2 * S + 4) + 16;
 }
 
 template <int BN, int S>
@@ -657,11 +741,11 @@ bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint
 }
 
 int tc_rows_tile_n(int n_cols, int row_tiles) {
-  // few columns (tau' over B streams): the widest tile that keeps one wave;
-  // many columns (the projection over T*B): 256
-  for (int bn : {64, 128, 256})
-    if ((long long)row_tiles * ((n_cols + bn - 1) / bn) <= 148) return bn;
-  return 256;
+  // few columns (tau' over B streams): 64 when that keeps one wave; else 128
+  // (with both planes of the activation a 128-column tile feeds 256 columns
+  // of MMA work per factor tile)
+  if ((long long)row_tiles * ((n_cols + 63) / 64) <= 148) return 64;
+  return 128;
 }
 int tc_gates_splits(int tiles, int nkb, int* nkb_per) {
   // about one wave: as many splits as the GPU holds grids of `tiles` CTAs
@@ -685,16 +769,15 @@ int tc_gates_tile_n(int H, int B) {
 
 cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s) {
   switch (bn) {
-    case 256: return launch_rows_t<256, 4>(A, Bm, a, n_cols, s);
-    case 128: return launch_rows_t<128, 6>(A, Bm, a, n_cols, s);
-    default: return launch_rows_t<64, 8>(A, Bm, a, n_cols, s);
+    case 128: return launch_rows_t<128, 4>(A, Bm, a, n_cols, s);
+    default: return launch_rows_t<64, 6>(A, Bm, a, n_cols, s);
   }
 }
 
 cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s) {
   switch (nt) {
-    case 128: return a.ks > 1 ? launch_gates_t<128, 6, true>(U, Tau, a, s) : launch_gates_t<128, 6, false>(U, Tau, a, s);
-    case 64: return a.ks > 1 ? launch_gates_t<64, 8, true>(U, Tau, a, s) : launch_gates_t<64, 8, false>(U, Tau, a, s);
+    case 128: return a.ks > 1 ? launch_gates_t<128, 4, true>(U, Tau, a, s) : launch_gates_t<128, 4, false>(U, Tau, a, s);
+    case 64: return a.ks > 1 ? launch_gates_t<64, 6, true>(U, Tau, a, s) : launch_gates_t<64, 6, false>(U, Tau, a, s);
     default: return a.ks > 1 ? launch_gates_t<32, 8, true>(U, Tau, a, s) : launch_gates_t<32, 8, false>(U, Tau, a, s);
   }
 }
@@ -702,7 +785,8 @@ cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs&
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s) {
   const long long total = (long long)N * (ld >> 3);
   const int blocks = (int)std::min<long long>((total + 255) / 256, 152LL * 16);
-  to_bf16_kernel<<<blocks, 256, 0, s>>>(x, N, D, out, ld);
+  const bool vec = (D & 7) == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  to_bf16_kernel<<<blocks, 256, 0, s>>>(x, N, D, out, ld, vec);
   return cudaGetLastError();
 }
 

@@ -427,12 +427,13 @@ cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const floa
   return cudaErrorInvalidValue;
 }
 
-bool xproj_cluster_fits(int N, int D, int lda, int ldxin, bool a_bf16) {
-  // bulk copies need 16-byte aligned rows and lengths
+bool xproj_cluster_fits(int N, int D, const void* A, int lda, const float* X, int ldxin, bool a_bf16) {
+  // 16-byte asynchronous copies need 16-byte aligned base pointers, rows and lengths
   const int a_align = a_bf16 ? 8 : 4;
+  const bool bases_aligned = ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(X)) & 15u) == 0;
   // up to 8 chunks of 32 columns: beyond that every chunk re-reading the
   // CTA's rows costs more than a tiled GEMM
-  return N >= 1 && N <= 8 * kCols && D % 8 == 0 && lda % a_align == 0 && ldxin % 4 == 0;
+  return N >= 1 && N <= 8 * kCols && D % 8 == 0 && lda % a_align == 0 && ldxin % 4 == 0 && bases_aligned;
 }
 
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,

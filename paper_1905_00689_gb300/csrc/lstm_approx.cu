@@ -38,12 +38,14 @@ int cuda_fail(lstm_approx_t* h, cudaError_t e, const char* what) {
 
 inline int round_up(int v, int m) { return (v + m - 1) / m * m; }
 
-// fp64 -> fp32 -> bf16, both steps round-to-nearest-even.
+// fp64 -> fp32 -> bf16, both steps round-to-nearest-even; infinities keep
+// their sign, every NaN becomes the quiet NaN 0x7FC0.
 inline uint16_t to_bf16_bits(double x) {
   const float f = static_cast<float>(x);
   uint32_t u;
   std::memcpy(&u, &f, 4);
-  if ((u & 0x7F800000u) == 0x7F800000u) return static_cast<uint16_t>(u >> 16);  // inf / nan
+  if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0x7FC0u;                            // nan
+  if ((u & 0x7FFFFFFFu) == 0x7F800000u) return static_cast<uint16_t>(u >> 16);  // inf
   const uint32_t lsb = (u >> 16) & 1u;
   u += 0x7FFFu + lsb;
   return static_cast<uint16_t>(u >> 16);
@@ -90,8 +92,9 @@ size_t layer_bytes_vx(const lstm_approx_t* h, const LayerStore& s) {
 size_t layer_bytes_vh(const lstm_approx_t* h) { return 4ull * h->Ks * h->ldh * elem_size(h->dtype); }
 size_t layer_bytes_u(const lstm_approx_t* h) { return 4ull * h->Ks * h->H * elem_size(h->dtype); }
 
-size_t xbf16_bytes(const lstm_approx_t* h, size_t TB) { return TB * (size_t)h->layers[0].ldx * 2; }
-size_t seqbf16_bytes(const lstm_approx_t* h, size_t TB) { return TB * (size_t)h->ldh * 2; }
+// bf16 pair planes (hi, lo) of the tensor path's activations
+size_t xbf16_bytes(const lstm_approx_t* h, size_t TB) { return 2 * TB * (size_t)h->layers[0].ldx * 2; }
+size_t seqbf16_bytes(const lstm_approx_t* h, size_t TB) { return 2 * TB * (size_t)h->ldh * 2; }
 
 void free_scratch(lstm_approx_t* h) {
   dfree(h, h->Px, h->cap_TB * 4ull * h->Ks * sizeof(float));
@@ -189,17 +192,12 @@ bool sparse_x_projection(const lstm_approx_t* h, const LayerStore& s, int K, int
   return h->opt_xproj == 2 || kept * 8 <= 4LL * K * s.D;
 }
 
-// The tensor path takes bf16 factors; its intermediate depths must fall on
-// the 16-term slices of one MMA instruction.
-bool tensor_path_fits(int dtype, const Checkpoints& ck) {
-  if (dtype != LSTM_APPROX_BF16) return false;
-  for (int j = 0; j < ck.n; ++j)
-    if (ck.k[j] % 16 != 0) return false;
-  return true;
-}
+// The tensor path takes bf16 factors at any depths (a depth off the MMA's
+// 16-term slices adds its last terms on the CUDA cores).
+bool tensor_path_fits(int dtype) { return dtype == LSTM_APPROX_BF16; }
 
 // Recurrence path of one layer.  Automatic: bf16 factors take the
-// tensor-core path when the depths allow it; fp32 factors take a persistent
+// tensor-core path; fp32 factors take a persistent
 // launch whenever a plan fits, at any batch (one cluster per stream;
 // clusters beyond one wave run in the next); everything else takes the
 // CUDA-core kernels.  A forced path that cannot take the shape returns 0
@@ -207,7 +205,7 @@ bool tensor_path_fits(int dtype, const Checkpoints& ck) {
 int select_path(int dtype, int H, int K, int T, const Checkpoints& ck, int force_path, int want_cs, int sm_count,
                 int variant, PersistentChoice* plan, std::string* why) {
   const bool bf16 = dtype == LSTM_APPROX_BF16;
-  const bool tensor_ok = tensor_path_fits(dtype, ck);
+  const bool tensor_ok = tensor_path_fits(dtype);
   if (force_path == 0) {
     if (tensor_ok) return LSTM_APPROX_PATH_TENSOR;
     if (!bf16 && choose_persistent(H, K, T, ck, want_cs, sm_count, variant, plan, why))
@@ -225,7 +223,7 @@ int select_path(int dtype, int H, int K, int T, const Checkpoints& ck, int force
       return 0;
     }
   } else if (force_path == LSTM_APPROX_PATH_TENSOR && !tensor_ok) {
-    *why = "tensor path needs bf16 factors and intermediate depths that are multiples of 16";
+    *why = "tensor path needs bf16 factors";
     return 0;
   }
   return force_path;
@@ -289,7 +287,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     const int kt = (K + 127) / 128;
     const int bnx = tc_rows_tile_n(TB, 4 * kt);
     TcMap mx;
-    if (!tc_make_map(&mx, in_bf16, D, TB, (uint64_t)ld_in * 2, bnx))
+    if (!tc_make_map(&mx, in_bf16, D, 2ull * TB, (uint64_t)ld_in * 2, bnx))
       return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
     TcRowsArgs ra{};
     ra.Kdim = D;
@@ -297,6 +295,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.Ks = h->Ks;
     ra.kt_per_gate = (K + 127) / 128;
     ra.N = TB;
+    ra.b_plane = TB;
     ra.mode = 0;
     ra.P = h->Px;
     ra.ldp = (int)ldp;
@@ -326,8 +325,8 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     }
   }
   TcMap mh, mt;
-  if (!tc_make_map(&mh, hb, H, B, (uint64_t)h->ldh * 2, bnh) ||
-      !tc_make_map(&mt, tau, ldp, B, (uint64_t)ldp * 2, nt))
+  if (!tc_make_map(&mh, hb, H, 2ull * B, (uint64_t)h->ldh * 2, bnh) ||
+      !tc_make_map(&mt, tau, ldp, 2ull * B, (uint64_t)ldp * 2, nt))
     return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the state");
   for (int t = 0; t < T; ++t) {
     TcRowsArgs ra{};
@@ -336,12 +335,14 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.Ks = h->Ks;
     ra.kt_per_gate = (K + 127) / 128;
     ra.N = B;
+    ra.b_plane = B;
     ra.mode = 1;
     ra.P = h->Px + (size_t)t * B * ldp;
     ra.ldp = (int)ldp;
     ra.sigma = s.sigma;
     ra.tau = tau;
     ra.ldt = (int)ldp;
+    ra.tau_plane = (long long)B * ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
     LA_CUDA(h, launch_tc_rows(s.map_vh, mh, ra, B, bnh, h->stream), "recurrent projection launch");
@@ -351,12 +352,19 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ga.Ks = h->Ks;
     ga.B = B;
     ga.nkb = (K + 63) / 64;
+    ga.tau_rows = B;
+    ga.U = static_cast<const __nv_bfloat16*>(s.U);
+    ga.tau = tau;
+    ga.ldt = (int)ldp;
+    ga.tau_plane = (long long)B * ldp;
     ga.bias = s.bias;
     ga.c_state = cs;
     ga.h_bf16 = hb;
     ga.ldh = h->ldh;
+    ga.h_plane = (long long)B * h->ldh;
     ga.out_h = out_h ? out_h + (size_t)t * B * H : nullptr;
     ga.seq_bf16 = top ? nullptr : static_cast<__nv_bfloat16*>(h->seq_bf16) + (size_t)t * B * h->ldh;
+    ga.seq_plane = (long long)TB * h->ldh;
     ga.ck = ck;
     ga.ckpt_h = ckpt_h ? ckpt_h + (size_t)t * B * H : nullptr;
     ga.ckpt_c = ckpt_c ? ckpt_c + (size_t)t * B * H : nullptr;
@@ -389,6 +397,17 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     cudaEventRecord(h->timing.run0, h->stream);
   }
   const long long ldp = 4LL * h->Ks;
+  // A bf16 run takes one path for all its layers, the one its top layer (the
+  // only one with intermediate depths) takes: the tensor-core path hands the
+  // sequence to the next layer in bf16, the CUDA-core kernels in fp32.
+  int run_path = 0;
+  if (bf16) {
+    PersistentChoice unused;
+    std::string why;
+    run_path = select_path(h->dtype, H, K, T, ck, h->opt_force_path, h->opt_cluster, h->sm_count,
+                           h->opt_persistent_variant, &unused, &why);
+    if (run_path == 0) return fail(h, LSTM_APPROX_EINVAL, "%s", why.c_str());
+  }
   for (int l = 0; l < h->L; ++l) {
     const LayerStore& s = h->layers[l];
     const bool top = l == h->L - 1;
@@ -399,8 +418,9 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // recurrence path
     PersistentChoice plan;
     std::string why;
-    const int path = select_path(h->dtype, H, K, T, lck, h->opt_force_path, h->opt_cluster, h->sm_count,
-                                 h->opt_persistent_variant, &plan, &why);
+    const int path = bf16 ? run_path
+                          : select_path(h->dtype, H, K, T, lck, h->opt_force_path, h->opt_cluster, h->sm_count,
+                                        h->opt_persistent_variant, &plan, &why);
     if (path == 0) return fail(h, LSTM_APPROX_EINVAL, "%s", why.c_str());
     const float* l_h0 = h0 ? h0 + (size_t)l * B * H : nullptr;
     const float* l_c0 = c0 ? c0 + (size_t)l * B * H : nullptr;
@@ -433,7 +453,7 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
         }
         LA_CUDA(h, launch_xproj_sparse(sr, K, h->Ks, in, s.D, T * B, h->Px, (int)ldp, h->stream),
                 "input projection launch");
-      } else if (xproj_cluster_fits(T * B, s.D, s.ldx, s.D, bf16))
+      } else if (xproj_cluster_fits(T * B, s.D, s.Vx, s.ldx, in, s.D, bf16))
         LA_CUDA(h,
                 launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->err,
                                      h->opt_wait_limit_us * 1000LL, h->stream, xproj_max_split),
@@ -591,7 +611,7 @@ int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dim
   if (!rc && cudaHostAlloc(reinterpret_cast<void**>(&h->err_host), sizeof(int), cudaHostAllocDefault) != cudaSuccess)
     rc = fail(h, LSTM_APPROX_ENOMEM, "pinned status word");
   if (!rc && dtype == LSTM_APPROX_BF16)
-    rc = dmalloc(h, &h->h_bf16, (size_t)max_batch * h->ldh * 2, "bf16 state");
+    rc = dmalloc(h, &h->h_bf16, 2 * (size_t)max_batch * h->ldh * 2, "bf16 state pair");
   if (rc) {
     lstm_approx_destroy(h);
     return rc;
@@ -816,6 +836,48 @@ int lstm_approx_get_mask(lstm_approx_t* h, int layer, int gate, int k, int32_t* 
   for (int c = 0; c < s.C; ++c)
     if (words[c / 32] >> (c % 32) & 1u) idx_out[n++] = c;
   *nz_out = n;
+  return LSTM_APPROX_OK;
+}
+
+int lstm_approx_get_term(lstm_approx_t* h, int layer, int gate, int k, float* sigma_out, float* u_out,
+                         float* v_out) {
+  if (!h) return LSTM_APPROX_EINVAL;
+  if (layer < 0 || layer >= h->L || gate < 0 || gate > 3 || !sigma_out || !u_out || !v_out)
+    return fail(h, LSTM_APPROX_EINVAL, "bad layer/gate/pointer");
+  const LayerStore& s = h->layers[layer];
+  if (k < 0 || k >= s.Kset[gate]) return fail(h, LSTM_APPROX_EINVAL, "term %d not set", k);
+  DeviceGuard dg(h->device);
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "stream synchronise");
+  const int H = h->H, D = s.D, Ks = h->Ks;
+  const bool bf16 = h->dtype == LSTM_APPROX_BF16;
+  const size_t es = elem_size(h->dtype);
+  const size_t row = (size_t)gate * Ks + k;
+  std::vector<unsigned char> vx((size_t)D * es), vh((size_t)H * es), uu((size_t)H * es);
+  LA_CUDA(h, cudaMemcpy(vx.data(), static_cast<const char*>(s.Vx) + row * s.ldx * es, vx.size(), cudaMemcpyDeviceToHost),
+          "factor read");
+  LA_CUDA(h, cudaMemcpy(vh.data(), static_cast<const char*>(s.Vh) + row * h->ldh * es, vh.size(), cudaMemcpyDeviceToHost),
+          "factor read");
+  // u_k[j] sits at (gate*H + j)*Ks + k: one strided column of U
+  LA_CUDA(h,
+          cudaMemcpy2D(uu.data(), es, static_cast<const char*>(s.U) + ((size_t)gate * H * Ks + k) * es, Ks * es, es, H,
+                       cudaMemcpyDeviceToHost),
+          "factor read");
+  LA_CUDA(h, cudaMemcpy(sigma_out, s.sigma + row, sizeof(float), cudaMemcpyDeviceToHost), "factor read");
+  auto widen = [&](const std::vector<unsigned char>& buf, size_t i) {
+    float f;
+    if (bf16) {
+      uint16_t b;
+      std::memcpy(&b, buf.data() + 2 * i, 2);
+      const uint32_t u = static_cast<uint32_t>(b) << 16;
+      std::memcpy(&f, &u, 4);
+    } else {
+      std::memcpy(&f, buf.data() + 4 * i, 4);
+    }
+    return f;
+  };
+  for (int j = 0; j < H; ++j) u_out[j] = widen(uu, j);
+  for (int c = 0; c < D; ++c) v_out[c] = widen(vx, c);
+  for (int c = 0; c < H; ++c) v_out[D + c] = widen(vh, c);
   return LSTM_APPROX_OK;
 }
 

@@ -179,24 +179,6 @@ __device__ __forceinline__ float tanh_f(float z) {
   return a < 0.25f ? small : big;
 }
 
-// Hardware tanh (tanh.approx: absolute error below 1e-3), for the bf16
-// path, whose operands are rounded to 2^-9 anyway.
-__device__ __forceinline__ float tanh_hw(float x) {
-  float r;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
-  return r;
-}
-
-// The cell update below with sigmoid z = (1 + tanh(z/2)) / 2 and tanh from
-// tanh_hw: five hardware operations per cell instead of ten.
-__device__ __forceinline__ void lstm_cell_hw(float yi, float yf, float yg, float yo, float c_prev, float& h_out,
-                                             float& c_out) {
-  const float i = fmaf(0.5f, tanh_hw(0.5f * yi), 0.5f), f = fmaf(0.5f, tanh_hw(0.5f * yf), 0.5f);
-  const float o = fmaf(0.5f, tanh_hw(0.5f * yo), 0.5f), g = tanh_hw(yg);
-  c_out = fmaf(f, c_prev, i * g);
-  h_out = o * tanh_hw(c_out);
-}
-
 // Gate nonlinearities and cell update (Sec. II): i, f, o sigmoid, g tanh;
 // c = f c_prev + i g; h = o tanh(c).  Pre-activations already include bias.
 __device__ __forceinline__ void lstm_cell_f(float yi, float yf, float yg, float yo, float c_prev,

@@ -123,7 +123,7 @@ extern "C" int lstm_approx_run_static(const float* Vx, const float* Vh, const fl
   e = cudaMemsetAsync(base, 0, (kHeaderFloats + (bias ? 0 : bias_floats)) * sizeof(float), s);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "clearing scratch: %s", cudaGetErrorString(e));
   // (a1) hoisted input projection into the static scratch
-  e = xproj_cluster_fits(T * B, D, D, D, false)
+  e = xproj_cluster_fits(T * B, D, Vx, D, x, D, false)
           ? launch_xproj_cluster(Vx, false, D, K, K, x, D, T * B, D, P, 4 * K, status, 2000000000LL, s, 8)
           : launch_rows_gemm(Vx, false, D, K, K, x, D, T * B, D, P, 4 * K, 0, nullptr, nullptr, 0, s);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "projection launch: %s", cudaGetErrorString(e));

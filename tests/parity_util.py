@@ -14,14 +14,9 @@ BF16_TOL = 2e-2   # max relative error, bf16 factors / fp32 accumulate
 
 
 def max_rel_err_vec(got, ref) -> float:
-    """Normwise relative error of every output vector (last axis: the H units).
-
-    max over vectors of max_j |got_j - ref_j| / max_j |ref_j|.  Used for the
-    bf16 operand path: rounding x, h and tau' to bf16 (unit roundoff 2^-9)
-    gives every pre-activation an absolute error of a few 2^-9 at the scale of
-    its vector, so the error is bounded relative to the vector, not to each
-    element (elements near zero would need an absolute bound).
-    """
+    """Normwise relative error of every output vector (last axis: the H units):
+    max over vectors of max_j |got_j - ref_j| / max_j |ref_j|.  Reported
+    beside the elementwise error; no bound is asserted on it."""
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     assert got.shape == ref.shape, (got.shape, ref.shape)
@@ -103,18 +98,24 @@ def oracle_run(layers, x, K, dtype="fp32", **kw):
     return oracle.run_lstm(rl, xr, K, **kw)
 
 
-def assert_parity(got, ref, tol, keys=("h", "c_last", "ckpt_h", "ckpt_c"), metric=None):
-    """Every output within `tol`: elementwise (max_rel_err) for the fp32 bound,
-    normwise per output vector (max_rel_err_vec) for the bf16 bound."""
-    if metric is None:
-        metric = max_rel_err_vec if tol == BF16_TOL else max_rel_err
+# (test id, bound, {output: (elementwise, normwise)}) of every parity check of
+# the session, printed by the terminal-summary hook in conftest.py
+REPORT = []
+CURRENT_TEST = [""]
+
+
+def assert_parity(got, ref, tol, keys=("h", "c_last", "ckpt_h", "ckpt_c")):
+    """Every output within `tol` under the elementwise metric (max_rel_err),
+    for both factor types.  Returns {key: (elementwise, normwise)} errors;
+    the normwise figure is a report only."""
     errs = {}
     for k in keys:
         if k in got and k in ref:
             assert np.all(np.isfinite(got[k])), f"{k}: non-finite output"
-            errs[k] = metric(got[k], ref[k])
-    bad = {k: v for k, v in errs.items() if v > tol}
-    assert not bad, f"max relative error above {tol}: {errs}"
+            errs[k] = (max_rel_err(got[k], ref[k]), max_rel_err_vec(got[k], ref[k]))
+    REPORT.append((CURRENT_TEST[0], tol, errs))
+    bad = {k: v for k, v in errs.items() if v[0] > tol}
+    assert not bad, f"max relative error (elementwise, normwise) above {tol}: {errs}"
     return errs
 
 

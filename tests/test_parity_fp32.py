@@ -221,3 +221,27 @@ def test_host_entry_pinned_and_pageable_buffers(cuda_device, pinned):
     assert np.array_equal(oc.numpy().astype(np.float64), got["c_last"])
     assert np.array_equal(kh.numpy().astype(np.float64), got["ckpt_h"])
     assert np.array_equal(kc.numpy().astype(np.float64), got["ckpt_c"])
+
+
+@pytest.mark.parametrize("dtype,B", [("fp32", 1), ("fp32", 3), ("bf16", 5)])
+def test_input_view_not_16_byte_aligned(cuda_device, dtype, B):
+    """x passed as a view 4 bytes into its allocation: the kernels that copy
+    x in 16-byte pieces are not taken (the result equals the oracle's)."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox
+    D, H, T, K = 64, 64, 5, 16
+    gates = [draw_factor_set(H, D + H, K, 60, 6800 + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 12).astype(np.float32)
+    dev = torch.device("cuda:0")
+    buf = torch.zeros(T * B * D + 4, device=dev)
+    xv = buf[1:1 + T * B * D].view(T, B, D)
+    assert xv.data_ptr() % 16 == 4
+    xv.copy_(torch.from_numpy(x))
+    m = LSTMApprox(1, [D], H, K, B, dtype)
+    m.set_layer(0, gates)
+    out = torch.full((T, B, H), float("nan"), device=dev)
+    m.run(xv, K, out)
+    m.sync()
+    ref = oracle_run([gates], x, K, dtype=dtype)
+    assert_parity({"h": out.double().cpu().numpy()}, ref, FP32_TOL if dtype == "fp32" else 2e-2, keys=("h",))
+    m.close()

@@ -1,9 +1,10 @@
-"""GPU parity of the tensor-core path (bf16 factors and operands, fp32 accumulate).
+"""GPU parity of the tensor-core path (bf16 factors, fp32 accumulate).
 
 The oracle receives the factors as the library stores them (sigma fp32,
-u and v bf16); the bound 2e-2 covers the kernels' bf16 operand rounding of
-x, h and tau'.  Full-size workloads are checked on sampled streams (streams
-are independent, so the oracle runs on those streams alone).
+u and v bf16); the activations x, h and tau' enter the MMAs as bf16 pairs
+(hi + lo), so the elementwise bound 2e-2 holds with a wide margin (the
+errors are a few 1e-4).  Full-size workloads are checked on sampled streams
+(streams are independent, so the oracle runs on those streams alone).
 """
 import numpy as np
 import pytest
@@ -34,6 +35,12 @@ def _sample(got, streams, T=None):
     # split boundaries, inside splits and at K
     (48, 128, 3, 8, 256, 100, [64, 96, 128, 192, 256]),
     (32, 128, 2, 4, 512, 60, [16, 320, 512]),
+    # depths off the 16-term slices: below the first slice, inside a slice,
+    # at the start of a split's range (no MMA issued before the cut), and
+    # at K when K is not a multiple of 16
+    (40, 200, 4, 3, 80, 70, [5, 21, 79]),
+    (48, 128, 3, 8, 256, 100, [5, 67, 130, 200, 256]),
+    (64, 136, 2, 40, 45, 80, [1, 17, 45]),
 ])
 def test_tensor_path_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     gates = [draw_factor_set(H, D + H, K, nz, 5100 + 7 * D + g) for g in range(4)]
@@ -72,7 +79,7 @@ def test_throughput_workload_full_size(cuda_device, K):
     assert_parity(_sample(got, streams), ref, BF16_TOL)
 
 
-@pytest.mark.parametrize("K,cps", [(8, []), (24, [16]), (40, [16, 32])])
+@pytest.mark.parametrize("K,cps", [(8, []), (24, [16]), (40, [16, 32]), (40, [3, 33, 40])])
 def test_prefix_of_stored_terms(cuda_device, K, cps):
     """Runs at K below the stored rank, with K not a multiple of the MMA's 16
     terms: the terms past K in the last slice must contribute nothing."""
@@ -130,3 +137,31 @@ def test_two_layer_progressive_workload_full_size(cuda_device):
     streams = [5, 63]
     ref = oracle_run(layers, x[:, streams], 1024, dtype="bf16", checkpoints=cps)
     assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+def test_two_layer_unaligned_depths_automatic_path(cuda_device):
+    """Two bf16 layers, no forced path, a depth off the 16-term slices: every
+    layer takes the tensor path (the sequence between layers stays in the
+    tensor path's bf16 pair planes)."""
+    from paper_1905_00689_gb300 import BF16, plan
+    D, H, T, B, K = 72, 96, 4, 12, 48
+    layers = [[draw_factor_set(H, (D if l == 0 else H) + H, K, int(0.4 * ((D if l == 0 else H) + H)),
+                               6600 + 10 * l + g) for g in range(4)] for l in range(2)]
+    x = draw_inputs(T, B, D, "uniform", 9)
+    cps = [5, K]
+    got, m = run_gpu(layers, x, K, dtype="bf16", checkpoints=cps)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR == plan(BF16, H, T, B, K, cps)["path"]
+    ref = oracle_run(layers, x, K, dtype="bf16", checkpoints=cps)
+    assert_parity(got, ref, BF16_TOL)
+
+
+def test_two_layer_simt_forced_unaligned_depths(cuda_device):
+    """The same stack forced onto the CUDA-core kernels for every layer."""
+    D, H, T, B, K = 72, 96, 4, 12, 48
+    layers = [[draw_factor_set(H, (D if l == 0 else H) + H, K, int(0.4 * ((D if l == 0 else H) + H)),
+                               6600 + 10 * l + g) for g in range(4)] for l in range(2)]
+    x = draw_inputs(T, B, D, "uniform", 9)
+    got, m = run_gpu(layers, x, K, dtype="bf16", checkpoints=[5, K], force_path=PATH_SIMT)
+    assert m.query(Q_LAST_PATH) == PATH_SIMT
+    ref = oracle_run(layers, x, K, dtype="bf16", checkpoints=[5, K])
+    assert_parity(got, ref, BF16_TOL)

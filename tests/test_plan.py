@@ -134,15 +134,16 @@ def test_every_plan_covers_its_shape_and_fits(H, K, cs, variant):
                                  (2048, 2048), (136, 130)])
 @pytest.mark.parametrize("K", [8, 64, 256, 1024])
 def test_tensor_tiles(H, B, K):
-    """Stream tiles: the narrowest of 32/64/128 (gates) and 64/128/256 (tau')
-    that keeps the grid within one wave of 148 CTAs, else the widest; the
-    gate GEMM's terms split over min(148 // tiles, 8, chunks of 64) CTAs."""
+    """Stream tiles: the narrowest of 32/64/128 (gates) that keeps the grid
+    within one wave of 148 CTAs, else the widest; tau' takes 64 streams when
+    that keeps one wave, else 128; the gate GEMM's terms split over
+    min(148 // tiles, 8, chunks of 64) CTAs."""
     p = plan(BF16, H, 2, B, K)
     units = -(-H // 128)
     nt = next((n for n in (32, 64, 128) if units * -(-B // n) <= 148), 128)
     assert p["gate_tile_streams"] == nt
     rows = 4 * -(-K // 128)
-    bn = next((n for n in (64, 128, 256) if rows * -(-B // n) <= 148), 256)
+    bn = 64 if rows * -(-B // 64) <= 148 else 128
     assert p["tau_tile_streams"] == bn
     tiles = units * -(-B // nt)
     chunks = -(-K // 64)
@@ -156,7 +157,8 @@ def test_tensor_tiles(H, B, K):
 
 def test_paths():
     assert plan(BF16, 64, 2, 4, 32, [16])["path"] == PATH_TENSOR
-    assert plan(BF16, 64, 2, 4, 32, [10])["path"] == PATH_SIMT       # a depth off the 16-term slices
+    assert plan(BF16, 64, 2, 4, 32, [10])["path"] == PATH_TENSOR     # a depth off the 16-term slices
+    assert plan(BF16, 64, 2, 4, 32, [10], PATH_SIMT)["path"] == PATH_SIMT
     assert plan(FP32, 2048, 2, 1, 32)["path"] == PATH_SIMT           # no persistent kernel for H > 1024
     assert plan(FP32, 64, 2, 1, 300)["path"] == PATH_SIMT            # nor for K > 256
     assert plan(FP32, 64, 2, 4096, 32)["path"] == PATH_PERSISTENT    # at any batch
@@ -166,7 +168,6 @@ def test_paths():
 
 @pytest.mark.parametrize("args,text", [
     ((BF16, 64, 2, 1, 32, (), PATH_PERSISTENT), "fp32 factors only"),
-    ((BF16, 64, 2, 1, 32, [8], PATH_TENSOR), "multiples of 16"),
     ((FP32, 64, 2, 1, 32, (), PATH_TENSOR), "bf16"),
     ((FP32, 64, 2, 1, 300, (), PATH_PERSISTENT), "persistent path unavailable"),
     ((FP32, 600, 2, 1, 32, (), PATH_PERSISTENT, 0, 2), "persistent path unavailable"),

@@ -142,21 +142,36 @@ def synthetic_layer_factors(w: Workload, layer: int, K: int, keep: float) -> Lis
     return [draw_factor_set(w.H, C, K, nz, weight_seed(w, layer, g) + 50_000) for g in range(4)]
 
 
-def round_bf16(a: np.ndarray) -> np.ndarray:
-    """Round to bfloat16 (through float32, both steps round-to-nearest-even).
+def bf16_bits(a: np.ndarray) -> np.ndarray:
+    """bfloat16 bit patterns of `a` rounded through float32 (both steps
+    round-to-nearest-even, ties to the even pattern).
 
-    Returns float64 values that are exactly representable in bfloat16.  This
-    is the storage rounding of the bf16 factor path, written out from the
-    IEEE/bfloat16 definitions so that the oracle can be fed the same values.
+    Written from the formats' definitions: bfloat16 is the upper half of an
+    IEEE binary32, so rounding adds 0x7FFF plus the lowest kept bit and
+    drops the low 16 bits; a carry out of the mantissa moves to the next
+    binade (and past the largest finite value, to infinity).  Infinities
+    keep their sign; every NaN becomes the quiet NaN 0x7FC0.
     """
     f = np.ascontiguousarray(np.asarray(a, dtype=np.float64).astype(np.float32))
     bits = f.view(np.uint32).astype(np.uint64)
     lsb = (bits >> 16) & 1
-    rounded = ((bits + 0x7FFF + lsb) >> 16) << 16
-    # keep NaN/Inf payloads as they are (none occur in these workloads)
-    special = (bits & 0x7F800000) == 0x7F800000
-    rounded = np.where(special, bits & 0xFFFF0000, rounded)
-    return rounded.astype(np.uint32).view(np.float32).astype(np.float64)
+    rounded = (bits + 0x7FFF + lsb) >> 16
+    nan = (bits & 0x7FFFFFFF) > 0x7F800000
+    inf = (bits & 0x7FFFFFFF) == 0x7F800000
+    out = np.where(inf, bits >> 16, rounded)
+    out = np.where(nan, 0x7FC0, out)
+    return out.astype(np.uint16)
+
+
+def round_bf16(a: np.ndarray) -> np.ndarray:
+    """Round to bfloat16 (through float32, both steps round-to-nearest-even).
+
+    Returns float64 values that are exactly representable in bfloat16: the
+    storage rounding of the bf16 factor path, so that the oracle can be fed
+    the values the library stores.
+    """
+    bits = bf16_bits(a).astype(np.uint32) << 16
+    return bits.view(np.float32).astype(np.float64)
 
 
 def round_fp32(a: np.ndarray) -> np.ndarray:
