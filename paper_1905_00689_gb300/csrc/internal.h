@@ -254,9 +254,9 @@ struct TcGatesArgs {
   int H, K, Ks, B;
   int nkb;                  // 64-term chunks: ceil(K / 64)
   int tau_rows;             // rows of one plane of tau's map (B: the lo plane starts there)
-  const __nv_bfloat16* U;   // factor U [4][H][Ks] and the stored tau' pair [2][B][ldt]: the terms of an
-  const __nv_bfloat16* tau; // intermediate depth that is not a multiple of 16 past the last 16-term slice
-  int ldt;                  // are added from these on the CUDA cores
+  const __nv_bfloat16* U;   // factor U [4][H][Ks] and the stored tau' pair [2][B][ldt]: the reduce kernel
+  const __nv_bfloat16* tau; // adds the terms of an intermediate depth past its last 16-term slice boundary
+  int ldt;                  // from these on the CUDA cores
   long long tau_plane;
   const float* bias;        // [4][H]
   float* c_state;           // [B][H] fp32, c_{t-1} in, c_t out
@@ -280,6 +280,7 @@ struct TcGatesArgs {
   // the cell update of Sec. II in a second kernel.
   int ks, nkb_per;
   float* part;
+  bool raw;                 // raw-sum mode: ks > 1, or an intermediate depth that is not a multiple of 16
 };
 // `nt` (32, 64 or 128) must match the box rows of Tau's map.
 cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s);

@@ -38,7 +38,11 @@
 // chunks [kb0, kb1) each).  Such a CTA stores its raw gate sums, and at a
 // depth that ends inside its range the sums up to that depth, to a scratch
 // array; tc_gates_reduce_kernel then adds the splits in split order and runs
-// the cell update at full depth and at every intermediate depth.
+// the cell update at full depth and at every intermediate depth.  The same
+// raw-sum mode (with one split if the grid is large enough) serves runs with
+// an intermediate depth that is not a multiple of the MMA's 16 terms: the
+// MMA stream stops at the depth's last slice boundary and the reduce kernel
+// adds the remaining terms from U and the stored tau' pair.
 //
 // Every mbarrier wait is bounded in wall time; a wait that runs out writes
 // the device status word, the CTA stops issuing work, waits (bounded) for
@@ -81,38 +85,28 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& w, float* f) {
   }
 }
 
-// Gate sums at an intermediate depth k_j that is not a multiple of 16: the
-// MMA stream stopped at the slice boundary k0 = k_j - r (0 < r < 16), and
-// this adds the r terms [k0, k_j) for unit j and the 16 streams from nbeg,
-// y[g][c] += sum_{k0 <= k < k_j} u_{g,k}[j] (tau'_hi + tau'_lo)[n][(g, k)],
-// from the factor U and the stored tau' pair, on the CUDA cores.
-__device__ __noinline__ void add_remainder_terms(const TcGatesArgs& a, int j, int nbeg, int k0, int r,
-                                                 float (&y)[4][16]) {
-#pragma unroll 1
-  for (int g = 0; g < 4; ++g) {
-    float u[16];
-    const uint4* up = reinterpret_cast<const uint4*>(a.U + ((long long)g * a.H + j) * a.Ks + k0);
-    bf16x8_to_f32(__ldg(up), u);
-    bf16x8_to_f32(__ldg(up + 1), u + 8);
-#pragma unroll 1
-    for (int c = 0; c < 16; ++c) {
-      const int n = nbeg + c;
-      if (n >= a.B) break;
-      const long long o = (long long)n * a.ldt + (long long)g * a.Ks + k0;
-      const uint4* th = reinterpret_cast<const uint4*>(a.tau + o);
-      const uint4* tl = reinterpret_cast<const uint4*>(a.tau + a.tau_plane + o);
-      float hi[16], lo[16];
-      bf16x8_to_f32(th[0], hi);
-      bf16x8_to_f32(th[1], hi + 8);
-      bf16x8_to_f32(tl[0], lo);
-      bf16x8_to_f32(tl[1], lo + 8);
-      float acc = 0.f;
+// Terms [k0, k0 + r) of gate g for stream n and unit j (0 < r < 16, k0 a
+// multiple of 16): sum of u_{g,k}[j] (tau'_hi + tau'_lo)[n][(g, k)], from the
+// factor U and the stored tau' pair.  These are the terms of an intermediate
+// depth k_j = k0 + r that is not a multiple of the MMA's 16-term slices: the
+// MMA stream stops at k0 and the reduce kernel adds them on the CUDA cores.
+__device__ __forceinline__ float remainder_terms(const TcGatesArgs& a, int g, int n, int j, int k0, int r) {
+  const uint4* up = reinterpret_cast<const uint4*>(a.U + ((long long)g * a.H + j) * a.Ks + k0);
+  const long long o = (long long)n * a.ldt + (long long)g * a.Ks + k0;
+  const uint4* th = reinterpret_cast<const uint4*>(a.tau + o);
+  const uint4* tl = reinterpret_cast<const uint4*>(a.tau + a.tau_plane + o);
+  float acc = 0.f;
 #pragma unroll
-      for (int k = 0; k < 16; ++k)
-        if (k < r) acc = fmaf(u[k], hi[k] + lo[k], acc);
-      y[g][c] += acc;
-    }
+  for (int h8 = 0; h8 < 2; ++h8) {
+    float u[8], hi[8], lo[8];
+    bf16x8_to_f32(__ldg(up + h8), u);
+    bf16x8_to_f32(th[h8], hi);
+    bf16x8_to_f32(tl[h8], lo);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (8 * h8 + k < r) acc = fmaf(u[k], hi[k] + lo[k], acc);
   }
+  return acc;
 }
 
 // ---------------------------------------------------------------------------
@@ -416,29 +410,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
     const uint32_t trow = tmem + ((32u * q) << 16);
     griddep_wait();  // c_t-1 and the outputs are shared with the kernels before this one
-    // c_{t-1} of this thread's unit for its streams, loaded once while the
-    // MMAs run (up to 32 streams; wider tiles load it per chunk below)
-    constexpr bool kCpPre = kHalf <= 32;
-    float cpv[kCpPre ? kHalf : 1];
-    if constexpr (kCpPre) {
-#pragma unroll
-      for (int c = 0; c < kHalf; ++c) {
-        const int n = n0 + cbeg + c;
-        cpv[c] = (!split && unit_ok && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
-      }
-    }
     for (int step = jj_lo; step <= jj_hi; ++step) {
       const bool final_sums = step == jj_hi;
       const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)((step - jj_lo) & 1),
                                limit, err);
       tc_fence_after();
       const bool write = ok && *err == 0 && unit_ok;
-      // an intermediate depth off the 16-term slices: the MMAs stopped at
-      // rem_k0, the last rem_r terms are added on the CUDA cores; when this
-      // CTA issued no MMA before rem_k0 the accumulator holds nothing yet
-      const int kj = final_sums ? 0 : a.ck.k[step];
-      const int rem_r = kj & 15, rem_k0 = kj - rem_r;
-      const bool acc_valid = final_sums || rem_k0 > kb0 * kTileK;
+      // a depth whose last 16-term slice boundary is the start of this CTA's
+      // range: no MMA was issued below it, the raw sums are zero (the reduce
+      // kernel adds the terms past the boundary)
+      const bool acc_valid = final_sums || ((a.ck.k[step] >> 4) << 4) > kb0 * kTileK;
       if constexpr (SPLIT) {
         // raw gate sums of this CTA's terms: slot z for its whole range, slot
         // ks + step at a depth that ends inside it
@@ -449,18 +430,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
           tmem_wait_ld();
           if (!write) continue;
-          if (!acc_valid)
-#pragma unroll
-            for (int g = 0; g < 4; ++g)
-#pragma unroll
-              for (int c = 0; c < 16; ++c) y[g][c] = 0.f;
-          if (rem_r) add_remainder_terms(a, j, n0 + c0, rem_k0, rem_r, y);
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
             const int n = n0 + c0 + c;
             if (n >= a.B) break;
 #pragma unroll
-            for (int g = 0; g < 4; ++g) a.part[((slot * 4 + g) * a.B + n) * a.H + j] = y[g][c];
+            for (int g = 0; g < 4; ++g) a.part[((slot * 4 + g) * a.B + n) * a.H + j] = acc_valid ? y[g][c] : 0.f;
           }
         }
         if (!final_sums) {
@@ -469,53 +444,49 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         continue;
       }
-      constexpr int kUnroll = kCpPre ? kHalf / 16 : 1;  // registers for cpv, one chunk live otherwise
-#pragma unroll kUnroll
-      for (int ci = 0; ci < kHalf / 16; ++ci) {
-        const int c0 = cbeg + 16 * ci;
-        float cp[16];  // c_{t-1}, loaded before any store of this chunk
+      // four streams per round: a compact loop that stays in the instruction
+      // cache (fully unrolled cells of 16-stream chunks, at about 50
+      // instructions each, did not), with c_{t-1} fetched one round ahead
+      auto load_c = [&](int cb, float (&dst)[4]) {
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          if constexpr (kCpPre) {
-            cp[c] = cpv[16 * ci + c];
-          } else {
-            const int n = n0 + c0 + c;
-            cp[c] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
-          }
+        for (int e = 0; e < 4; ++e) {
+          const int n = n0 + cb + e;
+          dst[e] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
         }
-        float y[4][16];
+      };
+      float cpn[4];
+      load_c(cbeg, cpn);
+#pragma unroll 1
+      for (int c4 = cbeg; c4 < cbeg + kHalf; c4 += 4) {
+        float cp[4] = {cpn[0], cpn[1], cpn[2], cpn[3]};  // loaded before any store of this round
+        if (c4 + 4 < cbeg + kHalf) load_c(c4 + 4, cpn);
+        float y[4][4];
+        __syncwarp();
+        tmem_ld4x4_sync(trow + c4, trow + NT + c4, trow + 2 * NT + c4, trow + 3 * NT + c4, y);
+        if (write) {
 #pragma unroll
-        for (int g = 0; g < 4; ++g) tmem_ld16(trow + g * NT + c0, y[g]);
-        tmem_wait_ld();
-        if (!write) continue;
-        if (!acc_valid)
-#pragma unroll
-          for (int g = 0; g < 4; ++g)
-#pragma unroll
-            for (int c = 0; c < 16; ++c) y[g][c] = 0.f;
-        if (rem_r) add_remainder_terms(a, j, n0 + c0, rem_k0, rem_r, y);
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-          const int n = n0 + c0 + c;
-          if (n >= a.B) break;
-          const long long sj = (long long)n * a.H + j;
-          float hh, cc;
-          lstm_cell_f(y[0][c] + bias[0], y[1][c] + bias[1], y[2][c] + bias[2], y[3][c] + bias[3], cp[c], hh, cc);
-          if (!final_sums) {
-            const long long o = (long long)step * a.ck_stride + sj;  // (no split: jj_lo = 0)
-            if (a.ckpt_h) a.ckpt_h[o] = hh;
-            if (a.ckpt_c) a.ckpt_c[o] = cc;
-          } else {
-            a.c_state[sj] = cc;
-            if (a.out_h) a.out_h[sj] = hh;
-            __nv_bfloat16 hi, lo;
-            bf16_pair(hh, hi, lo);
-            const long long hj = (long long)n * a.ldh + j;
-            a.h_bf16[hj] = hi;
-            a.h_bf16[a.h_plane + hj] = lo;
-            if (a.seq_bf16) {
-              a.seq_bf16[hj] = hi;
-              a.seq_bf16[a.seq_plane + hj] = lo;
+          for (int e = 0; e < 4; ++e) {
+            const int n = n0 + c4 + e;
+            if (n >= a.B) break;
+            const long long sj = (long long)n * a.H + j;
+            float hh, cc;
+            lstm_cell_f(y[0][e] + bias[0], y[1][e] + bias[1], y[2][e] + bias[2], y[3][e] + bias[3], cp[e], hh, cc);
+            if (!final_sums) {
+              const long long o = (long long)step * a.ck_stride + sj;  // (no split: jj_lo = 0)
+              if (a.ckpt_h) a.ckpt_h[o] = hh;
+              if (a.ckpt_c) a.ckpt_c[o] = cc;
+            } else {
+              a.c_state[sj] = cc;
+              if (a.out_h) a.out_h[sj] = hh;
+              __nv_bfloat16 hi, lo;
+              bf16_pair(hh, hi, lo);
+              const long long hj = (long long)n * a.ldh + j;
+              a.h_bf16[hj] = hi;
+              a.h_bf16[a.h_plane + hj] = lo;
+              if (a.seq_bf16) {
+                a.seq_bf16[hj] = hi;
+                a.seq_bf16[a.seq_plane + hj] = lo;
+              }
             }
           }
         }
@@ -534,10 +505,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
-// After a term-axis split of the gate GEMM: one thread per (stream n, unit
-// j) adds the splits' raw gate sums in split order and runs the cell update
-// of Sec. II, at full depth and at each intermediate depth k_j (the splits
-// before the one k_j ends in, then that split's sums up to k_j).
+// After the gate GEMM in raw-sum mode (a term-axis split, or intermediate
+// depths off the 16-term slices): one thread per (stream n, unit j) adds the
+// splits' raw gate sums in split order and runs the cell update of Sec. II,
+// at full depth and at each intermediate depth k_j (the splits before the one
+// k_j ends in, then that split's sums up to k_j's last slice boundary, then
+// the terms from there to k_j).
 __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
   griddep_launch_dependents();  // the next step's tau' kernel may start its set-up
   const long long total = (long long)a.B * a.H;
@@ -553,12 +526,14 @@ __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
   const float cp = a.c_state[i];
   for (int jj = 0; jj < a.ck.n; ++jj) {
     const int sj = ((a.ck.k[jj] + kTileK - 1) / kTileK - 1) / a.nkb_per;  // split the depth ends in
+    const int r = a.ck.k[jj] & 15;  // terms past the depth's last 16-term slice boundary
     float y[4];
 #pragma unroll
     for (int g = 0; g < 4; ++g) {
       float v = 0.f;
       for (int z = 0; z < sj; ++z) v += part[(z * 4 + g) * gs];
       y[g] = v + part[((a.ks + jj) * 4 + g) * gs] + bias[g];
+      if (r != 0) y[g] += remainder_terms(a, g, n, j, a.ck.k[jj] - r, r);
     }
     float hh, cc;
     lstm_cell_f(y[0], y[1], y[2], y[3], cp, hh, cc);
@@ -715,9 +690,9 @@ cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& 
     attr = true;
   }
   const cudaError_t e =
-      launch_pdl(kern, dim3((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT, a.ks > 1 ? a.ks : 1), smem, s,
+      launch_pdl(kern, dim3((a.H + kTileM - 1) / kTileM, (a.B + NT - 1) / NT, a.ks), smem, s,
                  *reinterpret_cast<const CUtensorMap*>(U.bytes), *reinterpret_cast<const CUtensorMap*>(Tau.bytes), a);
-  if (e != cudaSuccess || a.ks <= 1) return e;
+  if (e != cudaSuccess || !SPLIT) return e;
   const long long total = (long long)a.B * a.H;
   return launch_pdl_block(tc_gates_reduce_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, s, a);
 }
@@ -776,9 +751,9 @@ cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a,
 
 cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs& a, int nt, cudaStream_t s) {
   switch (nt) {
-    case 128: return a.ks > 1 ? launch_gates_t<128, 4, true>(U, Tau, a, s) : launch_gates_t<128, 4, false>(U, Tau, a, s);
-    case 64: return a.ks > 1 ? launch_gates_t<64, 6, true>(U, Tau, a, s) : launch_gates_t<64, 6, false>(U, Tau, a, s);
-    default: return a.ks > 1 ? launch_gates_t<32, 8, true>(U, Tau, a, s) : launch_gates_t<32, 8, false>(U, Tau, a, s);
+    case 128: return a.raw ? launch_gates_t<128, 4, true>(U, Tau, a, s) : launch_gates_t<128, 4, false>(U, Tau, a, s);
+    case 64: return a.raw ? launch_gates_t<64, 6, true>(U, Tau, a, s) : launch_gates_t<64, 6, false>(U, Tau, a, s);
+    default: return a.raw ? launch_gates_t<32, 8, true>(U, Tau, a, s) : launch_gates_t<32, 8, false>(U, Tau, a, s);
   }
 }
 

@@ -231,18 +231,21 @@ int select_path(int dtype, int H, int K, int T, const Checkpoints& ck, int force
 
 struct TensorTiles {
   int bnh = 0, nt = 0, ks = 1, nkb_per = 0;
+  bool raw = false;  // raw gate sums and a reduce kernel (term split, or depths off the 16-term slices)
 };
 
 // Tiles of the tensor-core path for one layer: streams per tile of the tau'
 // GEMM (bnh) and of the gate GEMM (nt), and the gate GEMM's term-axis
 // splits (ks, of nkb_per 64-term chunks each; small grids split the terms
 // over more CTAs).
-TensorTiles tensor_tiles(int H, int B, int K) {
+TensorTiles tensor_tiles(int H, int B, int K, const Checkpoints& ck) {
   TensorTiles t;
   t.bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
   t.nt = tc_gates_tile_n(H, B);
   const int gate_tiles = ((H + 127) / 128) * ((B + t.nt - 1) / t.nt);
   t.ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &t.nkb_per);
+  t.raw = t.ks > 1;
+  for (int j = 0; j < ck.n; ++j) t.raw = t.raw || ck.k[j] % 16 != 0;
   return t;
 }
 
@@ -310,9 +313,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
   LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
   h->launches += 1;
-  const TensorTiles tt = tensor_tiles(H, B, K);
+  const TensorTiles tt = tensor_tiles(H, B, K, ck);
   const int bnh = tt.bnh, nt = tt.nt, ks = tt.ks, nkb_per = tt.nkb_per;
-  if (ks > 1) {
+  if (tt.raw) {
     const size_t need = (size_t)(ks + ck.n) * 4 * B * H * sizeof(float);
     if (need > h->gpart_bytes) {
       LA_CUDA(h, cudaStreamSynchronize(h->stream), "synchronising before growing the split buffer");
@@ -374,8 +377,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ga.ks = ks;
     ga.nkb_per = nkb_per;
     ga.part = h->gpart;
+    ga.raw = tt.raw;
     LA_CUDA(h, launch_tc_gates(s.map_u, mt, ga, nt, h->stream), "gate GEMM launch");
-    h->launches += ks > 1 ? 3 : 2;
+    h->launches += tt.raw ? 3 : 2;
   }
   if (out_c) LA_CUDA(h, cudaMemcpyAsync(out_c, cs, (size_t)B * H * sizeof(float), cudaMemcpyDeviceToDevice, h->stream),
                      "c copy");
@@ -1029,7 +1033,7 @@ int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int* chec
       v[LSTM_APPROX_PLAN_TMEM_COLUMNS] = pc.ag.tcols;
     }
   } else if (path == LSTM_APPROX_PATH_TENSOR) {
-    const TensorTiles tt = tensor_tiles(hidden, B, K);
+    const TensorTiles tt = tensor_tiles(hidden, B, K, ck);
     v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = tt.bnh;
     v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = tt.nt;
     v[LSTM_APPROX_PLAN_GATE_SPLITS] = tt.ks;

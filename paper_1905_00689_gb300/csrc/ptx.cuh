@@ -254,6 +254,27 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
+// Four loads of 32 lanes x 4 consecutive 32-bit columns (at t0 .. t3) and the
+// wait for them in one statement, so that no use of the values can be
+// scheduled before they have arrived: v[i][c] = column t_i + c of this
+// thread's row.
+__device__ __forceinline__ void tmem_ld4x4_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3,
+                                                float (&v)[4][4]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%16];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4, %5, %6, %7}, [%17];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%8, %9, %10, %11}, [%18];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%12, %13, %14, %15}, [%19];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(t0), "r"(t1), "r"(t2), "r"(t3)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i >> 2][i & 3] = __uint_as_float(r[i]);
+}
+
 // Two tmem_ld16 and one wait for both in one statement, so that no use of
 // the values can be scheduled before they have arrived.
 __device__ __forceinline__ void tmem_ld16x2_sync(uint32_t ta, uint32_t tb, float (&va)[16], float (&vb)[16]) {
