@@ -212,10 +212,48 @@ def cpu_baseline(budget_s: float = 12.0) -> dict:
                        f"checkpoints {list(CKPTS)}) in {s_per_run * runs:.1f} s, fp64 NumPy, 1 thread")}
 
 
+# the oracle on every workload: (workload, keep, K, intermediate depths, T and
+# streams of the bounded sample); streams are independent, so the oracle's
+# throughput on a few streams and steps is its throughput on the whole workload
+ORACLE_CONFIGS = (("c1", 0.5, 64, (), None, 1), ("c2", 0.25, 256, (16, 64), None, 1),
+                  ("c3", 0.5, 512, (), 4, 1), ("c4", 0.5, 512, (), 2, 1), ("c4", 0.1, 128, (), 4, 1),
+                  ("c5", 0.3, 1024, (16, 64, 256, 1024), 2, 1))
+
+
+def oracle_config_sweep(budget_s: float = 4.0) -> list:
+    """The fp64 oracle (as it stands, one thread) timed on a bounded sample of
+    every workload: timesteps*streams/s and the sample it was taken on."""
+    import oracle
+    out = []
+    for name, keep, K, cps, T_s, B_s in ORACLE_CONFIGS:
+        w = WORKLOADS[name]
+        T_s = T_s or w.T
+        layers = [synthetic_layer_factors(w, l, K, keep) for l in range(w.L)]
+        x = workload_inputs(w, T=T_s, B=B_s).astype(np.float32).astype(np.float64)
+        runs, t0 = 0, time.perf_counter()
+        while True:
+            oracle.run_lstm(layers, x, K, checkpoints=cps)
+            runs += 1
+            el = time.perf_counter() - t0
+            if el >= budget_s:
+                break
+        out.append({"workload": w.name, "keep": keep, "K": K, "checkpoints": list(cps),
+                    "value": T_s * B_s * runs / el, "unit": UNIT, "cores": 1,
+                    "sample": f"{runs} runs of T={T_s}, B={B_s} in {el:.1f} s"})
+    return out
+
+
 def run_reference(args):
     ws, rank, _ = _dist_env()
     if rank != 0:
         return
+    if args.all_configs:  # the oracle on every workload (one line per workload), then the usual line
+        env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        code = (f"import sys, json; sys.path.insert(0, {HERE!r}); import bench; "
+                f"print(json.dumps(bench.oracle_config_sweep()))")
+        r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=1200)
+        print(json.dumps({"impl": "reference", "oracle_by_workload": json.loads(r.stdout) if r.returncode == 0
+                          else "failed: " + r.stderr[-300:]}), flush=True)
     import oracle
     layers = [synthetic_layer_factors(WL, 0, K_MAIN, KEEP)]
     x = workload_inputs(WL).astype(np.float32).astype(np.float64)
@@ -652,6 +690,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--all-configs", action="store_true",
+                    help="with --impl reference: first time the oracle on every workload (a few seconds each)")
     ap.add_argument("--no-large", action="store_true", help="skip the large-batch tensor-core measurements")
     ap.add_argument("--profile", choices=sorted(WORKLOADS), default=None,
                     help="only run one workload's path (warmup + steps runs), for profilers")

@@ -29,6 +29,7 @@
 #ifndef LSTM_APPROX_H
 #define LSTM_APPROX_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -174,6 +175,37 @@ int lstm_approx_run_static(const float *Vx, const float *Vh, const float *U, con
                            const float *h0, const float *c0, float *out_h, float *out_c,
                            const int *checkpoints, int J, float *ckpt_h, float *ckpt_c,
                            void *cuda_stream, char *msg, int msg_len);
+
+/*
+ * Dense comparator: the LSTM of Sec. II with the full gate matrices
+ * W_g = [Wx_g Wh_g] (no approximation), for one fp32 layer, on the same kind
+ * of persistent cluster kernel as the approximate path (one cluster per
+ * stream; Wh held in tensor memory for the whole launch; one h exchange per
+ * timestep).  It serves as the dense baseline against which the speed-up of
+ * the approximation is measured (the paper compares its approximate design
+ * with dense designs on each platform, Sec. VI-B, Table I).
+ *
+ *   Wx    DEVICE [4H][D] fp32, row g*H + j = the input part of row j of W_g
+ *   Wh    DEVICE [4H][H] fp32, row g*H + j = the recurrent part of that row
+ *   bias  DEVICE [4][H] or NULL;  D >= 1, 1 <= H <= 512
+ *   x, h0, c0, out_h, out_c: as lstm_approx_run with L = 1 (DEVICE, fp32)
+ *   workspace  DEVICE buffer of at least
+ *              lstm_approx_dense_workspace_bytes(H, T, B) bytes, 256-byte
+ *              aligned, owned by the caller (the hoisted Wx x_t and a status
+ *              word); it must not be used by another call in flight
+ *   cuda_stream  cudaStream_t (NULL = legacy default stream)
+ *   msg   optional host buffer of msg_len bytes for an error text
+ *
+ * Synchronous: waits for the stream.  Returns OK, EINVAL (sizes, NULL,
+ * workspace too small or misaligned), ECUDA or ETIMEOUT (a bounded
+ * in-kernel wait ran out).  Allocates nothing.
+ */
+int lstm_approx_dense_run(const float *Wx, const float *Wh, const float *bias, int D, int H,
+                          const float *x, int T, int B, const float *h0, const float *c0,
+                          float *out_h, float *out_c, void *workspace, size_t workspace_bytes,
+                          void *cuda_stream, char *msg, int msg_len);
+/* Workspace bytes lstm_approx_dense_run needs for (H, T, B); 0 for invalid sizes. */
+size_t lstm_approx_dense_workspace_bytes(int H, int T, int B);
 
 /*
  * Wait for the handle's stream and report kernel-side status: OK, or

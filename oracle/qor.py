@@ -39,25 +39,46 @@ from .factors import decompose_gate, decompose_gate_variant
 from .recurrence import lstm_cell, op_count, run_lstm
 
 
-def dense_lstm(weights: Sequence[np.ndarray], x: np.ndarray) -> np.ndarray:
-    """h_t of the dense LSTM of Sec. II: y_g = W_g [x_t; h_{t-1}], h0 = c0 = 0."""
+def dense_lstm(weights: Sequence[np.ndarray], x: np.ndarray, bias=None, h0=None, c0=None,
+               return_c: bool = False):
+    """h_t of the dense LSTM of Sec. II: y_g = W_g [x_t; h_{t-1}] (+ b_g).
+
+    bias: None or [4][H]; h0, c0: None (zeros) or [B][H].  Returns h [T][B][H],
+    and the final c [B][H] as well when return_c."""
     T, B, _ = x.shape
     H = weights[0].shape[0]
-    h = np.zeros((B, H))
-    c = np.zeros((B, H))
+    h = np.zeros((B, H)) if h0 is None else np.asarray(h0, dtype=np.float64)
+    c = np.zeros((B, H)) if c0 is None else np.asarray(c0, dtype=np.float64)
     out = np.zeros((T, B, H))
     for t in range(T):
         xt = np.concatenate([x[t], h], axis=1)          # [B][C]
         y = [xt @ W.T for W in weights]                 # four [B][H]
-        h, c = lstm_cell(y, c)
+        h, c = lstm_cell(y, c, bias)
         out[t] = h
-    return out
+    return (out, c) if return_c else out
 
 
 def softmax(z: np.ndarray) -> np.ndarray:
     z = z - z.max(axis=-1, keepdims=True)
     e = np.exp(z)
     return e / e.sum(axis=-1, keepdims=True)
+
+
+def head_matrix(H: int, classes: int = 10, seed: int = 1905) -> np.ndarray:
+    """The seeded random linear head A (classes x H, entries N(0, 1/sqrt(H)))
+    that stands in for the driving model's output layer."""
+    return np.random.Generator(np.random.PCG64(seed)).normal(0.0, 1.0 / np.sqrt(H), (classes, H))
+
+
+def curve_point(h: np.ndarray, h_ref: np.ndarray, A: np.ndarray) -> Dict:
+    """Quality of approximate hidden states h against the dense ones h_ref
+    (same shape, last axis H): the relative error ||h - h_ref|| / ||h_ref||
+    over all entries, and KL(p_ref || p) of the head's softmax averaged over
+    every output vector."""
+    p_ref = softmax(h_ref @ A.T)
+    p = softmax(h @ A.T)
+    kl = float(np.mean(np.sum(p_ref * (np.log(p_ref) - np.log(p)), axis=-1)))
+    return {"rel_h_error": float(np.linalg.norm(h - h_ref) / np.linalg.norm(h_ref)), "head_kl": kl}
 
 
 def reconstruct(f: dict, K: int, C: int) -> np.ndarray:
@@ -77,8 +98,7 @@ def qor_table(weights: Sequence[np.ndarray], x: np.ndarray, nzs: Sequence[int], 
         raise ValueError(scheme)
     H, C = weights[0].shape
     h_ref = dense_lstm(weights, x)
-    A = np.random.Generator(np.random.PCG64(seed)).normal(0.0, 1.0 / np.sqrt(H), (classes, H))
-    p_ref = softmax(h_ref @ A.T)
+    A = head_matrix(H, classes, seed)
     w_norm = np.sqrt(sum(float(np.sum(W * W)) for W in weights))
     rows = []
     for nz in nzs:
@@ -88,12 +108,11 @@ def qor_table(weights: Sequence[np.ndarray], x: np.ndarray, nzs: Sequence[int], 
             layer = [decompose_gate_variant(W, max(Ks), nz, residual=False) for W in weights]
         for K in Ks:
             h = run_lstm([layer], x, K)["h"]
-            p = softmax(h @ A.T)
-            kl = float(np.mean(np.sum(p_ref * (np.log(p_ref) - np.log(p)), axis=-1)))
+            pt = curve_point(h, h_ref, A)
             w_err = np.sqrt(sum(float(np.sum((W - reconstruct(f, K, C)) ** 2)) for W, f in zip(weights, layer)))
             rows.append({"NZ": nz, "K": K, "scheme": scheme,
-                         "rel_h_error": float(np.linalg.norm(h - h_ref) / np.linalg.norm(h_ref)),
-                         "head_kl": kl,
+                         "rel_h_error": pt["rel_h_error"],
+                         "head_kl": pt["head_kl"],
                          "rel_w_error": w_err / w_norm,
                          "ops": 4 * op_count(H, nz, K), "dense_ops": 4 * 2 * H * C})
     return rows

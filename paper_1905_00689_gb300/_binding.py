@@ -35,7 +35,7 @@ EXPORTS = (
     "lstm_approx_create", "lstm_approx_set_factors", "lstm_approx_run", "lstm_approx_run_host",
     "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
     "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times", "lstm_approx_run_static",
-    "lstm_approx_plan", "lstm_approx_get_term",
+    "lstm_approx_plan", "lstm_approx_get_term", "lstm_approx_dense_run", "lstm_approx_dense_workspace_bytes",
 )
 
 _lib = None
@@ -75,9 +75,13 @@ def load(path: str = LIB_PATH):
     lib.lstm_approx_run_static.argtypes = [P, P, P, P, P, I, I, I, P, I, I, P, P, P, P, P, I, P, P, P,
                                            ctypes.c_char_p, I]
     lib.lstm_approx_plan.argtypes = [I, I, I, I, I, P, I, I, I, I, P, I, ctypes.c_char_p, I]
+    lib.lstm_approx_dense_run.argtypes = [P, P, P, I, I, P, I, I, P, P, P, P, P, ctypes.c_size_t, P,
+                                          ctypes.c_char_p, I]
+    lib.lstm_approx_dense_workspace_bytes.argtypes = [I, I, I]
     for name in EXPORTS:
-        if name not in ("lstm_approx_last_error", "lstm_approx_destroy"):
+        if name not in ("lstm_approx_last_error", "lstm_approx_destroy", "lstm_approx_dense_workspace_bytes"):
             getattr(lib, name).restype = ctypes.c_int
+    lib.lstm_approx_dense_workspace_bytes.restype = ctypes.c_size_t
     _lib = lib
     return lib
 
@@ -117,6 +121,32 @@ def run_static(Vx, Vh, U, sigma, bias, x, K, out_h, h0=None, c0=None, out_c=None
                                     _ptr(ckpt_h), _ptr(ckpt_c), ctypes.c_void_p(stream.cuda_stream), msg, 512)
     if rc != OK:
         raise LSTMApproxError(rc, msg.value.decode())
+
+
+def dense_run(Wx, Wh, bias, x, out_h, h0=None, c0=None, out_c=None, workspace=None, stream=None):
+    """lstm_approx_dense_run on torch tensors (device, fp32): the dense LSTM
+    comparator.  `workspace` (a uint8 device tensor of at least
+    dense_workspace_bytes(H, T, B) bytes) is allocated here when not given."""
+    import torch
+    lib = load()
+    T, B, D = x.shape
+    H = Wh.shape[1]
+    need = lib.lstm_approx_dense_workspace_bytes(H, T, B)
+    if workspace is None:
+        workspace = torch.empty(need + 256, dtype=torch.uint8, device=x.device)
+        off = (-workspace.data_ptr()) % 256
+        workspace = workspace[off:off + need]
+    s = stream if stream is not None else torch.cuda.current_stream(x.device)
+    msg = ctypes.create_string_buffer(256)
+    rc = lib.lstm_approx_dense_run(_ptr(Wx), _ptr(Wh), _ptr(bias), D, H, _ptr(x), T, B, _ptr(h0), _ptr(c0),
+                                   _ptr(out_h), _ptr(out_c), workspace.data_ptr(), workspace.numel(),
+                                   ctypes.c_void_p(s.cuda_stream), msg, 256)
+    if rc != OK:
+        raise LSTMApproxError(rc, msg.value.decode())
+
+
+def dense_workspace_bytes(H: int, T: int, B: int) -> int:
+    return int(load().lstm_approx_dense_workspace_bytes(H, T, B))
 
 
 def plan(dtype: int, hidden: int, T: int, B: int, K: int, checkpoints: Sequence[int] = (), force_path: int = 0,

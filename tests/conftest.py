@@ -20,6 +20,10 @@ def pytest_runtest_setup(item):
 def pytest_terminal_summary(terminalreporter):
     """Largest elementwise and normwise error of every parity check, per test."""
     import parity_util
+    if parity_util.NOTES:
+        terminalreporter.section("tables measured in this session")
+        for line in parity_util.NOTES:
+            terminalreporter.write_line(line)
     if not parity_util.REPORT:
         return
     terminalreporter.section("parity errors (max over outputs: elementwise / normwise, bound)")

@@ -102,6 +102,7 @@ def oracle_run(layers, x, K, dtype="fp32", **kw):
 # the session, printed by the terminal-summary hook in conftest.py
 REPORT = []
 CURRENT_TEST = [""]
+NOTES = []  # lines a test asks to print in the session summary (tables measured on the GPU)
 
 
 def assert_parity(got, ref, tol, keys=("h", "c_last", "ckpt_h", "ckpt_c")):

@@ -28,6 +28,26 @@ def test_dense_reference_matches_torch_lstm():
     np.testing.assert_allclose(qor.dense_lstm(W, x), ref.numpy(), rtol=1e-12, atol=1e-13)
 
 
+def test_dense_reference_with_bias_and_initial_state_matches_torch_lstm():
+    torch = pytest.importorskip("torch")
+    D, H, T, B = 5, 4, 6, 3
+    W = _weights(H, D + H, 310)
+    rng = np.random.default_rng(7)
+    bias = rng.standard_normal((4, H))
+    h0, c0 = rng.standard_normal((B, H)), rng.standard_normal((B, H))
+    x = draw_inputs(T, B, D, "uniform", 5)
+    lstm = torch.nn.LSTM(D, H).double()
+    with torch.no_grad():
+        lstm.weight_ih_l0.copy_(torch.from_numpy(np.concatenate([w[:, :D] for w in W])))
+        lstm.weight_hh_l0.copy_(torch.from_numpy(np.concatenate([w[:, D:] for w in W])))
+        lstm.bias_ih_l0.copy_(torch.from_numpy(bias.reshape(-1)))
+        lstm.bias_hh_l0.zero_()
+        ref, (hn, cn) = lstm(torch.from_numpy(x), (torch.from_numpy(h0)[None], torch.from_numpy(c0)[None]))
+    got, c_last = qor.dense_lstm(W, x, bias=bias, h0=h0, c0=c0, return_c=True)
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(c_last, cn.numpy()[0], rtol=1e-12, atol=1e-13)
+
+
 def test_full_rank_unpruned_has_zero_error_and_kl():
     D, H, T = 6, 4, 5
     C = D + H

@@ -67,15 +67,19 @@ def test_tensor_path_matches_cuda_core_path(cuda_device):
 
 
 @pytest.mark.parametrize("K", [32, 128, 512])
-def test_throughput_workload_full_size(cuda_device, K):
-    """D=1024, H=512, T=20, B=256, keep 50%: checked on sampled streams."""
+@pytest.mark.parametrize("with_depths", [False, True])
+def test_throughput_workload_full_size(cuda_device, K, with_depths):
+    """D=1024, H=512, T=20, B=256, keep 50%, at each K of the workload, with
+    and without intermediate depths (one off the 16-term slices): checked on
+    sampled streams."""
     w = WORKLOADS["c3"]
     layers = [list(synthetic_layer("c3", 0, 512, 0.5))]
     x = workload_inputs(w)
-    got, m = run_gpu(layers, x, K, dtype="bf16", max_rank=512)
+    cps = [16, K // 2 + 3, K] if with_depths else []
+    got, m = run_gpu(layers, x, K, dtype="bf16", max_rank=512, checkpoints=cps)
     assert m.query(Q_LAST_PATH) == PATH_TENSOR
     streams = [0, 77, 255]
-    ref = oracle_run(layers, x[:, streams], K, dtype="bf16")
+    ref = oracle_run(layers, x[:, streams], K, dtype="bf16", checkpoints=cps)
     assert_parity(_sample(got, streams), ref, BF16_TOL)
 
 
@@ -115,13 +119,16 @@ def test_throughput_workload_decomposed_factors(cuda_device):
     assert_parity(got, ref, BF16_TOL)
 
 
-@pytest.mark.parametrize("keep,K", [(0.5, 128), (0.1, 512)])
+@pytest.mark.parametrize("keep", [0.5, 0.1])
+@pytest.mark.parametrize("K", [8, 32, 128, 512])
 def test_large_batch_workload_full_size(cuda_device, keep, K):
-    """D=2048, H=1024, T=64, B=1024: checked on sampled streams."""
+    """D=2048, H=1024, T=64, B=1024 at every K and keep level of the
+    workload (prefixes of one 512-term factor set): checked on sampled
+    streams."""
     w = WORKLOADS["c4"]
-    layers = [list(synthetic_layer("c4", 0, K, keep))]
+    layers = [list(synthetic_layer("c4", 0, 512, keep))]
     x = workload_inputs(w)
-    got, _ = run_gpu(layers, x, K, dtype="bf16", max_rank=K)
+    got, _ = run_gpu(layers, x, K, dtype="bf16", max_rank=512)
     streams = [0, 513, 1023]
     ref = oracle_run(layers, x[:, streams], K, dtype="bf16")
     assert_parity(_sample(got, streams), ref, BF16_TOL)
