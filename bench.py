@@ -54,8 +54,8 @@ L2_FLUSH_BYTES = 256 << 20
 # holds only for the kernel sources it was taken on: `captured_traffic`
 # returns None once their SHA-256 differs.
 TRAFFIC_SOURCES = ("k_persistent.cu", "ptx.cuh")
-TRAFFIC_CAPTURE = {"sha256": "051ad6aa49332dfe7fb878270b2383b7b30d8f51743c8c35a2a19fcd16741d38",
-                   "bytes": 4350976}
+TRAFFIC_CAPTURE = {"sha256": "129d11d27b27b4081597799e7eeec8d1070738bcbeeef841428a6c5385c10b41",
+                   "bytes": 4340736}
 
 
 def captured_traffic():
@@ -376,6 +376,7 @@ def run_ours(args):
     large = [] if (args.quick or args.no_large) else large_batch_sweep(dev, stream, peaks_bf16())
     paper_case = None if (args.quick or args.no_large) else paper_case_sweep(dev, stream)
     dense = None if args.quick else dense_comparator(dev, stream, x)
+    dense_kernel = None if args.quick else dense_kernel_comparator(dev, stream, flush, x, statistics.median(step_ms))
     k_sweeps = [] if (args.quick or args.no_large) else workload_k_sweeps(dev, flush)
 
     # ---- end to end through the host-buffer entry point ---------------------
@@ -430,6 +431,7 @@ def run_ours(args):
             "k_sweeps": k_sweeps,
             "paper_case_study": paper_case,
             "dense_lstm_comparator": dense,
+            "dense_kernel_comparator": dense_kernel,
         }
         if ws == 1 and not (args.no_cpu_baseline or args.quick):
             line["cpu_baseline"] = cpu_baseline()
@@ -552,14 +554,20 @@ def large_batch_sweep(dev, stream, peak):
             ph.append(m.phase_times())
         m.set_option(OPT_TIMING, 0)
         xp_ms = statistics.median(p[0] for p in ph)
-        exec_fl = sum(w.T * w.B * (2 * 4 * K * w.C(l) + 2 * 4 * K * w.H) for l in range(w.L))
-        xp_fl = sum(w.T * w.B * 2 * 4 * K * w.input_dim(l) for l in range(w.L))
+        # MMA work as issued: masked-dense products, each activation operand
+        # as its bf16 pair (two MMAs per factor tile)
+        exec_fl = sum(2 * w.T * w.B * (2 * 4 * K * w.C(l) + 2 * 4 * K * w.H) for l in range(w.L))
+        # the method's own operations (Sec. III): 4 gates x K (2R + 2NZ + 1) per stream-step
+        alg_fl = sum(w.T * w.B * 4 * K * (2 * w.H + 2 * nz_from_keep(keep, w.C(l)) + 1) for l in range(w.L))
+        xp_fl = sum(2 * w.T * w.B * 2 * 4 * K * w.input_dim(l) for l in range(w.L))
         xp_tf = xp_fl / (xp_ms / 1e3) / 1e12
         out.append({
             "workload": w.name, "keep": keep, "K": K, "checkpoints": list(cps),
             "path": {1: "simt", 2: "persistent", 3: "tensor"}.get(m.query(Q_LAST_PATH)),
             "ms_per_run": ms, "value": w.T * w.B / (ms / 1e3), "unit": UNIT,
             "executed_tflops": exec_fl / (ms / 1e3) / 1e12,
+            "executed_frac": exec_fl / (ms / 1e3) / 1e12 / peak_tf,
+            "algorithmic_tflops": alg_fl / (ms / 1e3) / 1e12,
             "input_projection": {"ms": xp_ms, "tflops": xp_tf, "peak": peak_tf, "frac": xp_tf / peak_tf,
                                  "peak_source": peak_src},
             "recurrence_ms": statistics.median(p[1] for p in ph),
@@ -590,6 +598,49 @@ def dense_comparator(dev, stream, x, steps: int = 200) -> dict:
     return {"kind": "dense torch.nn.LSTM (cuDNN), fp32, same D/H/T/B, warm caches", "ms_per_run": ms,
             "value": T * B / (ms / 1e3), "unit": UNIT,
             "dense_weight_bytes": 4 * 4 * WL.H * (D + WL.H)}
+
+
+def dense_kernel_comparator(dev, stream, flush, x, approx_ms: float) -> list:
+    """The library's dense LSTM kernel (lstm_approx_dense_run: the full gate
+    matrices of Sec. II on the same persistent cluster design) timed like the
+    approximate path: on the benchmark shape with the L2 flushed before every
+    run (as the main timed loop), and on the paper's case-study shape
+    (H = 64, C = 8320, one timestep) with warm caches (as paper_case_sweep):
+    the like-for-like baseline of the approximation's speed-up (Sec. VI-B)."""
+    import torch
+    from paper_1905_00689_gb300 import dense_run, dense_workspace_bytes
+    from workloads import draw_weight
+    out = []
+    f1 = WORKLOADS["f1"]
+    for w, xin, ref_ms, flushed in ((WL, x, approx_ms, True), (f1, None, None, False)):
+        D, H, T, B = w.D, w.H, w.T, w.B
+        W = [draw_weight(H, D + H, 77 + g) for g in range(4)]
+        Wx = torch.from_numpy(np.concatenate([m[:, :D] for m in W]).astype(np.float32)).to(dev)
+        Wh = torch.from_numpy(np.concatenate([m[:, D:] for m in W]).astype(np.float32)).to(dev)
+        xx = xin if xin is not None else torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+        oh = torch.empty((T, B, H), device=dev)
+        ws = torch.empty(dense_workspace_bytes(H, T, B), dtype=torch.uint8, device=dev)
+        run = lambda: dense_run(Wx, Wh, None, xx, oh, workspace=ws, stream=stream)
+        for _ in range(5):
+            run()
+        n = 100
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for i, (a, b) in enumerate(evs):
+            if flushed:
+                flush.fill_(float(i))
+            a.record(stream)
+            run()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+        row = {"workload": w.name, "kind": "dense LSTM kernel of this library (lstm_approx_dense_run), fp32, " +
+                                          ("L2 flushed before each run" if flushed else "warm caches"),
+               "ms_per_run": ms,
+               "value": T * B / (ms / 1e3), "unit": UNIT, "dense_weight_bytes": 4 * 4 * H * (D + H)}
+        if ref_ms is not None:
+            row["approx_speedup"] = ms / ref_ms
+        out.append(row)
+    return out
 
 
 # the paper's FPGA latencies for one timestep of its case-study LSTM (Table I),
@@ -659,6 +710,19 @@ def run_profile(args):
     import torch
     from paper_1905_00689_gb300 import LSTMApprox, Q_LAST_PATH
     w = WORKLOADS[args.profile]
+    if args.profile_dense:  # the dense comparator kernel on this workload's shape (fp32, one layer)
+        from paper_1905_00689_gb300 import dense_run
+        from workloads import draw_weight
+        dev = torch.device("cuda", 0)
+        W = [draw_weight(w.H, w.D + w.H, 77 + g) for g in range(4)]
+        Wx = torch.from_numpy(np.concatenate([m[:, :w.D] for m in W]).astype(np.float32)).to(dev)
+        Wh = torch.from_numpy(np.concatenate([m[:, w.D:] for m in W]).astype(np.float32)).to(dev)
+        x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+        oh = torch.empty((w.T, w.B, w.H), device=dev)
+        for _ in range(args.warmup + args.steps):
+            dense_run(Wx, Wh, None, x, oh)
+        print(json.dumps({"profile": w.name, "dense": True, "runs": args.warmup + args.steps}), flush=True)
+        return
     keep = w.keeps[0]
     K = max(w.Ks)
     cps = list(w.checkpoints)
@@ -697,6 +761,8 @@ def main():
                     help="only run one workload's path (warmup + steps runs), for profilers")
     ap.add_argument("--profile-k", type=int, default=0, help="with --profile: this K instead of the workload's largest")
     ap.add_argument("--profile-keep", type=float, default=0.0, help="with --profile: this keep fraction")
+    ap.add_argument("--profile-dense", action="store_true",
+                    help="with --profile: the dense comparator kernel on the workload's shape (fp32, one layer)")
     ap.add_argument("--quick", action="store_true",
                     help="main timed loop only (short side measurements, no K sweep, no CPU baseline)")
     args = ap.parse_args()
