@@ -27,8 +27,8 @@
 //
 // tc_gates_kernel computes, for 128 hidden units x NT streams, the four gate
 // sums at once in four tensor-memory accumulators and runs the cell update
-// of Sec. II in the epilogue (fp32 sigmoid and tanh, relative error a few
-// 1e-7), storing h_t as its bf16 pair for the next step.  Intermediate depths k_j (multiples of 16) are
+// of Sec. II in the epilogue (fp32 sigmoid, tanh as 2 sigmoid(2z) - 1:
+// absolute error about 2e-7), storing h_t as its bf16 pair for the next step.  Intermediate depths k_j (multiples of 16) are
 // read from the same accumulators when the MMA stream reaches them: the MMA
 // thread commits, the epilogue warps compute the cell from the partial sums
 // and hand the accumulators back -- no prefix is recomputed.
@@ -267,7 +267,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   constexpr uint32_t kBBytes = NT * kTileK * 2;       // one plane of the tau' tile
   constexpr uint32_t kStage = kABytes + 2 * kBBytes;  // U tile, hi plane, lo plane
-  constexpr uint32_t kCols = 4 * NT < 32 ? 32 : 4 * NT;
+  constexpr uint32_t kAcc = 4 * NT < 32 ? 32 : 4 * NT;  // the four gate accumulators
+  // up to 64 streams per tile, c_{t-1} of the tile is staged in tensor memory
+  // too (columns kAcc .. kAcc + NT), so the cell loop reads it with the sums
+  constexpr bool kCTmem = !SPLIT && NT <= 64;
+  constexpr uint32_t kCols = kCTmem ? 2 * kAcc : kAcc;
   static_assert(S >= 4, "a chunk of all four gates must be resident");
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -410,6 +414,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * a.H + j];
     const uint32_t trow = tmem + ((32u * q) << 16);
     griddep_wait();  // c_t-1 and the outputs are shared with the kernels before this one
+    if constexpr (kCTmem) {  // c_{t-1} of this thread's unit and streams -> tensor memory, while the MMAs run
+#pragma unroll
+      for (int c0 = 0; c0 < kHalf; c0 += 16) {
+        float cv[16];
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int n = n0 + cbeg + c0 + c;
+          cv[c] = (unit_ok && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+        }
+        tmem_st16(trow + kAcc + cbeg + c0, cv);
+      }
+      tmem_wait_st();
+    }
     for (int step = jj_lo; step <= jj_hi; ++step) {
       const bool final_sums = step == jj_hi;
       const bool ok = wait_cta(final_sums ? accum_bar : ckpt_bar, final_sums ? 0u : (uint32_t)((step - jj_lo) & 1),
@@ -444,33 +461,46 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         continue;
       }
-      // four streams per round: a compact loop that stays in the instruction
-      // cache (fully unrolled cells of 16-stream chunks, at about 50
-      // instructions each, did not), with c_{t-1} fetched one round ahead
-      auto load_c = [&](int cb, float (&dst)[4]) {
+      // eight streams per round: a compact loop that stays in the
+      // instruction cache (fully unrolled cells of whole 16-stream chunks,
+      // at about 50 instructions each, did not) with eight independent cells
+      // per thread in flight; c_{t-1} comes from tensor memory, or for wider
+      // tiles from global memory one round ahead
+      auto load_c = [&](int cb, float (&dst)[8]) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
+        for (int e = 0; e < 8; ++e) {
           const int n = n0 + cb + e;
-          dst[e] = (write && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
+          dst[e] = (!kCTmem && write && cb < cbeg + kHalf && n < a.B) ? a.c_state[(long long)n * a.H + j] : 0.f;
         }
       };
-      float cpn[4];
+      float cpn[8];
       load_c(cbeg, cpn);
 #pragma unroll 1
-      for (int c4 = cbeg; c4 < cbeg + kHalf; c4 += 4) {
-        float cp[4] = {cpn[0], cpn[1], cpn[2], cpn[3]};  // loaded before any store of this round
-        if (c4 + 4 < cbeg + kHalf) load_c(c4 + 4, cpn);
-        float y[4][4];
-        __syncwarp();
-        tmem_ld4x4_sync(trow + c4, trow + NT + c4, trow + 2 * NT + c4, trow + 3 * NT + c4, y);
-        if (write) {
+      for (int c8 = cbeg; c8 < cbeg + kHalf; c8 += 8) {
+        float cp[8], y[4][8];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int n = n0 + c4 + e;
+        for (int e = 0; e < 8; ++e) cp[e] = cpn[e];  // loaded before any store of this round
+        load_c(c8 + 8, cpn);
+        __syncwarp();
+        if constexpr (kCTmem) {
+          tmem_ld8x5_sync(trow + c8, trow + NT + c8, trow + 2 * NT + c8, trow + 3 * NT + c8, trow + kAcc + c8, y, cp);
+        } else {
+          tmem_ld8x4_sync(trow + c8, trow + NT + c8, trow + 2 * NT + c8, trow + 3 * NT + c8, y);
+        }
+        if (write) {
+          // the eight cells first (independent chains the scheduler can
+          // interleave), then their stores
+          float hv[8], cv[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            lstm_cell_s(y[0][e] + bias[0], y[1][e] + bias[1], y[2][e] + bias[2], y[3][e] + bias[3], cp[e], hv[e],
+                        cv[e]);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int n = n0 + c8 + e;
             if (n >= a.B) break;
             const long long sj = (long long)n * a.H + j;
-            float hh, cc;
-            lstm_cell_f(y[0][e] + bias[0], y[1][e] + bias[1], y[2][e] + bias[2], y[3][e] + bias[3], cp[e], hh, cc);
+            const float hh = hv[e], cc = cv[e];
             if (!final_sums) {
               const long long o = (long long)step * a.ck_stride + sj;  // (no split: jj_lo = 0)
               if (a.ckpt_h) a.ckpt_h[o] = hh;
@@ -536,7 +566,7 @@ __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
       if (r != 0) y[g] += remainder_terms(a, g, n, j, a.ck.k[jj] - r, r);
     }
     float hh, cc;
-    lstm_cell_f(y[0], y[1], y[2], y[3], cp, hh, cc);
+    lstm_cell_s(y[0], y[1], y[2], y[3], cp, hh, cc);
     const long long o = (long long)jj * a.ck_stride + i;
     if (a.ckpt_h) a.ckpt_h[o] = hh;
     if (a.ckpt_c) a.ckpt_c[o] = cc;
@@ -549,7 +579,7 @@ __global__ void __launch_bounds__(256) tc_gates_reduce_kernel(TcGatesArgs a) {
     y[g] = v + bias[g];
   }
   float hh, cc;
-  lstm_cell_f(y[0], y[1], y[2], y[3], cp, hh, cc);
+  lstm_cell_s(y[0], y[1], y[2], y[3], cp, hh, cc);
   a.c_state[i] = cc;
   if (a.out_h) a.out_h[i] = hh;
   __nv_bfloat16 hi, lo;

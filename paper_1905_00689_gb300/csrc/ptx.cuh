@@ -179,6 +179,31 @@ __device__ __forceinline__ float tanh_f(float z) {
   return a < 0.25f ? small : big;
 }
 
+// tanh z = 2 sigmoid(2z) - 1: branch-free, absolute error about 2e-7 (the
+// cancellation near 0 costs relative accuracy there, not absolute).  For
+// the bf16 tensor-core epilogues, whose bound is 2e-2 elementwise; the fp32
+// paths use tanh_f.
+__device__ __forceinline__ float tanh_s(float z) { return fmaf(2.0f, sigmoid_f(2.0f * z), -1.0f); }
+
+// The cell update below for the bf16 tensor-core epilogues, with seven
+// special-function operations per cell instead of ten: the four gates are
+// sigmoids (the cell gate as tanh z = 2 sigmoid(2z) - 1) of denominators
+// d = 1 + e^-z, and their four reciprocals come from one reciprocal of the
+// product d0 d1 d2 d3 (1/d0 = d1 (d2 d3) / (d0 d1 d2 d3), and so on: about
+// 4 ulp).  The arguments are clamped at -20 so that the product stays
+// finite; that moves a sigmoid by at most 2.1e-9.
+__device__ __forceinline__ void lstm_cell_s(float yi, float yf, float yg, float yo, float c_prev, float& h_out,
+                                            float& c_out) {
+  const float d0 = 1.0f + __expf(-fmaxf(yi, -20.0f)), d1 = 1.0f + __expf(-fmaxf(yf, -20.0f));
+  const float d2 = 1.0f + __expf(-fmaxf(2.0f * yg, -20.0f)), d3 = 1.0f + __expf(-fmaxf(yo, -20.0f));
+  const float p01 = d0 * d1, p23 = d2 * d3;
+  const float r = rcp_approx(p01 * p23);
+  const float r01 = r * p23, r23 = r * p01;  // 1 / (d0 d1), 1 / (d2 d3)
+  const float i = r01 * d1, f = r01 * d0, g = fmaf(2.0f, r23 * d3, -1.0f), o = r23 * d2;
+  c_out = fmaf(f, c_prev, i * g);
+  h_out = o * tanh_s(c_out);
+}
+
 // Gate nonlinearities and cell update (Sec. II): i, f, o sigmoid, g tanh;
 // c = f c_prev + i g; h = o tanh(c).  Pre-activations already include bias.
 __device__ __forceinline__ void lstm_cell_f(float yi, float yf, float yg, float yo, float c_prev,
@@ -254,25 +279,53 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
-// Four loads of 32 lanes x 4 consecutive 32-bit columns (at t0 .. t3) and the
-// wait for them in one statement, so that no use of the values can be
+// Four loads of 32 lanes x 8 consecutive 32-bit columns (at t0 .. t3) and
+// the wait for them in one statement, so that no use of the values can be
 // scheduled before they have arrived: v[i][c] = column t_i + c of this
 // thread's row.
-__device__ __forceinline__ void tmem_ld4x4_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3,
-                                                float (&v)[4][4]) {
-  uint32_t r[16];
+__device__ __forceinline__ void tmem_ld8x4_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3,
+                                                float (&v)[4][8]) {
+  uint32_t r[32];
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%16];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4, %5, %6, %7}, [%17];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%8, %9, %10, %11}, [%18];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%12, %13, %14, %15}, [%19];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%32];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%8, %9, %10, %11, %12, %13, %14, %15}, [%33];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%16, %17, %18, %19, %20, %21, %22, %23}, [%34];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%24, %25, %26, %27, %28, %29, %30, %31}, [%35];\n\t"
       "tcgen05.wait::ld.sync.aligned;"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(t0), "r"(t1), "r"(t2), "r"(t3)
       : "memory");
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i >> 2][i & 3] = __uint_as_float(r[i]);
+  for (int i = 0; i < 32; ++i) v[i >> 3][i & 7] = __uint_as_float(r[i]);
+}
+
+// Five loads of 32 lanes x 8 consecutive 32-bit columns (at t0 .. t4) and
+// the wait for them in one statement: v[i][c] = column t_i + c of this
+// thread's row (i < 4), w[c] = column t4 + c.
+__device__ __forceinline__ void tmem_ld8x5_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, uint32_t t4,
+                                                float (&v)[4][8], float (&w)[8]) {
+  uint32_t r[40];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%40];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%8, %9, %10, %11, %12, %13, %14, %15}, [%41];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%16, %17, %18, %19, %20, %21, %22, %23}, [%42];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%24, %25, %26, %27, %28, %29, %30, %31}, [%43];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%32, %33, %34, %35, %36, %37, %38, %39}, [%44];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39])
+      : "r"(t0), "r"(t1), "r"(t2), "r"(t3), "r"(t4)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i >> 3][i & 7] = __uint_as_float(r[i]);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) w[i] = __uint_as_float(r[32 + i]);
 }
 
 // Two tmem_ld16 and one wait for both in one statement, so that no use of
