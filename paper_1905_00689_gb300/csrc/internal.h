@@ -50,6 +50,7 @@ struct LayerStore {
   std::vector<int> xoff_h[4];
   bool maps_ready = false;  // tensor maps of Vx, Vh, U (bf16 path), built on first use
   TcMap map_vx, map_vh, map_u;
+  TcMap map_vx_p[3], map_vh_p[3];  // the same with boxes of 8, 16, 32 rows (packed gates)
 };
 
 struct Timing {
@@ -235,6 +236,8 @@ struct TcRowsArgs {
   int Kdim;          // reduction length (D of the layer, or H)
   int K, Ks;         // refinement depth of the run; gate stride of the packed rows
   int kt_per_gate;   // 128-row tiles per gate: ceil(K / 128)
+  int rpg;           // 0, or packed gates (K <= rpg, rpg 8, 16 or 32): one tile of the four gates'
+                     // first rpg rows, whose factor map has boxes of rpg rows
   int N;             // valid columns (T*B for the projection, B for tau')
   int b_plane;       // rows of one plane of the activation's map (its lo plane starts there)
   int mode;          // 0: P[n][row] = sum; 1: tau[n][row] = pair of sigma[row] (sum + P[n][row]), 0 for k >= K

@@ -129,6 +129,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.x / a.kt_per_gate, kt = blockIdx.x % a.kt_per_gate;
   const int row0 = g * a.Ks + kt * kTileM;
+  // packed gates (a.rpg > 0, K <= rpg <= 32): the tile's rows are the first
+  // rpg terms of each gate, gate g at tile rows [g rpg, (g + 1) rpg), loaded
+  // by four copies of rpg rows; tile rows from 4 rpg on stay zero
+  const int rpg = a.rpg;
+  const uint32_t a_bytes = rpg > 0 ? 4u * rpg * kTileK * 2 : kABytes;
   const int col0 = blockIdx.y * BN;
   const int nkb = (a.Kdim + kTileK - 1) / kTileK;
   const volatile int* err = a.err;
@@ -145,6 +150,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     mbar_init(drain_bar, 1);
     fence_mbarrier_init_cluster();
   }
+  if (rpg > 0) {  // the factor tile's rows no copy writes: zero in every stage, before the MMAs read them
+    const uint32_t zbytes = kABytes - a_bytes;
+    for (uint32_t i = threadIdx.x; i < S * (zbytes / 16); i += blockDim.x) {
+      const uint32_t st = i / (zbytes / 16), o = i % (zbytes / 16);
+      *reinterpret_cast<uint4*>(smem_raw + (base - raw) + st * kStage + a_bytes + 16 * o) = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_shared();
+  }
   if (warp == 2) {
     tmem_alloc(smem_u32(tmem_slot), kCols);
     tmem_relinquish();
@@ -153,6 +166,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the factor copies of one stage into the tile at st
+  auto load_a = [&](uint32_t st, uint32_t bar, int kb) {
+    if (rpg == 0) {
+      tma_load_2d(st, &tma, bar, kb * kTileK, row0);
+    } else {
+#pragma unroll
+      for (int gg = 0; gg < 4; ++gg) tma_load_2d(st + gg * rpg * kTileK * 2, &tma, bar, kb * kTileK, gg * a.Ks);
+    }
+  };
 
   if (warp == 0 && lane == 0) {  // ---- TMA producer ----
     tma_prefetch_map(&tma);
@@ -163,8 +185,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // before this one: issue them before waiting for it
     const int npre = nkb < S ? nkb : S;
     for (int kb = 0; kb < npre; ++kb) {
-      mbar_arrive_expect_tx(bar0 + 8u * kb, kStage);
-      tma_load_2d(base + kb * kStage, &tma, bar0 + 8u * kb, kb * kTileK, row0);
+      mbar_arrive_expect_tx(bar0 + 8u * kb, a_bytes + 2 * kBBytes);
+      load_a(base + kb * kStage, bar0 + 8u * kb, kb);
     }
     griddep_wait();
     for (int kb = 0; kb < nkb; ++kb) {
@@ -172,8 +194,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
       const uint32_t st = base + s * kStage;
       if (kb >= npre) {
-        mbar_arrive_expect_tx(bar0 + 8u * s, kStage);
-        tma_load_2d(st, &tma, bar0 + 8u * s, kb * kTileK, row0);
+        mbar_arrive_expect_tx(bar0 + 8u * s, a_bytes + 2 * kBBytes);
+        load_a(st, bar0 + 8u * s, kb);
       }
       tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);                      // hi plane
       tma_load_2d(st + kABytes + kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, a.b_plane + col0);  // lo plane
@@ -211,9 +233,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     constexpr int kHalf = BN / 2;
     const int cbeg = (ep >> 2) * kHalf;
     const int lrow = 32 * q + lane;
-    const int k = kt * kTileM + lrow;
-    const int row = row0 + lrow;
-    const bool row_ok = k < a.K;
+    const int k = rpg > 0 ? lrow % rpg : kt * kTileM + lrow;
+    const int row = rpg > 0 ? (lrow / rpg) * a.Ks + k : row0 + lrow;
+    const bool row_ok = k < a.K && (rpg == 0 || lrow < 4 * rpg);
     const uint32_t trow = tmem + ((32u * q) << 16);
     float preg[kHalf];  // P_t of this thread's row and columns, loaded while the mainloop runs
     if (add_p) {
@@ -241,7 +263,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (n >= a.N) break;
         if (!add_p) {
           if (row_ok) a.P[(long long)n * a.ldp + row] = v[j];
-        } else {
+        } else if (rpg == 0 || lrow < 4 * rpg) {
           __nv_bfloat16 hi, lo;
           bf16_pair(row_ok ? sig * (v[j] + preg[cc + j]) : 0.f, hi, lo);
           a.tau[(long long)n * a.ldt + row] = hi;
@@ -704,7 +726,7 @@ cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, 
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  return launch_pdl(kern, dim3(4 * a.kt_per_gate, (n_cols + BN - 1) / BN), smem, s,
+  return launch_pdl(kern, dim3(a.rpg > 0 ? 1 : 4 * a.kt_per_gate, (n_cols + BN - 1) / BN), smem, s,
                     *reinterpret_cast<const CUtensorMap*>(A.bytes), *reinterpret_cast<const CUtensorMap*>(Bm.bytes),
                     a);
 }
@@ -775,6 +797,7 @@ int tc_gates_tile_n(int H, int B) {
 cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s) {
   switch (bn) {
     case 128: return launch_rows_t<128, 4>(A, Bm, a, n_cols, s);
+    case 32: return launch_rows_t<32, 8>(A, Bm, a, n_cols, s);
     default: return launch_rows_t<64, 6>(A, Bm, a, n_cols, s);
   }
 }

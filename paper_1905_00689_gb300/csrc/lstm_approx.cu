@@ -238,9 +238,13 @@ struct TensorTiles {
 // GEMM (bnh) and of the gate GEMM (nt), and the gate GEMM's term-axis
 // splits (ks, of nkb_per 64-term chunks each; small grids split the terms
 // over more CTAs).
+// Rows per gate of the packed factor tile (0: one 128-row tile per gate).
+int tensor_rows_per_gate(int K) { return K <= 8 ? 8 : K <= 16 ? 16 : K <= 32 ? 32 : 0; }
+
 TensorTiles tensor_tiles(int H, int B, int K, const Checkpoints& ck) {
   TensorTiles t;
-  t.bnh = tc_rows_tile_n(B, 4 * ((K + 127) / 128));
+  // packed gates: one row tile, so narrower stream tiles keep more SMs busy
+  t.bnh = tensor_rows_per_gate(K) > 0 ? 32 : tc_rows_tile_n(B, 4 * ((K + 127) / 128));
   t.nt = tc_gates_tile_n(H, B);
   const int gate_tiles = ((H + 127) / 128) * ((B + t.nt - 1) / t.nt);
   t.ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &t.nkb_per);
@@ -257,6 +261,10 @@ int ensure_factor_maps(lstm_approx_t* h, int l) {
       !tc_make_map(&s.map_vh, s.Vh, h->H, rows, (uint64_t)h->ldh * 2, 128) ||
       !tc_make_map(&s.map_u, s.U, h->Ks, 4ull * h->H, (uint64_t)h->Ks * 2, 128))
     return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for layer %d factors", l);
+  for (int i = 0; i < 3; ++i)
+    if (!tc_make_map(&s.map_vx_p[i], s.Vx, s.D, rows, (uint64_t)s.ldx * 2, 8u << i) ||
+        !tc_make_map(&s.map_vh_p[i], s.Vh, h->H, rows, (uint64_t)h->ldh * 2, 8u << i))
+      return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for layer %d factors", l);
   s.maps_ready = true;
   return LSTM_APPROX_OK;
 }
@@ -273,6 +281,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   if (rc) return rc;
   const bool top = l == h->L - 1;
   const long long limit_ns = h->opt_wait_limit_us * 1000LL;
+  // up to 32 terms the products take one tile of all four gates' rows
+  const int rpg = tensor_rows_per_gate(K);
+  const int pi = rpg == 8 ? 0 : (rpg == 16 ? 1 : 2);
   __nv_bfloat16* in_bf16;
   int ld_in;
   if (l == 0) {  // operand conversion (outside the timed projection phase)
@@ -288,7 +299,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   {
     PhaseTimer pt(h, 0);
     const int kt = (K + 127) / 128;
-    const int bnx = tc_rows_tile_n(TB, 4 * kt);
+    const int bnx = tc_rows_tile_n(TB, rpg > 0 ? 1 : 4 * kt);
     TcMap mx;
     if (!tc_make_map(&mx, in_bf16, D, 2ull * TB, (uint64_t)ld_in * 2, bnx))
       return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
@@ -297,6 +308,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.K = K;
     ra.Ks = h->Ks;
     ra.kt_per_gate = (K + 127) / 128;
+    ra.rpg = rpg;
     ra.N = TB;
     ra.b_plane = TB;
     ra.mode = 0;
@@ -304,7 +316,8 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.ldp = (int)ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(s.map_vx, mx, ra, TB, bnx, h->stream), "input projection launch");
+    LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vx_p[pi] : s.map_vx, mx, ra, TB, bnx, h->stream),
+            "input projection launch");
     h->launches += 1;
   }
   PhaseTimer pt(h, 1);
@@ -313,6 +326,10 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
   LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
   h->launches += 1;
+  // packed gates write only the first rpg terms of each gate's tau' rows; the
+  // gate GEMM reads 64-term chunks, so the rest of the pair must be zero
+  if (rpg > 0)
+    LA_CUDA(h, cudaMemsetAsync(tau, 0, 2ull * B * 4 * h->Ks * sizeof(__nv_bfloat16), h->stream), "tau' clear");
   const TensorTiles tt = tensor_tiles(H, B, K, ck);
   const int bnh = tt.bnh, nt = tt.nt, ks = tt.ks, nkb_per = tt.nkb_per;
   if (tt.raw) {
@@ -337,6 +354,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.K = K;
     ra.Ks = h->Ks;
     ra.kt_per_gate = (K + 127) / 128;
+    ra.rpg = rpg;
     ra.N = B;
     ra.b_plane = B;
     ra.mode = 1;
@@ -348,7 +366,8 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.tau_plane = (long long)B * ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(s.map_vh, mh, ra, B, bnh, h->stream), "recurrent projection launch");
+    LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vh_p[pi] : s.map_vh, mh, ra, B, bnh, h->stream),
+            "recurrent projection launch");
     TcGatesArgs ga{};
     ga.H = H;
     ga.K = K;

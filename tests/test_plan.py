@@ -135,15 +135,16 @@ def test_every_plan_covers_its_shape_and_fits(H, K, cs, variant):
 @pytest.mark.parametrize("K", [8, 64, 256, 1024])
 def test_tensor_tiles(H, B, K):
     """Stream tiles: the narrowest of 32/64/128 (gates) that keeps the grid
-    within one wave of 148 CTAs, else the widest; tau' takes 64 streams when
-    that keeps one wave, else 128; the gate GEMM's terms split over
-    min(148 // tiles, 8, chunks of 64) CTAs."""
+    within one wave of 148 CTAs, else the widest; tau' takes 32 streams up to
+    K = 32 (one tile of all four gates' rows), else 64 when that keeps one
+    wave, else 128; the gate GEMM's terms split over min(148 // tiles, 8,
+    chunks of 64) CTAs."""
     p = plan(BF16, H, 2, B, K)
     units = -(-H // 128)
     nt = next((n for n in (32, 64, 128) if units * -(-B // n) <= 148), 128)
     assert p["gate_tile_streams"] == nt
     rows = 4 * -(-K // 128)
-    bn = 64 if rows * -(-B // 64) <= 148 else 128
+    bn = 32 if K <= 32 else (64 if rows * -(-B // 64) <= 148 else 128)
     assert p["tau_tile_streams"] == bn
     tiles = units * -(-B // nt)
     chunks = -(-K // 64)
