@@ -65,3 +65,38 @@ def test_dist_env_defaults(monkeypatch):
     monkeypatch.setenv("RANK", "3")
     monkeypatch.setenv("LOCAL_RANK", "1")
     assert bench._dist_env() == (4, 3, 1)
+
+
+def _shard_main(rank, world, port, out):
+    import numpy as np
+    import oracle
+    from workloads import draw_factor_set, draw_inputs, rounded_factors
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world)
+    try:
+        D, H, T, B, K = 12, 16, 4, 6, 8
+        gates = rounded_factors([draw_factor_set(H, D + H, K, 10, 8800 + g) for g in range(4)], "bf16")
+        x = draw_inputs(T, B, D, "uniform", 88)
+        lo, hi = rank * B // world, (rank + 1) * B // world   # this rank's streams
+        mine = oracle.run_lstm([gates], x[:, lo:hi], K, checkpoints=[3, K])
+        parts = [None] * world
+        dist.all_gather_object(parts, (lo, hi, mine["h"], mine["ckpt_h"]))
+        if rank == 0:
+            full = oracle.run_lstm([gates], x, K, checkpoints=[3, K])
+            h = np.concatenate([p[2] for p in parts], axis=1)
+            ck = np.concatenate([p[3] for p in parts], axis=2)
+            out["ok"] = (np.allclose(h, full["h"], rtol=0, atol=1e-13) and
+                         np.allclose(ck, full["ckpt_h"], rtol=0, atol=1e-13) and
+                         [p[:2] for p in parts] == [(r * B // world, (r + 1) * B // world) for r in range(world)])
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world", [2, 3])
+def test_streams_split_across_ranks_concatenate_to_the_whole_batch(world):
+    """Large-batch sharding: each rank runs its B/G streams with the same
+    factors and no collective on the data path; concatenating the ranks'
+    outputs along the stream axis gives the whole batch's outputs (streams
+    are independent).  Checked on the oracle with gloo ranks."""
+    out = mp.Manager().dict()
+    mp.start_processes(_shard_main, args=(world, _free_port(), out), nprocs=world, join=True, start_method="spawn")
+    assert out["ok"]
