@@ -21,7 +21,12 @@ Readings where the paper is silent:
 * the triplet's sign is fixed so that v's largest-magnitude entry (lowest
   index among ties) is positive -- sigma u v^T and the mask do not depend on
   it;
-* the top triplet is taken from LAPACK's full SVD (numpy.linalg.svd, fp64).
+* the top triplet is taken from LAPACK's full SVD (numpy.linalg.svd, fp64)
+  when min(R, C) <= 512, and from ARPACK's implicitly restarted Lanczos
+  iteration for the largest singular value (scipy.sparse.linalg.svds,
+  k = 1, tolerance 1e-13) above that, where a full SVD per refinement step
+  takes minutes; both give the same sigma u v^T up to the accuracy of the
+  iteration (pinned against each other in the tests).
 """
 from __future__ import annotations
 
@@ -45,10 +50,29 @@ def prune(v: np.ndarray, nz: int):
     return kept.astype(np.int32), v[kept].copy()
 
 
-def top_triplet(R: np.ndarray):
-    """Top singular triplet (sigma, u, v) of R, with ||u|| = ||v|| = 1."""
-    U, s, Vt = np.linalg.svd(R, full_matrices=False)
-    sigma, u, v = float(s[0]), U[:, 0].copy(), Vt[0].copy()
+LANCZOS_ABOVE = 512  # min(R, C) above which the top triplet comes from the Lanczos iteration
+
+
+def top_triplet(R: np.ndarray, method: str = "auto"):
+    """Top singular triplet (sigma, u, v) of R, with ||u|| = ||v|| = 1.
+
+    method: "svd" (LAPACK, full SVD), "lanczos" (ARPACK, largest singular
+    value only) or "auto" (Lanczos when min(R.shape) > LANCZOS_ABOVE)."""
+    if method == "auto":
+        method = "lanczos" if min(R.shape) > LANCZOS_ABOVE else "svd"
+    if method == "svd":
+        U, s, Vt = np.linalg.svd(R, full_matrices=False)
+        sigma, u, v = float(s[0]), U[:, 0].copy(), Vt[0].copy()
+    elif method == "lanczos":
+        from scipy.sparse.linalg import svds
+        # a fixed start vector keeps the result reproducible run to run
+        v0 = np.ones(min(R.shape)) / np.sqrt(min(R.shape))
+        U, s, Vt = svds(R, k=1, tol=1e-13, v0=v0, solver="arpack")
+        sigma, u, v = float(s[0]), U[:, 0].copy(), Vt[0].copy()
+        nu, nv = np.linalg.norm(u), np.linalg.norm(v)
+        u, v = u / nu, v / nv
+    else:
+        raise ValueError(method)
     a = np.abs(v)
     lead = int(np.flatnonzero(a == a.max())[0])
     if v[lead] < 0:
@@ -56,11 +80,13 @@ def top_triplet(R: np.ndarray):
     return sigma, u, v
 
 
-def decompose_gate(W: np.ndarray, K: int, nz: int, return_residual_norms: bool = False) -> dict:
+def decompose_gate(W: np.ndarray, K: int, nz: int, return_residual_norms: bool = False,
+                   method: str = "auto") -> dict:
     """K residual refinement steps of Eq. 1 for one gate matrix W (R x C).
 
     Returns {"sigma": [K], "u": [K][R], "idx": [K][nz], "val": [K][nz]} and,
-    if asked, "resid_fro2": ||R^(n)||_F^2 for n = 1..K+1.
+    if asked, "resid_fro2": ||R^(n)||_F^2 for n = 1..K+1.  method selects the
+    top-triplet routine (see top_triplet).
     """
     W = np.asarray(W, dtype=np.float64)
     R_rows, C = W.shape
@@ -73,7 +99,7 @@ def decompose_gate(W: np.ndarray, K: int, nz: int, return_residual_norms: bool =
     for n in range(K):
         residual = W - W_tilde          # R^(n) = W - W~^(n-1)
         fro2.append(float(np.sum(residual * residual)))
-        s_n, u_n, v_n = top_triplet(residual)
+        s_n, u_n, v_n = top_triplet(residual, method)
         i_n, p_n = prune(v_n, nz)       # prune(v^(n), NZ); u is not pruned
         v_pruned = np.zeros(C)
         v_pruned[i_n] = p_n

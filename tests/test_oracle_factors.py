@@ -12,6 +12,7 @@ Each test fixes a property that a plausible mistake would break:
 import numpy as np
 import pytest
 
+import oracle
 from oracle import factors as F
 from workloads import draw_weight, nz_from_keep
 
@@ -173,3 +174,42 @@ def test_pruned_u_keeps_the_largest_entries():
     for n in range(3):
         assert np.count_nonzero(f["u"][n]) == 4
     np.testing.assert_array_equal(prune_dense(np.array([0.1, -3.0, 2.0, 2.0]), 2), [0.0, -3.0, 2.0, 0.0])
+
+
+# ---- the Lanczos route for large gate matrices ----------------------------
+
+def test_lanczos_top_triplet_equals_lapack():
+    """ARPACK's largest singular triplet equals LAPACK's full SVD (two
+    independent library routines) on a Gaussian matrix above the size limit
+    and on a residual after three pruned refinement steps."""
+    from oracle.factors import LANCZOS_ABOVE, top_triplet
+    rng = np.random.default_rng(31)
+    R = rng.standard_normal((LANCZOS_ABOVE + 8, 3 * LANCZOS_ABOVE)) / np.sqrt(3 * LANCZOS_ABOVE)
+    f = oracle.decompose_gate(R, 3, 700, method="svd")
+    residual = R - oracle.reconstruct(f, 3, R.shape[1])
+    for M in (R, residual):
+        a = top_triplet(M, "svd")
+        b = top_triplet(M, "lanczos")
+        assert abs(a[0] - b[0]) <= 1e-12 * a[0]
+        assert np.abs(a[0] * np.outer(a[1], a[2]) - b[0] * np.outer(b[1], b[2])).max() <= 1e-12
+        # same sign convention: v's largest-magnitude entry positive
+        assert np.array_equal(np.sign(a[2]), np.sign(b[2]))
+        assert abs(np.linalg.norm(b[1]) - 1) < 1e-14 and abs(np.linalg.norm(b[2]) - 1) < 1e-14
+    assert top_triplet(R)[0] == top_triplet(R, "lanczos")[0]  # the automatic choice above the limit
+
+
+def test_lanczos_decomposition_matches_lapack_and_keeps_the_frobenius_law():
+    from oracle.factors import LANCZOS_ABOVE
+    rng = np.random.default_rng(32)
+    H, C, K, nz = LANCZOS_ABOVE + 4, 1100, 6, 300
+    W = rng.standard_normal((H, C)) / np.sqrt(C)
+    a = oracle.decompose_gate(W, K, nz, method="svd")
+    b = oracle.decompose_gate(W, K, nz, return_residual_norms=True)  # automatic: Lanczos
+    assert np.array_equal(a["idx"], b["idx"])
+    np.testing.assert_allclose(b["sigma"], a["sigma"], rtol=1e-11)
+    np.testing.assert_allclose(b["u"], a["u"], atol=1e-10)
+    np.testing.assert_allclose(b["val"], a["val"], atol=1e-10)
+    # ||R^(n+1)||^2 = ||R^(n)||^2 - sigma_n^2 ||v'_n||^2 (exact for any accurate triplet)
+    f2 = b["resid_fro2"]
+    drop = b["sigma"] ** 2 * np.sum(b["val"] ** 2, axis=1)
+    np.testing.assert_allclose(f2[:-1] - f2[1:], drop, rtol=1e-9)

@@ -172,3 +172,32 @@ def test_two_layer_simt_forced_unaligned_depths(cuda_device):
     assert m.query(Q_LAST_PATH) == PATH_SIMT
     ref = oracle_run(layers, x, K, dtype="bf16", checkpoints=[5, K])
     assert_parity(got, ref, BF16_TOL)
+
+
+def test_large_batch_workload_decomposed_factors(cuda_device):
+    """D=2048, H=1024, T=64, B=1024, keep 50%, with the oracle's own residual
+    decomposition of the workload's Gaussian gate matrices (K = 16, the top
+    triplets by the Lanczos iteration) and depths 5 and 16: sampled streams."""
+    w = WORKLOADS["c4"]
+    layers = [list(decomposed_layer("c4", 0, 16, 0.5))]
+    x = workload_inputs(w)
+    cps = [5, 16]
+    got, m = run_gpu(layers, x, 16, dtype="bf16", checkpoints=cps)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    streams = [0, 700, 1023]
+    ref = oracle_run(layers, x[:, streams], 16, dtype="bf16", checkpoints=cps)
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+def test_two_layer_workload_decomposed_factors(cuda_device):
+    """The two-layer D=4096, H=2048, T=16, B=64 workload (keep 30%) with the
+    oracle's decomposition of both layers' gate matrices (K = 8) and depths
+    3 and 8: sampled streams."""
+    w = WORKLOADS["c5"]
+    layers = [list(decomposed_layer("c5", l, 8, 0.3)) for l in range(2)]
+    x = workload_inputs(w)
+    cps = [3, 8]
+    got, _ = run_gpu(layers, x, 8, dtype="bf16", checkpoints=cps)
+    streams = [2, 41]
+    ref = oracle_run(layers, x[:, streams], 8, dtype="bf16", checkpoints=cps)
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
