@@ -378,6 +378,7 @@ def run_ours(args):
     dense = None if args.quick else dense_comparator(dev, stream, x)
     dense_kernel = None if args.quick else dense_kernel_comparator(dev, stream, flush, x, statistics.median(step_ms))
     k_sweeps = [] if (args.quick or args.no_large) else workload_k_sweeps(dev, flush)
+    tau_layouts = [] if (args.quick or args.no_large) else tau_layout_comparison(dev, stream)
 
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
@@ -429,6 +430,7 @@ def run_ours(args):
             "gpu_launches": launches, "sweep": sweep, "clocks": clocks,
             "large_batch": large,
             "k_sweeps": k_sweeps,
+            "tau_layouts": tau_layouts,
             "paper_case_study": paper_case,
             "dense_lstm_comparator": dense,
             "dense_kernel_comparator": dense_kernel,
@@ -600,6 +602,44 @@ def dense_comparator(dev, stream, x, steps: int = 200) -> dict:
             "dense_weight_bytes": 4 * 4 * WL.H * (D + WL.H)}
 
 
+def tau_layout_comparison(dev, stream) -> list:
+    """The tensor path's recurrent projection with masked-dense v rows on the
+    tensor cores against v's kept entries (compressed rows) on the CUDA cores
+    (LSTM_APPROX_OPT_TAU_LAYOUT), D=2048 H=1024 T=64 B=1024 at both keep
+    levels: recurrence milliseconds per run (CUDA events on the library's
+    stream, median of 5) and per timestep."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, OPT_TAU_LAYOUT, OPT_TIMING
+    w = WORKLOADS["c4"]
+    x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+    oh = torch.empty((w.T, w.B, w.H), device=dev)
+    out = []
+    for keep in (0.1, 0.5):
+        m = LSTMApprox(1, [w.D], w.H, 512, w.B, "bf16", stream=stream)
+        m.set_layer(0, synthetic_layer_factors(w, 0, 512, keep))
+        for K in (128, 512):
+            row = {"workload": w.name, "keep": keep, "K": K}
+            for layout, name in ((0, "masked_dense_tensor"), (1, "compressed_cuda_cores")):
+                m.set_option(OPT_TAU_LAYOUT, layout)
+                for _ in range(2):
+                    m.run(x, K, oh)
+                m.set_option(OPT_TIMING, 1)
+                rec = []
+                for _ in range(5):
+                    m.run(x, K, oh)
+                    rec.append(m.phase_times()[1])
+                m.set_option(OPT_TIMING, 0)
+                ms = statistics.median(rec)
+                row[name] = {"recurrence_ms": ms, "us_per_timestep": 1e3 * ms / w.T}
+            row["faster"] = min(("masked_dense_tensor", "compressed_cuda_cores"),
+                                key=lambda k: row[k]["recurrence_ms"])
+            out.append(row)
+        m.set_option(OPT_TAU_LAYOUT, 0)
+        m.close()
+        torch.cuda.empty_cache()
+    return out
+
+
 def dense_kernel_comparator(dev, stream, flush, x, approx_ms: float) -> list:
     """The library's dense LSTM kernel (lstm_approx_dense_run: the full gate
     matrices of Sec. II on the same persistent cluster design) timed like the
@@ -737,6 +777,9 @@ def run_profile(args):
     m = LSTMApprox(w.L, [w.D] + [w.H] * (w.L - 1), w.H, K, w.B, w.dtype)
     for l in range(w.L):
         m.set_layer(l, synthetic_layer_factors(w, l, K, keep))
+    if args.profile_tau_compressed:
+        from paper_1905_00689_gb300 import OPT_TAU_LAYOUT
+        m.set_option(OPT_TAU_LAYOUT, 1)
     x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
     oh = torch.empty((w.T, w.B, w.H), device=dev)
     ck = torch.empty((max(1, len(cps)), w.T, w.B, w.H), device=dev)
@@ -761,6 +804,8 @@ def main():
                     help="only run one workload's path (warmup + steps runs), for profilers")
     ap.add_argument("--profile-k", type=int, default=0, help="with --profile: this K instead of the workload's largest")
     ap.add_argument("--profile-keep", type=float, default=0.0, help="with --profile: this keep fraction")
+    ap.add_argument("--profile-tau-compressed", action="store_true",
+                    help="with --profile (bf16 workloads): the compressed layout of v's h part for tau'")
     ap.add_argument("--profile-dense", action="store_true",
                     help="with --profile: the dense comparator kernel on the workload's shape (fp32, one layer)")
     ap.add_argument("--quick", action="store_true",

@@ -278,10 +278,15 @@ enum lstm_approx_option_key {
                                        exchanges per timestep, any H <= 1024),
                                        2 = one-exchange kernel (H <= 512,
                                        K <= 256, cluster of 4, 8 or 16) */
-  LSTM_APPROX_OPT_XPROJ = 6 /* input projection of the small-batch fp32 path
+  LSTM_APPROX_OPT_XPROJ = 6, /* input projection of the small-batch fp32 path
                                (T*B <= 32): 0 = automatic (compressed when v
                                keeps at most 1/8 of the x columns), 1 =
                                masked-dense rows, 2 = compressed rows */
+  LSTM_APPROX_OPT_TAU_LAYOUT = 7 /* the tensor path's recurrent projection tau'
+                               (bf16 factors): 0 = masked-dense v rows on the
+                               tensor cores (default: faster at every shape
+                               measured), 1 = v's kept h entries (compressed
+                               rows) on the CUDA cores, H <= 1280 */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 

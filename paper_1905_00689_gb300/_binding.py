@@ -21,7 +21,8 @@ OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, ESTATE = range(6)
 FP32, BF16 = 0, 1
 Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT = range(5)
 PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
-OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ = range(7)
+(OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ,
+ OPT_TAU_LAYOUT) = range(8)
 (PLAN_PATH, PLAN_PERSISTENT_VARIANT, PLAN_CLUSTER, PLAN_TERMS_PER_CTA, PLAN_UNITS_PER_WARP, PLAN_TERMS_PER_LANE,
  PLAN_VH_LAYOUT, PLAN_H_QUADS, PLAN_SMEM_BYTES, PLAN_TMEM_COLUMNS, PLAN_TAU_TILE_STREAMS, PLAN_GATE_TILE_STREAMS,
  PLAN_GATE_SPLITS, PLAN_ITEMS) = range(14)

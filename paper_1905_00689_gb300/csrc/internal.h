@@ -51,6 +51,14 @@ struct LayerStore {
   bool maps_ready = false;  // tensor maps of Vx, Vh, U (bf16 path), built on first use
   TcMap map_vx, map_vh, map_u;
   TcMap map_vx_p[3], map_vh_p[3];  // the same with boxes of 8, 16, 32 rows (packed gates)
+  // compressed recurrent part of v (bf16 factors): CSR over storage rows g*Ks + k
+  int* hoff = nullptr;
+  int* hcol = nullptr;
+  float* hval = nullptr;
+  size_t hcap = 0;                 // entries allocated
+  std::vector<int> hrows[4];       // per gate: host copy of its rows' kept h columns, counts per row
+  std::vector<float> hvals[4];
+  std::vector<int> hcount[4];
 };
 
 struct Timing {
@@ -91,6 +99,7 @@ struct lstm_approx {
   // options and counters
   int opt_force_path = 0, opt_cluster = 0, opt_persistent_variant = 0;
   int opt_xproj = 0;  // 0 automatic, 1 masked-dense, 2 compressed (fp32, T*B <= 32)
+  int opt_tau_layout = 0;  // tensor path's tau': 0 masked-dense (tensor cores), 1 compressed (CUDA cores)
   long long opt_wait_limit_us = 2000000;
   int opt_test_stall = 0;
   long long launches = 0;
@@ -290,6 +299,28 @@ cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs&
 // Term-axis splits for a gate GEMM of `tiles` CTAs over nkb 64-term chunks
 // (1: no split); *nkb_per receives the chunks per split.
 int tc_gates_splits(int tiles, int nkb, int* nkb_per);
+
+// Compressed tau' (the recurrent part of the pruned v as (column, value)
+// entries per storage row g*Ks + k, entries off[row] .. off[row + 1]) on the
+// CUDA cores, for the tensor path; H <= tau_sparse_max_h().
+struct TauSparseArgs {
+  const int* off;
+  const int* col;            // h column of each entry
+  const float* val;          // the entry (the bf16-stored value, widened)
+  const float* sigma;        // [4][Ks]
+  const float* P;            // [B][ldp] P_t
+  int ldp;
+  const __nv_bfloat16* h;    // pair planes [2][B][ldh] of h_{t-1}
+  int ldh;
+  long long h_plane;
+  __nv_bfloat16* tau;        // pair planes [2][B][ldt]
+  int ldt;
+  long long tau_plane;
+  int H, K, Ks, B;
+  int Rp;                    // K rounded up to 64: rows [K, Rp) of each gate store zero
+};
+cudaError_t launch_tau_sparse(const TauSparseArgs& a, cudaStream_t s);
+int tau_sparse_max_h();
 
 cudaError_t launch_to_bf16(const float* x, int N, int D, __nv_bfloat16* out, int ld, cudaStream_t s);
 cudaError_t launch_tc_init_state(const float* h0, const float* c0, int B, int H, __nv_bfloat16* h_bf16, int ldh,

@@ -366,8 +366,30 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.tau_plane = (long long)B * ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vh_p[pi] : s.map_vh, mh, ra, B, bnh, h->stream),
-            "recurrent projection launch");
+    if (h->opt_tau_layout == 1) {  // compressed rows of v's h part on the CUDA cores
+      TauSparseArgs sa{};
+      sa.off = s.hoff;
+      sa.col = s.hcol;
+      sa.val = s.hval;
+      sa.sigma = s.sigma;
+      sa.P = ra.P;
+      sa.ldp = (int)ldp;
+      sa.h = hb;
+      sa.ldh = h->ldh;
+      sa.h_plane = (long long)B * h->ldh;
+      sa.tau = tau;
+      sa.ldt = (int)ldp;
+      sa.tau_plane = (long long)B * ldp;
+      sa.H = H;
+      sa.K = K;
+      sa.Ks = h->Ks;
+      sa.B = B;
+      sa.Rp = (K + 63) / 64 * 64;
+      LA_CUDA(h, launch_tau_sparse(sa, h->stream), "recurrent projection launch");
+    } else {
+      LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vh_p[pi] : s.map_vh, mh, ra, B, bnh, h->stream),
+              "recurrent projection launch");
+    }
     TcGatesArgs ga{};
     ga.H = H;
     ga.K = K;
@@ -705,6 +727,62 @@ int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz
           cudaMemcpy(s.mask + row0 * s.mask_words, mask.data(), mask.size() * sizeof(uint32_t),
                      cudaMemcpyHostToDevice),
           "factor upload");
+  if (bf16) {  // the h part again, compressed, for the compressed tau' layout of the tensor path
+    std::vector<int>& cols = s.hrows[gate];
+    std::vector<float>& vals = s.hvals[gate];
+    std::vector<int>& cnt = s.hcount[gate];
+    cols.clear();
+    vals.clear();
+    cnt.assign(K, 0);
+    for (int k = 0; k < K; ++k)
+      for (int m = 0; m < nz; ++m) {
+        const int c = v_idx[(size_t)k * nz + m];
+        if (c < D) continue;
+        const uint32_t bits = static_cast<uint32_t>(to_bf16_bits(v_val[(size_t)k * nz + m])) << 16;
+        float f;
+        std::memcpy(&f, &bits, 4);
+        cols.push_back(c - D);
+        vals.push_back(f);
+        ++cnt[k];
+      }
+    // CSR over the storage rows g*Ks + k of all four gates (rows not set: empty)
+    std::vector<int> off(4 * (size_t)Ks + 1, 0), allc;
+    std::vector<float> allv;
+    for (int g = 0; g < 4; ++g) {
+      size_t e = 0;
+      for (int k = 0; k < Ks; ++k) {
+        const int row = g * Ks + k;
+        const int c = k < (int)s.hcount[g].size() ? s.hcount[g][k] : 0;
+        for (int i = 0; i < c; ++i) {
+          allc.push_back(s.hrows[g][e + i]);
+          allv.push_back(s.hvals[g][e + i]);
+        }
+        e += c;
+        off[row + 1] = (int)allc.size();
+      }
+    }
+    const size_t n = allc.empty() ? 1 : allc.size();
+    if (s.hoff == nullptr) {
+      int rc = dmalloc(h, reinterpret_cast<void**>(&s.hoff), off.size() * 4, "compressed factor storage");
+      if (rc) return rc;
+    }
+    if (n > s.hcap) {
+      dfree(h, s.hcol, s.hcap * 4);
+      dfree(h, s.hval, s.hcap * 4);
+      s.hcol = nullptr;
+      s.hval = nullptr;
+      s.hcap = 0;
+      int rc = dmalloc(h, reinterpret_cast<void**>(&s.hcol), n * 4, "compressed factor storage");
+      if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.hval), n * 4, "compressed factor storage");
+      if (rc) return rc;
+      s.hcap = n;
+    }
+    LA_CUDA(h, cudaMemcpy(s.hoff, off.data(), off.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+    if (!allc.empty()) {
+      LA_CUDA(h, cudaMemcpy(s.hcol, allc.data(), allc.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+      LA_CUDA(h, cudaMemcpy(s.hval, allv.data(), allv.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+    }
+  }
   if (!bf16) {  // the x part again, compressed: kept (column, value) runs of every row k
     std::vector<int> off(Ks + 1, 0), cols;
     std::vector<float> vals;
@@ -928,6 +1006,9 @@ void lstm_approx_destroy(lstm_approx_t* h) {
       cudaFree(s.xidx[g]);
       cudaFree(s.xval[g]);
     }
+    cudaFree(s.hoff);
+    cudaFree(s.hcol);
+    cudaFree(s.hval);
   }
   cudaFree(h->h_state);
   cudaFree(h->c_state);
@@ -981,6 +1062,14 @@ int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
     case LSTM_APPROX_OPT_XPROJ:
       if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad projection choice %lld", value);
       h->opt_xproj = (int)value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_TAU_LAYOUT:
+      if (value < 0 || value > 1) return fail(h, LSTM_APPROX_EINVAL, "bad tau' layout %lld", value);
+      if (value == 1 && h->dtype != LSTM_APPROX_BF16)
+        return fail(h, LSTM_APPROX_EINVAL, "the compressed tau' layout is for bf16 factors (the tensor path)");
+      if (value == 1 && h->H > tau_sparse_max_h())
+        return fail(h, LSTM_APPROX_EINVAL, "the compressed tau' layout takes H <= %d", tau_sparse_max_h());
+      h->opt_tau_layout = (int)value;
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_PERSISTENT_VARIANT:
       if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad persistent variant %lld", value);

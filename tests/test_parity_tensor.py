@@ -201,3 +201,44 @@ def test_two_layer_workload_decomposed_factors(cuda_device):
     streams = [2, 41]
     ref = oracle_run(layers, x[:, streams], 8, dtype="bf16", checkpoints=cps)
     assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+@pytest.mark.parametrize("D,H,T,B,K,nz,cps", [
+    (40, 200, 4, 3, 80, 70, [5, 21, 79]),      # ragged H, B, K; depths off the slices
+    (64, 136, 2, 40, 45, 80, [17, 45]),        # two stream tiles, ragged tail
+    (48, 128, 3, 8, 256, 100, [64, 130]),      # many rows, term split of the gate GEMM
+    (32, 96, 3, 5, 8, 20, []),                 # packed gates (K <= 32)
+])
+def test_compressed_tau_layout(cuda_device, D, H, T, B, K, nz, cps):
+    """The compressed layout of v's h part (kept entries per row, CUDA cores)
+    for the recurrent projection, against the oracle."""
+    gates = [draw_factor_set(H, D + H, K, nz, 5400 + 7 * D + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 67)
+    got, m = run_gpu([gates], x, K, dtype="bf16", checkpoints=cps, tau_layout=1)
+    assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    ref = oracle_run([gates], x, K, dtype="bf16", checkpoints=cps)
+    assert_parity(got, ref, BF16_TOL)
+
+
+@pytest.mark.parametrize("keep,K", [(0.1, 128), (0.5, 512)])
+def test_compressed_tau_layout_large_batch_full_size(cuda_device, keep, K):
+    """D=2048, H=1024, T=64, B=1024 with the compressed tau' layout: sampled streams."""
+    w = WORKLOADS["c4"]
+    layers = [list(synthetic_layer("c4", 0, 512, keep))]
+    x = workload_inputs(w)
+    got, _ = run_gpu(layers, x, K, dtype="bf16", max_rank=512, tau_layout=1)
+    streams = [0, 513, 1023]
+    ref = oracle_run(layers, x[:, streams], K, dtype="bf16")
+    assert_parity(_sample(got, streams), ref, BF16_TOL)
+
+
+def test_compressed_tau_layout_refused_where_it_does_not_apply(cuda_device):
+    from paper_1905_00689_gb300 import LSTMApprox, LSTMApproxError, OPT_TAU_LAYOUT
+    m = LSTMApprox(1, [8], 16, 4, 1, "fp32")
+    with pytest.raises(LSTMApproxError):
+        m.set_option(OPT_TAU_LAYOUT, 1)
+    m.close()
+    m = LSTMApprox(1, [8], 2048, 4, 1, "bf16")
+    with pytest.raises(LSTMApproxError):
+        m.set_option(OPT_TAU_LAYOUT, 1)
+    m.close()
