@@ -768,10 +768,12 @@ bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint
 }
 
 int tc_rows_tile_n(int n_cols, int row_tiles) {
-  // few columns (tau' over B streams): 64 when that keeps one wave; else 128
-  // (with both planes of the activation a 128-column tile feeds 256 columns
-  // of MMA work per factor tile)
-  if ((long long)row_tiles * ((n_cols + 63) / 64) <= 148) return 64;
+  // the narrowest of 32, 64, 128 columns that keeps one wave (few columns:
+  // more CTAs, each streaming fewer activation bytes); many columns (the
+  // projection over T*B): 128, where both planes of the activation make a
+  // 128-column tile feed 256 columns of MMA work per factor tile
+  for (int bn : {32, 64})
+    if ((long long)row_tiles * ((n_cols + bn - 1) / bn) <= 148) return bn;
   return 128;
 }
 int tc_gates_splits(int tiles, int nkb, int* nkb_per) {

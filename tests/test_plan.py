@@ -49,7 +49,7 @@ def test_large_batch_workloads():
     # D=1024, H=512, B=256, K=512: 4 unit tiles x 8 tiles of 32 streams, the
     # terms split 4 ways to fill the GPU
     p = plan(BF16, 512, 20, 256, 512)
-    assert (p["path"], p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"]) == (PATH_TENSOR, 32, 4, 64)
+    assert (p["path"], p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"]) == (PATH_TENSOR, 32, 4, 32)
     # D=2048, H=1024, B=1024, K=512: 8 x 16 tiles of 64 streams, no split;
     # the tau' GEMM's 16 row tiles take 128 streams per tile
     p = plan(BF16, 1024, 64, 1024, 512)
@@ -136,15 +136,15 @@ def test_every_plan_covers_its_shape_and_fits(H, K, cs, variant):
 def test_tensor_tiles(H, B, K):
     """Stream tiles: the narrowest of 32/64/128 (gates) that keeps the grid
     within one wave of 148 CTAs, else the widest; tau' takes 32 streams up to
-    K = 32 (one tile of all four gates' rows), else 64 when that keeps one
-    wave, else 128; the gate GEMM's terms split over min(148 // tiles, 8,
-    chunks of 64) CTAs."""
+    K = 32 (one tile of all four gates' rows), else the narrowest of 32/64
+    that keeps one wave, else 128; the gate GEMM's terms split over
+    min(148 // tiles, 8, chunks of 64) CTAs."""
     p = plan(BF16, H, 2, B, K)
     units = -(-H // 128)
     nt = next((n for n in (32, 64, 128) if units * -(-B // n) <= 148), 128)
     assert p["gate_tile_streams"] == nt
     rows = 4 * -(-K // 128)
-    bn = 32 if K <= 32 else (64 if rows * -(-B // 64) <= 148 else 128)
+    bn = 32 if K <= 32 else next((n for n in (32, 64) if rows * -(-B // n) <= 148), 128)
     assert p["tau_tile_streams"] == bn
     tiles = units * -(-B // nt)
     chunks = -(-K // 64)
