@@ -252,8 +252,10 @@ enum lstm_approx_query_key {
   LSTM_APPROX_Q_LAST_PATH = 1,   /* recurrence path of the last run (enum below) */
   LSTM_APPROX_Q_CLUSTER = 2,     /* CTAs per cluster of the last persistent run */
   LSTM_APPROX_Q_DEVICE_BYTES = 3, /* device bytes currently held by the handle */
-  LSTM_APPROX_Q_PERSISTENT_VARIANT = 4 /* persistent kernel of the last persistent run
+  LSTM_APPROX_Q_PERSISTENT_VARIANT = 4, /* persistent kernel of the last persistent run
                                           (1 or 2, see LSTM_APPROX_OPT_PERSISTENT_VARIANT) */
+  LSTM_APPROX_Q_TENSOR_SEQ = 5   /* 1 if the last tensor-path layer ran as one launch
+                                    for all timesteps (see LSTM_APPROX_OPT_TENSOR_SEQ) */
 };
 enum lstm_approx_path {
   LSTM_APPROX_PATH_NONE = 0,
@@ -282,11 +284,17 @@ enum lstm_approx_option_key {
                                (T*B <= 32): 0 = automatic (compressed when v
                                keeps at most 1/8 of the x columns), 1 =
                                masked-dense rows, 2 = compressed rows */
-  LSTM_APPROX_OPT_TAU_LAYOUT = 7 /* the tensor path's recurrent projection tau'
+  LSTM_APPROX_OPT_TAU_LAYOUT = 7, /* the tensor path's recurrent projection tau'
                                (bf16 factors): 0 = masked-dense v rows on the
                                tensor cores (default: faster at every shape
                                measured), 1 = v's kept h entries (compressed
                                rows) on the CUDA cores, H <= 1280 */
+  LSTM_APPROX_OPT_TENSOR_SEQ = 8 /* tensor path: 0 = automatic (one launch per
+                               tile of streams for all T timesteps where the
+                               layer fits: K <= 32, H = 256, 512 or 1024,
+                               intermediate depths multiples of 16 or >= K,
+                               masked-dense tau'), 1 = two launches per
+                               timestep */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 
@@ -339,7 +347,11 @@ enum lstm_approx_plan_item {
   LSTM_APPROX_PLAN_TAU_TILE_STREAMS = 10,  /* tensor path: streams per tile of the tau' GEMM */
   LSTM_APPROX_PLAN_GATE_TILE_STREAMS = 11, /* tensor path: streams per tile of the gate GEMM */
   LSTM_APPROX_PLAN_GATE_SPLITS = 12,       /* tensor path: term-axis splits of the gate GEMM */
-  LSTM_APPROX_PLAN_ITEMS = 13
+  LSTM_APPROX_PLAN_TENSOR_SEQ = 13,        /* tensor path: 1 = one launch per tile of streams for
+                                              all T (then CLUSTER = H / 128 CTAs per tile and both
+                                              tile items = the streams per tile), 0 = two launches
+                                              per timestep */
+  LSTM_APPROX_PLAN_ITEMS = 14
 };
 int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int *checkpoints, int J,
                      int force_path, int cluster, int persistent_variant, int *out, int n_out,

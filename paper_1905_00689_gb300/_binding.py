@@ -19,16 +19,16 @@ LIB_PATH = os.path.join(HERE, "liblstm_approx.so")
 
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, ESTATE = range(6)
 FP32, BF16 = 0, 1
-Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT = range(5)
+Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT, Q_TENSOR_SEQ = range(6)
 PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
 (OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ,
- OPT_TAU_LAYOUT) = range(8)
+ OPT_TAU_LAYOUT, OPT_TENSOR_SEQ) = range(9)
 (PLAN_PATH, PLAN_PERSISTENT_VARIANT, PLAN_CLUSTER, PLAN_TERMS_PER_CTA, PLAN_UNITS_PER_WARP, PLAN_TERMS_PER_LANE,
  PLAN_VH_LAYOUT, PLAN_H_QUADS, PLAN_SMEM_BYTES, PLAN_TMEM_COLUMNS, PLAN_TAU_TILE_STREAMS, PLAN_GATE_TILE_STREAMS,
- PLAN_GATE_SPLITS, PLAN_ITEMS) = range(14)
+ PLAN_GATE_SPLITS, PLAN_TENSOR_SEQ, PLAN_ITEMS) = range(15)
 PLAN_KEYS = ("path", "persistent_variant", "cluster", "terms_per_cta", "units_per_warp", "terms_per_lane",
              "vh_layout", "h_quads", "smem_bytes", "tmem_columns", "tau_tile_streams", "gate_tile_streams",
-             "gate_splits")
+             "gate_splits", "tensor_seq")
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ETIMEOUT: "ETIMEOUT",
                 ESTATE: "ESTATE"}
 

@@ -56,6 +56,7 @@ struct LayerStore {
   int* hcol = nullptr;
   float* hval = nullptr;
   size_t hcap = 0;                 // entries allocated
+  bool hcsr_dirty = false;         // the host copies below changed since the last upload
   std::vector<int> hrows[4];       // per gate: host copy of its rows' kept h columns, counts per row
   std::vector<float> hvals[4];
   std::vector<int> hcount[4];
@@ -100,10 +101,12 @@ struct lstm_approx {
   int opt_force_path = 0, opt_cluster = 0, opt_persistent_variant = 0;
   int opt_xproj = 0;  // 0 automatic, 1 masked-dense, 2 compressed (fp32, T*B <= 32)
   int opt_tau_layout = 0;  // tensor path's tau': 0 masked-dense (tensor cores), 1 compressed (CUDA cores)
+  int opt_tensor_seq = 0;  // tensor path: 0 one launch for all timesteps where the layer fits, 1 per-step launches
   long long opt_wait_limit_us = 2000000;
   int opt_test_stall = 0;
   long long launches = 0;
   int last_path = 0, last_cluster = 0, last_variant = 0;
+  int last_tensor_seq = 0;  // 1 if the last tensor-path layer ran as one launch for all timesteps
   long long device_bytes = 0;
   lstm_approx_impl::Timing timing;
   std::string last_error;
@@ -299,6 +302,41 @@ cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs&
 // Term-axis splits for a gate GEMM of `tiles` CTAs over nkb 64-term chunks
 // (1: no split); *nkb_per receives the chunks per split.
 int tc_gates_splits(int tiles, int nkb, int* nkb_per);
+
+// One launch per tile of NS streams for all T timesteps of a layer (bf16
+// factors, K <= 32, H = 128 CS with CS in {1, 2, 4, 8}): a cluster of CS
+// CTAs, CTA r owning hidden units [128 r, 128 r + 128), keeps its columns of
+// the packed V_h, its rows of U, its h_t and c_t on chip; per step the CTAs
+// add their partial tau' over distributed shared memory and exchange the
+// bf16 pair of tau'.
+struct TcSeqArgs {
+  int H, K, Ks, B, T;
+  int rpg;                  // packed rows per gate: 8, 16 or 32 (K <= rpg)
+  int cs;                   // CTAs per cluster, H / 128
+  const float* P;           // [T*B][ldp] hoisted input projection, column g*Ks + k
+  int ldp;
+  const float* sigma;       // [4][Ks]
+  const float* bias;        // [4][H]
+  const float* h0;          // [B][H] or null (zero)
+  const float* c0;          // [B][H] or null (zero)
+  float* out_h;             // element (t, n, unit) at (t*B + n)*H + unit, or null
+  float* c_last;            // [B][H] c after the last step, or null
+  __nv_bfloat16* seq_bf16;  // pair of h_t for the next layer: (t*B + n)*ldh + unit, lo plane at + seq_plane; or null
+  int ldh;
+  long long seq_plane;
+  Checkpoints ck;           // intermediate depths: multiples of 16, or >= K
+  float* ckpt_h;            // element (j, t, n, unit) at j*ck_stride + (t*B + n)*H + unit, or null
+  float* ckpt_c;
+  long long ck_stride;
+  int* err;
+  long long limit_ns;
+  int test_stall;           // 1: CTA 0 of the first tile withholds its first partial tau' (the waits run out)
+};
+// Whether a layer of this shape takes the one-launch kernel; *ns receives
+// its streams per tile (32 or 64).
+bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, std::string* why);
+// Vh_p: the packed V_h map with boxes of rpg rows; U: the U map (128-row boxes).
+cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, int ns, cudaStream_t s);
 
 // Compressed tau' (the recurrent part of the pruned v as (column, value)
 // entries per storage row g*Ks + k, entries off[row] .. off[row + 1]) on the

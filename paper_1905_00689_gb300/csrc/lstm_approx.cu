@@ -253,6 +253,55 @@ TensorTiles tensor_tiles(int H, int B, int K, const Checkpoints& ck) {
   return t;
 }
 
+// The compressed h part of layer l's v on the device, for the compressed
+// tau' layout: CSR over the storage rows g*Ks + k of all four gates (rows not
+// set: empty), assembled from the per-gate host copies that set_factors
+// keeps, when they changed since the last upload.
+int ensure_tau_csr(lstm_approx_t* h, int l) {
+  LayerStore& s = h->layers[l];
+  if (!s.hcsr_dirty && s.hoff != nullptr) return LSTM_APPROX_OK;
+  const int Ks = h->Ks;
+  std::vector<int> off(4 * (size_t)Ks + 1, 0), allc;
+  std::vector<float> allv;
+  for (int g = 0; g < 4; ++g) {
+    size_t e = 0;
+    for (int k = 0; k < Ks; ++k) {
+      const int c = k < (int)s.hcount[g].size() ? s.hcount[g][k] : 0;
+      for (int i = 0; i < c; ++i) {
+        allc.push_back(s.hrows[g][e + i]);
+        allv.push_back(s.hvals[g][e + i]);
+      }
+      e += c;
+      off[g * Ks + k + 1] = (int)allc.size();
+    }
+  }
+  const size_t n = allc.empty() ? 1 : allc.size();
+  // earlier runs on the handle's stream may still read the old copy
+  LA_CUDA(h, cudaStreamSynchronize(h->stream), "synchronising before the factor upload");
+  if (s.hoff == nullptr) {
+    const int rc = dmalloc(h, reinterpret_cast<void**>(&s.hoff), off.size() * 4, "compressed factor storage");
+    if (rc) return rc;
+  }
+  if (n > s.hcap) {
+    dfree(h, s.hcol, s.hcap * 4);
+    dfree(h, s.hval, s.hcap * 4);
+    s.hcol = nullptr;
+    s.hval = nullptr;
+    s.hcap = 0;
+    int rc = dmalloc(h, reinterpret_cast<void**>(&s.hcol), n * 4, "compressed factor storage");
+    if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.hval), n * 4, "compressed factor storage");
+    if (rc) return rc;
+    s.hcap = n;
+  }
+  LA_CUDA(h, cudaMemcpy(s.hoff, off.data(), off.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+  if (!allc.empty()) {
+    LA_CUDA(h, cudaMemcpy(s.hcol, allc.data(), allc.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+    LA_CUDA(h, cudaMemcpy(s.hval, allv.data(), allv.size() * 4, cudaMemcpyHostToDevice), "factor upload");
+  }
+  s.hcsr_dirty = false;
+  return LSTM_APPROX_OK;
+}
+
 int ensure_factor_maps(lstm_approx_t* h, int l) {
   LayerStore& s = h->layers[l];
   if (s.maps_ready) return LSTM_APPROX_OK;
@@ -279,6 +328,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   const long long ldp = 4LL * h->Ks;
   int rc = ensure_factor_maps(h, l);
   if (rc) return rc;
+  if (h->opt_tau_layout == 1 && (rc = ensure_tau_csr(h, l))) return rc;
   const bool top = l == h->L - 1;
   const long long limit_ns = h->opt_wait_limit_us * 1000LL;
   // up to 32 terms the products take one tile of all four gates' rows
@@ -324,6 +374,43 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   __nv_bfloat16* hb = static_cast<__nv_bfloat16*>(h->h_bf16);
   __nv_bfloat16* tau = static_cast<__nv_bfloat16*>(h->tau);
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
+  int ns = 0;
+  if (h->opt_tensor_seq == 0 && h->opt_tau_layout == 0 && (long long)B * ldp < (1LL << 31) &&
+      tc_seq_fits(H, B, K, ck, &ns, nullptr)) {
+    // one launch per tile of streams for all T timesteps
+    TcSeqArgs qa{};
+    qa.H = H;
+    qa.K = K;
+    qa.Ks = h->Ks;
+    qa.B = B;
+    qa.T = T;
+    qa.rpg = rpg;
+    qa.cs = H / 128;
+    qa.P = h->Px;
+    qa.ldp = (int)ldp;
+    qa.sigma = s.sigma;
+    qa.bias = s.bias;
+    qa.h0 = h0;
+    qa.c0 = c0;
+    qa.out_h = out_h;
+    qa.c_last = out_c;
+    qa.seq_bf16 = top ? nullptr : static_cast<__nv_bfloat16*>(h->seq_bf16);
+    qa.ldh = h->ldh;
+    qa.seq_plane = (long long)TB * h->ldh;
+    qa.ck = ck;
+    qa.ckpt_h = ckpt_h;
+    qa.ckpt_c = ckpt_c;
+    qa.ck_stride = (long long)T * B * H;
+    qa.err = h->err;
+    qa.limit_ns = limit_ns;
+    qa.test_stall = h->opt_test_stall;
+    h->opt_test_stall = 0;
+    LA_CUDA(h, launch_tc_seq(s.map_vh_p[pi], s.map_u, qa, ns, h->stream), "recurrence launch");
+    h->launches += 1;
+    h->last_tensor_seq = 1;
+    return LSTM_APPROX_OK;
+  }
+  h->last_tensor_seq = 0;
   LA_CUDA(h, launch_tc_init_state(h0, c0, B, H, hb, h->ldh, cs, h->stream), "state init launch");
   h->launches += 1;
   // packed gates write only the first rpg terms of each gate's tau' rows; the
@@ -745,43 +832,7 @@ int lstm_approx_set_factors(lstm_approx_t* h, int layer, int gate, int K, int nz
         vals.push_back(f);
         ++cnt[k];
       }
-    // CSR over the storage rows g*Ks + k of all four gates (rows not set: empty)
-    std::vector<int> off(4 * (size_t)Ks + 1, 0), allc;
-    std::vector<float> allv;
-    for (int g = 0; g < 4; ++g) {
-      size_t e = 0;
-      for (int k = 0; k < Ks; ++k) {
-        const int row = g * Ks + k;
-        const int c = k < (int)s.hcount[g].size() ? s.hcount[g][k] : 0;
-        for (int i = 0; i < c; ++i) {
-          allc.push_back(s.hrows[g][e + i]);
-          allv.push_back(s.hvals[g][e + i]);
-        }
-        e += c;
-        off[row + 1] = (int)allc.size();
-      }
-    }
-    const size_t n = allc.empty() ? 1 : allc.size();
-    if (s.hoff == nullptr) {
-      int rc = dmalloc(h, reinterpret_cast<void**>(&s.hoff), off.size() * 4, "compressed factor storage");
-      if (rc) return rc;
-    }
-    if (n > s.hcap) {
-      dfree(h, s.hcol, s.hcap * 4);
-      dfree(h, s.hval, s.hcap * 4);
-      s.hcol = nullptr;
-      s.hval = nullptr;
-      s.hcap = 0;
-      int rc = dmalloc(h, reinterpret_cast<void**>(&s.hcol), n * 4, "compressed factor storage");
-      if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&s.hval), n * 4, "compressed factor storage");
-      if (rc) return rc;
-      s.hcap = n;
-    }
-    LA_CUDA(h, cudaMemcpy(s.hoff, off.data(), off.size() * 4, cudaMemcpyHostToDevice), "factor upload");
-    if (!allc.empty()) {
-      LA_CUDA(h, cudaMemcpy(s.hcol, allc.data(), allc.size() * 4, cudaMemcpyHostToDevice), "factor upload");
-      LA_CUDA(h, cudaMemcpy(s.hval, allv.data(), allv.size() * 4, cudaMemcpyHostToDevice), "factor upload");
-    }
+    s.hcsr_dirty = true;  // the device copy is rebuilt by the first run that uses it
   }
   if (!bf16) {  // the x part again, compressed: kept (column, value) runs of every row k
     std::vector<int> off(Ks + 1, 0), cols;
@@ -1033,6 +1084,7 @@ int lstm_approx_query(const lstm_approx_t* h, int key, long long* value) {
     case LSTM_APPROX_Q_CLUSTER: *value = h->last_cluster; return LSTM_APPROX_OK;
     case LSTM_APPROX_Q_DEVICE_BYTES: *value = h->device_bytes; return LSTM_APPROX_OK;
     case LSTM_APPROX_Q_PERSISTENT_VARIANT: *value = h->last_variant; return LSTM_APPROX_OK;
+    case LSTM_APPROX_Q_TENSOR_SEQ: *value = h->last_tensor_seq; return LSTM_APPROX_OK;
     default: return LSTM_APPROX_EINVAL;
   }
 }
@@ -1070,6 +1122,10 @@ int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
       if (value == 1 && h->H > tau_sparse_max_h())
         return fail(h, LSTM_APPROX_EINVAL, "the compressed tau' layout takes H <= %d", tau_sparse_max_h());
       h->opt_tau_layout = (int)value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_TENSOR_SEQ:
+      if (value < 0 || value > 1) return fail(h, LSTM_APPROX_EINVAL, "bad tensor launch choice %lld", value);
+      h->opt_tensor_seq = (int)value;
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_PERSISTENT_VARIANT:
       if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad persistent variant %lld", value);
@@ -1141,10 +1197,19 @@ int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int* chec
       v[LSTM_APPROX_PLAN_TMEM_COLUMNS] = pc.ag.tcols;
     }
   } else if (path == LSTM_APPROX_PATH_TENSOR) {
-    const TensorTiles tt = tensor_tiles(hidden, B, K, ck);
-    v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = tt.bnh;
-    v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = tt.nt;
-    v[LSTM_APPROX_PLAN_GATE_SPLITS] = tt.ks;
+    int ns = 0;
+    if (tc_seq_fits(hidden, B, K, ck, &ns, nullptr)) {
+      v[LSTM_APPROX_PLAN_TENSOR_SEQ] = 1;
+      v[LSTM_APPROX_PLAN_CLUSTER] = hidden / 128;
+      v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = ns;
+      v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = ns;
+      v[LSTM_APPROX_PLAN_GATE_SPLITS] = 1;
+    } else {
+      const TensorTiles tt = tensor_tiles(hidden, B, K, ck);
+      v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = tt.bnh;
+      v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = tt.nt;
+      v[LSTM_APPROX_PLAN_GATE_SPLITS] = tt.ks;
+    }
   }
   for (int i = 0; i < n_out; ++i) out[i] = i < LSTM_APPROX_PLAN_ITEMS ? v[i] : 0;
   return LSTM_APPROX_OK;

@@ -279,6 +279,20 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
+// 32 lanes x 8 consecutive 32-bit columns and the wait for them in one
+// statement.
+__device__ __forceinline__ void tmem_ld8_sync(uint32_t taddr, float (&v)[8]) {
+  uint32_t r[8];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // Four loads of 32 lanes x 8 consecutive 32-bit columns (at t0 .. t3) and
 // the wait for them in one statement, so that no use of the values can be
 // scheduled before they have arrived: v[i][c] = column t_i + c of this
@@ -414,6 +428,21 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
   d |= static_cast<uint64_t>(1) << 46;                   // descriptor version of tcgen05
   d |= static_cast<uint64_t>(2) << 61;                   // 128-byte swizzle
   return d;
+}
+
+// The same with 8-row groups `sbo` bytes apart (a multiple of 1024), for a
+// tile whose row groups are interleaved with other tiles' groups.
+__device__ __forceinline__ uint64_t umma_desc_sw128_sbo(uint32_t saddr, uint32_t sbo) {
+  return (umma_desc_sw128(saddr) & ~(static_cast<uint64_t>(0x3FFF) << 32)) |
+         (static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32);
+}
+
+// Byte offset of bf16 element k (< 64) of row r in a K-major tile of
+// 128-byte rows with 128-byte swizzling (the layout TMA writes and the MMA
+// descriptors above read), relative to the 1024-byte aligned group of 8 rows
+// that holds row r: the 16-byte chunk index is XORed with r mod 8.
+__host__ __device__ __forceinline__ uint32_t sw128_offset(int r, int k) {
+  return static_cast<uint32_t>((r & 7) * 128 + ((((k >> 3) ^ r) & 7) << 4) + (k & 7) * 2);
 }
 
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 D, both

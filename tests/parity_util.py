@@ -52,11 +52,11 @@ def synthetic_layer(wname: str, layer: int, K: int, keep: float):
 
 
 def run_gpu(layers, x, K, dtype="fp32", h0=None, c0=None, checkpoints=(), force_path=0, cluster=0,
-            max_rank=None, max_batch=None, want_c=True, variant=0, xproj=0, tau_layout=0):
+            max_rank=None, max_batch=None, want_c=True, variant=0, xproj=0, tau_layout=0, tensor_seq=0):
     """Set factors, run through the C-ABI, return numpy outputs and the handle."""
     import torch
     from paper_1905_00689_gb300 import (LSTMApprox, OPT_CLUSTER, OPT_FORCE_PATH, OPT_PERSISTENT_VARIANT,
-                                        OPT_TAU_LAYOUT, OPT_XPROJ)
+                                        OPT_TAU_LAYOUT, OPT_TENSOR_SEQ, OPT_XPROJ)
     dev = torch.device("cuda:0")
     T, B, D = x.shape
     L = len(layers)
@@ -75,6 +75,8 @@ def run_gpu(layers, x, K, dtype="fp32", h0=None, c0=None, checkpoints=(), force_
         m.set_option(OPT_XPROJ, xproj)
     if tau_layout:
         m.set_option(OPT_TAU_LAYOUT, tau_layout)
+    if tensor_seq:
+        m.set_option(OPT_TENSOR_SEQ, tensor_seq)
     xt = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(dev)
     out_h = torch.full((T, B, H), float("nan"), device=dev)
     out_c = torch.full((L, B, H), float("nan"), device=dev) if want_c else None

@@ -140,6 +140,10 @@ def test_tensor_tiles(H, B, K):
     that keeps one wave, else 128; the gate GEMM's terms split over
     min(148 // tiles, 8, chunks of 64) CTAs."""
     p = plan(BF16, H, 2, B, K)
+    if K <= 32 and H in (256, 512, 1024):  # one launch for all timesteps (test_tensor_seq_plan)
+        assert p["tensor_seq"] == 1
+        return
+    assert p["tensor_seq"] == 0
     units = -(-H // 128)
     nt = next((n for n in (32, 64, 128) if units * -(-B // n) <= 148), 128)
     assert p["gate_tile_streams"] == nt
@@ -154,6 +158,31 @@ def test_tensor_tiles(H, B, K):
     else:
         per = -(-chunks // ks)
         assert p["gate_splits"] == -(-chunks // per)  # no empty split
+
+
+@pytest.mark.parametrize("H,B", [(256, 1), (256, 3000), (512, 256), (512, 1300), (1024, 1024), (1024, 5)])
+@pytest.mark.parametrize("K", [1, 8, 16, 17, 32])
+def test_tensor_seq_plan(H, B, K):
+    """One launch per tile of streams for all timesteps: a cluster of H / 128
+    CTAs per tile; 32 streams per tile at H = 256, and at H = 512 while the
+    clusters fit in one wave of 148 CTAs, else 64 (each CTA owns 8 or 16
+    streams)."""
+    p = plan(BF16, H, 2, B, K)
+    cs = H // 128
+    ns = 32 if cs == 2 or (cs == 4 and -(-B // 32) * cs <= 148) else 64
+    assert (p["tensor_seq"], p["cluster"], p["tau_tile_streams"], p["gate_tile_streams"], p["gate_splits"]) == \
+        (1, cs, ns, ns, 1)
+    assert ns // cs in (8, 16)
+
+
+@pytest.mark.parametrize("H,K,ck,seq", [
+    (512, 32, [16], 1), (512, 32, [16, 32], 1), (512, 20, [16, 20], 1),  # depths on the slices, or = K
+    (512, 32, [10], 0), (512, 32, [8, 16], 0),                            # a depth off the 16-term slices
+    (512, 33, [], 0), (2048, 16, [], 0), (384, 16, [], 0), (128, 16, [], 0), (96, 8, [], 0),
+])
+def test_tensor_seq_rejections(H, K, ck, seq):
+    """Shapes outside the one-launch kernel take two launches per timestep."""
+    assert plan(BF16, H, 2, 64, K, ck)["tensor_seq"] == seq
 
 
 def test_paths():
