@@ -379,6 +379,7 @@ def run_ours(args):
     dense_kernel = None if args.quick else dense_kernel_comparator(dev, stream, flush, x, statistics.median(step_ms))
     k_sweeps = [] if (args.quick or args.no_large) else workload_k_sweeps(dev, flush)
     tau_layouts = [] if (args.quick or args.no_large) else tau_layout_comparison(dev, stream)
+    tensor_launches = [] if (args.quick or args.no_large) else tensor_launch_comparison(dev, stream, flush)
 
     # ---- end to end through the host-buffer entry point ---------------------
     xh = torch.from_numpy(x_host).pin_memory()
@@ -431,6 +432,7 @@ def run_ours(args):
             "large_batch": large,
             "k_sweeps": k_sweeps,
             "tau_layouts": tau_layouts,
+            "tensor_launches": tensor_launches,
             "paper_case_study": paper_case,
             "dense_lstm_comparator": dense,
             "dense_kernel_comparator": dense_kernel,
@@ -600,6 +602,48 @@ def dense_comparator(dev, stream, x, steps: int = 200) -> dict:
     return {"kind": "dense torch.nn.LSTM (cuDNN), fp32, same D/H/T/B, warm caches", "ms_per_run": ms,
             "value": T * B / (ms / 1e3), "unit": UNIT,
             "dense_weight_bytes": 4 * 4 * WL.H * (D + WL.H)}
+
+
+def tensor_launch_comparison(dev, stream, flush) -> list:
+    """The tensor path at the workloads' small depths as one launch per tile
+    of streams for all timesteps (the default where the layer fits) against
+    two launches per timestep (LSTM_APPROX_OPT_TENSOR_SEQ = 1): whole-run
+    timesteps·streams/s and µs per timestep (CUDA events on the library's
+    stream, L2 flushed before each run, median of 10)."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox, OPT_TENSOR_SEQ, Q_TENSOR_SEQ
+    out = []
+    for name, keep, Ks in (("c3", 0.5, (32,)), ("c4", 0.5, (8, 32)), ("c4", 0.1, (8, 32))):
+        w = WORKLOADS[name]
+        m = LSTMApprox(1, [w.D], w.H, max(Ks), w.B, "bf16", stream=stream)
+        m.set_layer(0, synthetic_layer_factors(w, 0, max(Ks), keep))
+        x = torch.from_numpy(workload_inputs(w).astype(np.float32)).to(dev)
+        oh = torch.empty((w.T, w.B, w.H), device=dev)
+        for K in Ks:
+            row = {"workload": w.name, "keep": keep, "K": K}
+            for seq, key in ((0, "one_launch"), (1, "per_timestep")):
+                m.set_option(OPT_TENSOR_SEQ, seq)
+                for _ in range(3):
+                    m.run(x, K, oh)
+                evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(10)]
+                torch.cuda.synchronize(dev)
+                with torch.cuda.stream(stream):  # the flush on the timed stream, outside the events
+                    for i, (a, b) in enumerate(evs):
+                        flush.fill_(float(i))
+                        a.record(stream)
+                        m.run(x, K, oh)
+                        b.record(stream)
+                torch.cuda.synchronize(dev)
+                ms = statistics.median(a.elapsed_time(b) for a, b in evs)
+                row[key] = {"value": w.T * w.B / (ms / 1e3), "unit": UNIT, "us_per_timestep": 1e3 * ms / w.T,
+                            "one_launch_taken": bool(m.query(Q_TENSOR_SEQ))}
+            out.append(row)
+        m.set_option(OPT_TENSOR_SEQ, 0)
+        m.close()
+        del x, oh
+        torch.cuda.empty_cache()
+    return out
 
 
 def tau_layout_comparison(dev, stream) -> list:

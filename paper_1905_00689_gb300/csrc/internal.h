@@ -51,6 +51,7 @@ struct LayerStore {
   bool maps_ready = false;  // tensor maps of Vx, Vh, U (bf16 path), built on first use
   TcMap map_vx, map_vh, map_u;
   TcMap map_vx_p[3], map_vh_p[3];  // the same with boxes of 8, 16, 32 rows (packed gates)
+  TcMap map_u64;                   // U as 32-term boxes of 128 rows, 64-byte swizzled (one-launch kernel)
   // compressed recurrent part of v (bf16 factors): CSR over storage rows g*Ks + k
   int* hoff = nullptr;
   int* hcol = nullptr;
@@ -238,9 +239,10 @@ cudaError_t launch_persistent_choice(const PersistentChoice& c, const Persistent
 // lo plane of R rows, so one tensor map of 2R rows covers both.
 
 // 2-D K-major bf16 tensor [rows][inner] with `pitch_bytes` between rows, as
-// TMA tiles of 64 inner elements x box_rows rows, 128-byte swizzled.
+// TMA tiles of box_rows rows of one swizzled row each: 64 inner elements
+// with 128-byte swizzling, or 32 with 64-byte swizzling.
 bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
-                 uint32_t box_rows);
+                 uint32_t box_rows, uint32_t swizzle_bytes = 128);
 int tc_rows_tile_n(int n_cols, int row_tiles);  // column tile of launch_tc_rows
 int tc_gates_tile_n(int H, int B);               // stream tile of launch_tc_gates
 
@@ -304,15 +306,15 @@ cudaError_t launch_tc_gates(const TcMap& U, const TcMap& Tau, const TcGatesArgs&
 int tc_gates_splits(int tiles, int nkb, int* nkb_per);
 
 // One launch per tile of NS streams for all T timesteps of a layer (bf16
-// factors, K <= 32, H = 128 CS with CS in {1, 2, 4, 8}): a cluster of CS
-// CTAs, CTA r owning hidden units [128 r, 128 r + 128), keeps its columns of
+// factors, K <= 32, H = 256, 512 or 1024): a cluster of CS CTAs, CTA r
+// owning hidden units [UC r, UC r + UC) (UC = 128 or 256), keeps its columns of
 // the packed V_h, its rows of U, its h_t and c_t on chip; per step the CTAs
 // add their partial tau' over distributed shared memory and exchange the
 // bf16 pair of tau'.
 struct TcSeqArgs {
   int H, K, Ks, B, T;
   int rpg;                  // packed rows per gate: 8, 16 or 32 (K <= rpg)
-  int cs;                   // CTAs per cluster, H / 128
+  int cs;                   // CTAs per cluster, H / (128 units per tile x unit tiles per CTA)
   const float* P;           // [T*B][ldp] hoisted input projection, column g*Ks + k
   int ldp;
   const float* sigma;       // [4][Ks]
@@ -333,10 +335,11 @@ struct TcSeqArgs {
   int test_stall;           // 1: CTA 0 of the first tile withholds its first partial tau' (the waits run out)
 };
 // Whether a layer of this shape takes the one-launch kernel; *ns receives
-// its streams per tile (32 or 64).
-bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, std::string* why);
-// Vh_p: the packed V_h map with boxes of rpg rows; U: the U map (128-row boxes).
-cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, int ns, cudaStream_t s);
+// its streams per tile (32 or 64), *mt its 128-unit tiles per CTA (1 or 2).
+bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, int* mt, std::string* why);
+// Vh_p: the packed V_h map with boxes of rpg rows; U64: U as 32-term boxes of
+// 128 rows with 64-byte swizzling.
+cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U64, const TcSeqArgs& a, int ns, int mt, cudaStream_t s);
 
 // Compressed tau' (the recurrent part of the pruned v as (column, value)
 // entries per storage row g*Ks + k, entries off[row] .. off[row + 1]) on the

@@ -751,18 +751,20 @@ cudaError_t launch_gates_t(const TcMap& U, const TcMap& Tau, const TcGatesArgs& 
 
 }  // namespace
 
-bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes, uint32_t box_rows) {
+bool tc_make_map(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes, uint32_t box_rows,
+                 uint32_t swizzle_bytes) {
   static_assert(sizeof(CUtensorMap) <= sizeof(m->bytes), "tensor map storage");
   EncodeTiled enc = encoder();
   if (!enc) return false;
   std::memset(m->bytes, 0, sizeof(m->bytes));
   const cuuint64_t dims[2] = {inner, rows};
   const cuuint64_t strides[1] = {pitch_bytes};
-  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
+  const cuuint32_t box[2] = {swizzle_bytes / 2u, box_rows};  // one swizzled row of bf16 elements
   const cuuint32_t estr[2] = {1, 1};
   const CUresult r = enc(reinterpret_cast<CUtensorMap*>(m->bytes), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                          const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }

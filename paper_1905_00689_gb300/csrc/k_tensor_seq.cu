@@ -4,13 +4,14 @@
 //
 // The per-timestep kernels of k_tensor.cu pay two dependent launches per
 // step and stream their whole factor tiles through shared memory every step,
-// which at small K costs about 18 us per step whatever K is.  Here a cluster
-// of CS = H / 128 CTAs serves a tile of NS streams (32 or 64) for the whole
-// sequence; CTA r owns hidden units [128 r, 128 r + 128) and keeps on chip:
+// which at small K costs about 14-18 us per step whatever K is.  Here a
+// cluster of CS CTAs serves a tile of NS streams (32 or 64) for the whole
+// sequence; CTA r owns UC = 128 MT hidden units [UC r, UC r + UC) (MT = 1 or
+// 2, CS = H / UC) and keeps on chip:
 //
 //   - its columns of the packed V_h (the four gates' first rpg rows, rpg =
-//     8, 16 or 32 >= K, the A operand of the tau' product), 32 KB;
-//   - its rows of U, one 128 x 64-term tile per gate, 64 KB;
+//     8, 16 or 32 >= K, the A operand of the tau' product), 32 KB per 128 units;
+//   - its rows of U, the first 32 terms of each gate, 32 KB per 128 units;
 //   - h_{t-1} of its units as the bf16 pair (the B operand of the tau'
 //     product), c_{t-1} in registers of the epilogue threads;
 //   - tau' of all terms and the tile's streams as the bf16 pair (the B
@@ -18,17 +19,18 @@
 //
 // One timestep (Eq. 1 and Sec. II):
 //   (a2) the CTA's partial tau' over its units, acc[(g,k)][n] =
-//        sum_{j in CTA} Vh[(g,k)][j] h_{t-1}[n][j]  (16 MMAs, M = 128, N = NS);
+//        sum_{j in CTA} Vh[(g,k)][j] h_{t-1}[n][j]  (M = 128, N = NS);
 //   exchange 1: the epilogue warps read the partials from tensor memory and
 //        send each CTA the columns of the streams it owns (SP = NS / CS
-//        streams per CTA) with st.async;
+//        streams per CTA, 8 or 16) with st.async;
 //   the owner adds the CS partials in rank order, forms
 //        tau' = sigma (sum + P_t) (zero for k >= K) and its pair, writes them
 //        into its tau' operand and, exchange 2, copies that block to every
 //        other CTA with one bulk copy each;
 //   (a3, a6) the four gate sums of the CTA's units, y_g = U_g tau'_g (one
-//        tensor-memory accumulator per gate), cut at each intermediate depth
-//        (a multiple of 16) for the checkpoint cells, as in k_tensor.cu;
+//        tensor-memory accumulator per gate and 128 units), cut at each
+//        intermediate depth (a multiple of 16) for the checkpoint cells, as
+//        in k_tensor.cu;
 //   (a4) the cells, with h_t written as the pair into the next step's tau'
 //        operand, and as fp32 (and for a lower layer as the pair) to memory.
 //
@@ -51,25 +53,25 @@ constexpr int kSeqEpw = 4;                 // epilogue warps per 32-lane quarter
 constexpr int kSeqEpi = 4 * kSeqEpw * 32;  // epilogue threads
 constexpr int kSeqThreads = 128 + kSeqEpi; // warp 0: TMA and MMA issue, warp 1: tensor memory, 2-3 idle
 constexpr int kSeqMaxRed = 4;              // owner elements (tau' values) per epilogue thread at most
-constexpr uint32_t kUnits = 128;           // hidden units per CTA
-constexpr uint32_t kSeqAtau = 32768;       // packed V_h columns: two 64-unit tiles of 128 rows
-constexpr uint32_t kSeqAgate = 65536;      // U rows: four 128 x 64-term tiles
+constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident at once on a GB300 (152 SMs)
 
-// Shared-memory layout, offsets from the 1024-byte aligned base:
-//   Atau  [2 unit halves][128 rows][128 B]
-//   Agate [4 gates][128 units][128 B]
-//   Bh    [2 planes][2 unit halves][NS streams][128 B]
-//   Btau  [NS/8 stream groups][4 gates][2 planes][8 streams][128 B]
+// Shared-memory layout, offsets from the 1024-byte aligned base (MT 128-unit
+// tiles per CTA, NS streams, 4 rpg packed rows):
+//   Atau  [2 MT unit blocks of 64][128 rows][128 B]        128-byte swizzle
+//   Agate [4 gates][MT][128 units][64 B] (terms 0..31)     64-byte swizzle
+//   Bh    [2 planes][2 MT unit blocks of 64][NS streams][128 B]
+//   Btau  [NS/8 stream groups][4 gates][2 planes][8 streams][64 B]   64-byte swizzle
 //   RS    [CS sources][4 rpg rows][SP streams] fp32 partial tau'
 //   barriers, tensor-memory slot
 struct SeqLayout {
-  uint32_t bh, btau, rs, bar, total;
+  uint32_t agate, bh, btau, rs, bar, total;
 };
-__host__ __device__ inline SeqLayout seq_layout(int ns, int r4) {
+__host__ __device__ inline SeqLayout seq_layout(int ns, int mt, int r4) {
   SeqLayout l;
-  l.bh = kSeqAtau + kSeqAgate;
-  l.btau = l.bh + (uint32_t)ns * 512u;
-  l.rs = l.btau + (uint32_t)ns * 1024u;
+  l.agate = 32768u * mt;
+  l.bh = l.agate + 32768u * mt;
+  l.btau = l.bh + (uint32_t)ns * 512u * mt;
+  l.rs = l.btau + (uint32_t)ns * 512u;
   l.bar = l.rs + (uint32_t)r4 * ns * 4u;
   l.total = l.bar + 128u + 1024u;  // barriers and slot, alignment slack
   return l;
@@ -89,19 +91,25 @@ __device__ __forceinline__ void seq_pair(float v, __nv_bfloat16& hi, __nv_bfloat
   lo = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-template <int NS>
+template <int NS, int MT>
 __global__ void __launch_bounds__(kSeqThreads, 1)
     tc_seq_kernel(const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmu, TcSeqArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  constexpr int SPW = NS / kSeqEpw;                  // streams per epilogue warp
-  constexpr uint32_t kCols = NS == 64 ? 512 : 256;  // tau' accumulator, then the four gate accumulators
-  constexpr uint32_t tAcc = 0, tGate = NS;
+  constexpr int SPW = NS / kSeqEpw;  // streams per epilogue warp
+  constexpr int UC = 128 * MT;       // hidden units per CTA
+  constexpr int NU = UC / 64;        // 64-unit blocks (K-dim tiles of the tau' product)
+  // tensor memory: the gate accumulators (gate g, unit tile m at column (g MT + m) NS); the
+  // tau' accumulator shares the first NS columns (it is read before the gate MMAs start,
+  // and they are read before the next tau' MMAs start)
+  constexpr uint32_t kUsed = 4u * MT * NS;
+  constexpr uint32_t kCols = kUsed <= 256 ? 256 : 512;
+  constexpr uint32_t tAcc = 0, tGate = 0;
   const int CS = a.cs, SP = NS / CS, rpg = a.rpg, R4 = 4 * rpg;
-  const SeqLayout L = seq_layout(NS, R4);
+  const SeqLayout L = seq_layout(NS, MT, R4);
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gb = smem_raw + (base - raw);  // generic pointer to the base
-  const uint32_t sAtau = base, sAgate = base + kSeqAtau, sBh = base + L.bh, sBtau = base + L.btau,
+  const uint32_t sAtau = base, sAgate = base + L.agate, sBh = base + L.bh, sBtau = base + L.btau,
                  sRS = base + L.rs, sBar = base + L.bar;
   const uint32_t fac_full = sBar, h_ready = sBar + 8, tacc_full = sBar + 16, rs_full = sBar + 24,
                  tau_full = sBar + 32, acc_full = sBar + 40, ckpt_bar = sBar + 48, ckpt_done = sBar + 56,
@@ -110,8 +118,8 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rank = (int)cluster_ctarank();
-  const int j0 = rank * (int)kUnits;       // first hidden unit of this CTA
-  const int n0 = (int)blockIdx.y * NS;     // first stream of this cluster's tile
+  const int j0 = rank * UC;             // first hidden unit of this CTA
+  const int n0 = (int)blockIdx.y * NS;  // first stream of this cluster's tile
   const int T = a.T, B = a.B, H = a.H;
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
@@ -136,15 +144,15 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     mbar_init(drain_bar, 1);
     fence_mbarrier_init_cluster();
   }
-  // zero what no copy writes: the V_h tile's rows from 4 rpg on, and the
+  // zero what no copy writes: the V_h tiles' rows from 4 rpg on, and the
   // tau' operand (its terms from rpg on stay zero for the whole launch)
   {
     const uint32_t zrow = (uint32_t)R4 * 128u, zlen = 16384u - zrow;
-    for (uint32_t i = threadIdx.x; i < 2u * zlen / 16u; i += blockDim.x) {
-      const uint32_t half = i / (zlen / 16u), o = i % (zlen / 16u);
-      *reinterpret_cast<uint4*>(gb + half * 16384u + zrow + 16u * o) = make_uint4(0, 0, 0, 0);
+    for (uint32_t i = threadIdx.x; i < NU * zlen / 16u; i += blockDim.x) {
+      const uint32_t blk = i / (zlen / 16u), o = i % (zlen / 16u);
+      *reinterpret_cast<uint4*>(gb + blk * 16384u + zrow + 16u * o) = make_uint4(0, 0, 0, 0);
     }
-    for (uint32_t i = threadIdx.x; i < (uint32_t)NS * 1024u / 16u; i += blockDim.x)
+    for (uint32_t i = threadIdx.x; i < (uint32_t)NS * 512u / 16u; i += blockDim.x)
       *reinterpret_cast<uint4*>(gb + L.btau + 16u * i) = make_uint4(0, 0, 0, 0);
     fence_proxy_async_shared();
   }
@@ -162,27 +170,26 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     if (lane == 0) {  // ---- factor copies, then the MMA issue of every step ----
       tma_prefetch_map(&tmv);
       tma_prefetch_map(&tmu);
-      mbar_arrive_expect_tx(fac_full, 2u * R4 * 128u + kSeqAgate);
-#pragma unroll
+      mbar_arrive_expect_tx(fac_full, (uint32_t)NU * R4 * 128u + 4u * MT * 8192u);
       for (int g = 0; g < 4; ++g)
-#pragma unroll
-        for (int half = 0; half < 2; ++half)
-          tma_load_2d(sAtau + half * 16384u + g * rpg * 128u, &tmv, fac_full, j0 + 64 * half, g * a.Ks);
-#pragma unroll
-      for (int g = 0; g < 4; ++g) tma_load_2d(sAgate + g * 16384u, &tmu, fac_full, 0, g * H + j0);
+        for (int blk = 0; blk < NU; ++blk)
+          tma_load_2d(sAtau + blk * 16384u + g * rpg * 128u, &tmv, fac_full, j0 + 64 * blk, g * a.Ks);
+      for (int g = 0; g < 4; ++g)
+        for (int m = 0; m < MT; ++m)
+          tma_load_2d(sAgate + (g * MT + m) * 8192u, &tmu, fac_full, 0, g * H + j0 + 128 * m);
       bool ok = seq_wait(fac_full, 0, limit, err);
       constexpr uint32_t idesc = umma_idesc_bf16(128, NS);
       for (int t = 0; t < T && ok; ++t) {
-        // (a2) partial tau' of this CTA's units: 8 slices of 16 units x both planes of h_{t-1}
+        // (a2) partial tau' of this CTA's units: UC / 16 slices x both planes of h_{t-1}
         if (!(ok = seq_wait(h_ready, t & 1, limit, err))) break;
         tc_fence_after();
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
+        for (int kk = 0; kk < UC / 16; ++kk) {
           const uint32_t cb = kk >> 2, w = kk & 3;
           const uint64_t da = umma_desc_sw128(sAtau + cb * 16384u) + 2ull * w;
 #pragma unroll
           for (int p = 0; p < 2; ++p) {
-            const uint64_t db = umma_desc_sw128(sBh + p * (NS * 256u) + cb * (NS * 128u)) + 2ull * w;
+            const uint64_t db = umma_desc_sw128(sBh + p * (NU * NS * 128u) + cb * (NS * 128u)) + 2ull * w;
             umma_bf16(tmem + tAcc, da, db, idesc, (kk | p) != 0 ? 1u : 0u);
           }
         }
@@ -195,14 +202,16 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
           const int s_end = c < ncut ? cut_sl[c] : nsl;
           for (; s < s_end; ++s)
 #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-              const uint64_t da = umma_desc_sw128(sAgate + g * 16384u) + 2ull * s;
+            for (int g = 0; g < 4; ++g)
 #pragma unroll
-              for (int p = 0; p < 2; ++p) {
-                const uint64_t db = umma_desc_sw128_sbo(sBtau + (2 * g + p) * 1024u, 8192u) + 2ull * s;
-                umma_bf16(tmem + tGate + g * NS, da, db, idesc, (s | p) != 0 ? 1u : 0u);
+              for (int m = 0; m < MT; ++m) {
+                const uint64_t da = umma_desc_sw64(sAgate + (g * MT + m) * 8192u, 512u) + 2ull * s;
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                  const uint64_t db = umma_desc_sw64(sBtau + (2 * g + p) * 512u, 4096u) + 2ull * s;
+                  umma_bf16(tmem + tGate + (g * MT + m) * NS, da, db, idesc, (s | p) != 0 ? 1u : 0u);
+                }
               }
-            }
           if (c < ncut) {  // partial sums at depth k_c: the epilogue runs the checkpoint cells
             umma_commit(ckpt_bar);
             ok = seq_wait(ckpt_done, (uint32_t)(t * ncut + c) & 1u, limit, err);
@@ -217,15 +226,17 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     }
   } else if (warp >= 4) {  // ---- epilogue: exchanges, tau', cells ----
     const int e = threadIdx.x - 128, ew = warp - 4, q = ew & 3, part = ew >> 2;
-    const int jl = 32 * q + lane, j = j0 + jl;  // this thread's hidden unit (tensor-memory lane)
     const uint32_t trow = tmem + ((32u * q) << 16);
-    float bias[4];
+    // this thread's hidden units jl = 128 m + 32 q + lane (tensor-memory lane 32 q + lane of unit tile m)
+    float bias[MT][4];
 #pragma unroll
-    for (int g = 0; g < 4; ++g) bias[g] = a.bias[g * H + j];
+    for (int m = 0; m < MT; ++m)
+#pragma unroll
+      for (int g = 0; g < 4; ++g) bias[m][g] = a.bias[g * H + j0 + 128 * m + 32 * q + lane];
     // owner elements: tau' of row (g, k) for stream rank*SP + sp, element
-    // i = row*SP + sp, taken by threads e, e + kSeqEpi, ...
+    // idx = row*SP + sp, taken by threads e, e + kSeqEpi, ...
     const int E = R4 * SP;
-    int r_at[kSeqMaxRed];  // byte offset in the tau' operand (hi plane) << 12 | offset in a source's RS block
+    int r_at[kSeqMaxRed];  // byte offset in the tau' operand (hi plane) << 12 | idx
     int r_p[kSeqMaxRed];   // offset of the element in P_t, or -1 (k >= K, or a stream past B)
     float r_sig[kSeqMaxRed];
 #pragma unroll
@@ -237,29 +248,32 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
       if (idx < E) {
         const int row = idx / SP, sp = idx - row * SP, g = row / rpg, k = row - g * rpg;
         const int nl = rank * SP + sp;
-        r_at[i] = (int)(((nl >> 3) * 8192u + (2u * g) * 1024u + sw128_offset(nl, k)) << 12) | idx;
+        r_at[i] = (int)(((nl >> 3) * 4096u + (2u * g) * 512u + sw64_offset(nl, k)) << 12) | idx;
         if (k < a.K) {
           r_sig[i] = a.sigma[g * a.Ks + k];
           if (n0 + nl < B) r_p[i] = (n0 + nl) * a.ldp + g * a.Ks + k;
         }
       }
     }
-    // h pair of (local stream nl, this unit) in the tau' product's operand
-    auto put_h = [&](int nl, float v) {
+    // h pair of (local stream nl, local unit jl) in the tau' product's operand
+    auto put_h = [&](int nl, int jl, float v) {
       __nv_bfloat16 hi, lo;
       seq_pair(v, hi, lo);
       const uint32_t o = (uint32_t)(jl >> 6) * (NS * 128u) + (uint32_t)(nl >> 3) * 1024u + sw128_offset(nl, jl & 63);
       *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o) = hi;
-      *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + NS * 256u + o) = lo;
+      *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + NU * NS * 128u + o) = lo;
     };
     griddep_wait();  // P, h0 and c0 may come from the kernels before this one
-    float c[SPW];
+    float c[MT][SPW];
 #pragma unroll
-    for (int s = 0; s < SPW; ++s) {
-      const int nl = part * SPW + s, n = n0 + nl;
-      c[s] = (a.c0 != nullptr && n < B) ? a.c0[(long long)n * H + j] : 0.f;
-      put_h(nl, (a.h0 != nullptr && n < B) ? a.h0[(long long)n * H + j] : 0.f);
-    }
+    for (int m = 0; m < MT; ++m)
+#pragma unroll
+      for (int s = 0; s < SPW; ++s) {
+        const int nl = part * SPW + s, n = n0 + nl, jl = 128 * m + 32 * q + lane;
+        const long long o = (long long)n * H + j0 + jl;
+        c[m][s] = (a.c0 != nullptr && n < B) ? a.c0[o] : 0.f;
+        put_h(nl, jl, (a.h0 != nullptr && n < B) ? a.h0[o] : 0.f);
+      }
     fence_proxy_async_shared();
     tc_fence_before();
     mbar_arrive(h_ready);
@@ -304,21 +318,20 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
         __nv_bfloat16 hi, lo;
         seq_pair(r_sig[i] != 0.f ? r_sig[i] * (sum + pv[i]) : 0.f, hi, lo);
         *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + (at >> 12)) = hi;
-        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + (at >> 12) + 1024) = lo;
+        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + (at >> 12) + 512) = lo;
       }
       fence_proxy_async_shared();
+      tc_fence_before();  // this thread's tensor-memory reads are done before the gate MMAs overwrite them
       mbar_arrive(red_done);
       // exchange 2: this CTA's block of tau' (its SP streams, all terms) -> every other CTA
-      if (e < (CS > 1 ? CS - 1 : 1)) {
+      if (e < CS - 1) {
         if (!seq_wait(red_done, t & 1, limit, err)) {
           atomicCAS(a.err, 0, kErrTcTimeout);
         } else {
-          if (e == 0) mbar_arrive_expect_tx(tau_full, (uint32_t)((CS - 1) * SP * 1024));
-          if (e < CS - 1) {
-            const int d = (rank + 1 + e) % CS;
-            const uint32_t src = sBtau + (uint32_t)rank * SP * 1024u;
-            bulk_copy_s2cluster(mapa_shared(src, d), src, (uint32_t)SP * 1024u, mapa_shared(tau_full, d));
-          }
+          if (e == 0) mbar_arrive_expect_tx(tau_full, (uint32_t)((CS - 1) * SP * 512));
+          const int d = (rank + 1 + e) % CS;
+          const uint32_t src = sBtau + (uint32_t)rank * SP * 512u;
+          bulk_copy_s2cluster(mapa_shared(src, d), src, (uint32_t)SP * 512u, mapa_shared(tau_full, d));
         }
       }
       // (a4, a6) cells: at each intermediate depth from the partial sums, then at full depth
@@ -329,39 +342,43 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
-        for (int i8 = 0; i8 < SPW / 8; ++i8) {
-          const int nl0 = part * SPW + 8 * i8;
-          float y[4][8];
-          tmem_ld8x4_sync(trow + tGate + nl0, trow + tGate + NS + nl0, trow + tGate + 2 * NS + nl0,
-                          trow + tGate + 3 * NS + nl0, y);
-          float hv[8], cv[8];
+        for (int m = 0; m < MT; ++m) {
+          const int jl = 128 * m + 32 * q + lane, j = j0 + jl;
 #pragma unroll
-          for (int k8 = 0; k8 < 8; ++k8)
-            lstm_cell_s(y[0][k8] + bias[0], y[1][k8] + bias[1], y[2][k8] + bias[2], y[3][k8] + bias[3],
-                        c[8 * i8 + k8], hv[k8], cv[k8]);
+          for (int i8 = 0; i8 < SPW / 8; ++i8) {
+            const int nl0 = part * SPW + 8 * i8;
+            const uint32_t tc0 = trow + tGate + m * NS + nl0;
+            float y[4][8];
+            tmem_ld8x4_sync(tc0, tc0 + MT * NS, tc0 + 2 * MT * NS, tc0 + 3 * MT * NS, y);
+            float hv[8], cv[8];
 #pragma unroll
-          for (int k8 = 0; k8 < 8; ++k8) {
-            const int nl = nl0 + k8, n = n0 + nl;
-            const long long o = ((long long)t * B + n) * H + j;
-            if (!fin) {
+            for (int k8 = 0; k8 < 8; ++k8)
+              lstm_cell_s(y[0][k8] + bias[m][0], y[1][k8] + bias[m][1], y[2][k8] + bias[m][2],
+                          y[3][k8] + bias[m][3], c[m][8 * i8 + k8], hv[k8], cv[k8]);
+#pragma unroll
+            for (int k8 = 0; k8 < 8; ++k8) {
+              const int nl = nl0 + k8, n = n0 + nl;
+              const long long o = ((long long)t * B + n) * H + j;
+              if (!fin) {
+                if (n < B) {
+                  if (a.ckpt_h) a.ckpt_h[(long long)cj * a.ck_stride + o] = hv[k8];
+                  if (a.ckpt_c) a.ckpt_c[(long long)cj * a.ck_stride + o] = cv[k8];
+                }
+                continue;
+              }
+              c[m][8 * i8 + k8] = cv[k8];
+              put_h(nl, jl, hv[k8]);
               if (n < B) {
-                if (a.ckpt_h) a.ckpt_h[(long long)cj * a.ck_stride + o] = hv[k8];
-                if (a.ckpt_c) a.ckpt_c[(long long)cj * a.ck_stride + o] = cv[k8];
+                if (a.out_h) a.out_h[o] = hv[k8];
+                if (a.seq_bf16) {
+                  __nv_bfloat16 hi, lo;
+                  seq_pair(hv[k8], hi, lo);
+                  const long long so = ((long long)t * B + n) * a.ldh + j;
+                  a.seq_bf16[so] = hi;
+                  a.seq_bf16[a.seq_plane + so] = lo;
+                }
+                if (a.c_last && t == T - 1) a.c_last[(long long)n * H + j] = cv[k8];
               }
-              continue;
-            }
-            c[8 * i8 + k8] = cv[k8];
-            put_h(nl, hv[k8]);
-            if (n < B) {
-              if (a.out_h) a.out_h[o] = hv[k8];
-              if (a.seq_bf16) {
-                __nv_bfloat16 hi, lo;
-                seq_pair(hv[k8], hi, lo);
-                const long long so = ((long long)t * B + n) * a.ldh + j;
-                a.seq_bf16[so] = hi;
-                a.seq_bf16[a.seq_plane + so] = lo;
-              }
-              if (a.c_last && t == T - 1) a.c_last[(long long)n * H + j] = cv[k8];
             }
           }
         }
@@ -390,10 +407,10 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
   }
 }
 
-template <int NS>
-cudaError_t launch_seq_t(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, cudaStream_t s) {
-  auto kern = tc_seq_kernel<NS>;
-  const size_t smem = seq_layout(NS, 128).total;  // the largest layout of this NS
+template <int NS, int MT>
+cudaError_t launch_seq_t(const TcMap& Vh_p, const TcMap& U64, const TcSeqArgs& a, cudaStream_t s) {
+  auto kern = tc_seq_kernel<NS, MT>;
+  const size_t smem = seq_layout(NS, MT, 128).total;  // the largest layout of this kernel
   static thread_local bool attr = false;
   if (!attr) {
     const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -403,7 +420,7 @@ cudaError_t launch_seq_t(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.cs, (a.B + NS - 1) / NS);
   cfg.blockDim = dim3(kSeqThreads);
-  cfg.dynamicSmemBytes = seq_layout(NS, 4 * a.rpg).total;
+  cfg.dynamicSmemBytes = seq_layout(NS, MT, 4 * a.rpg).total;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
@@ -415,34 +432,43 @@ cudaError_t launch_seq_t(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, 
   cfg.attrs = attrs;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, *reinterpret_cast<const CUtensorMap*>(Vh_p.bytes),
-                            *reinterpret_cast<const CUtensorMap*>(U.bytes), a);
+                            *reinterpret_cast<const CUtensorMap*>(U64.bytes), a);
 }
 
 }  // namespace
 
-bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, std::string* why) {
+bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, int* mt, std::string* why) {
   auto no = [&](const char* w) {
     if (why) *why = w;
     return false;
   };
   if (K > 32) return no("K above 32 (the factors of a CTA's units would not fit in shared memory)");
-  if (H % (int)kUnits != 0) return no("H not a multiple of 128");
-  const int cs = H / (int)kUnits;
-  if (cs != 2 && cs != 4 && cs != 8) return no("H / 128 not 2, 4 or 8");
   for (int j = 0; j < ck.n; ++j)
     if (ck.k[j] % 16 != 0 && ck.k[j] < K) return no("an intermediate depth off the 16-term slices");
-  // 32 streams per tile where each CTA still owns at least 8 streams and the
-  // clusters fit in one wave; else 64.  A CTA owns 8 or 16 streams, so its
-  // tau' block (at most 128 rows x 16 streams) takes kSeqMaxRed elements per
-  // epilogue thread at most.
-  int n = 64;
-  if (cs == 2 || (cs == 4 && (long long)((B + 31) / 32) * cs <= 148)) n = 32;
-  *ns = n;
-  return true;
+  // tiles of 32 streams over clusters of 4 (or 2) CTAs where they fit in one
+  // wave; each CTA owns 8 or 16 streams of a tile, so its tau' block (at
+  // most 128 rows x 16 streams) takes kSeqMaxRed elements per epilogue
+  // thread at most
+  const long long tiles32 = (B + 31) / 32;
+  switch (H) {
+    case 256: *ns = 32; *mt = 1; return true;                      // 2 CTAs x 128 units
+    case 512: *ns = tiles32 <= kSeqMaxClusters4 ? 32 : 64; *mt = 1; return true;  // 4 x 128
+    case 1024:
+      if (tiles32 <= kSeqMaxClusters4) {
+        *ns = 32;
+        *mt = 2;  // 4 CTAs x 256 units
+      } else {
+        *ns = 64;
+        *mt = 1;  // 8 CTAs x 128 units
+      }
+      return true;
+    default: return no("H not 256, 512 or 1024");
+  }
 }
 
-cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U, const TcSeqArgs& a, int ns, cudaStream_t s) {
-  return ns == 32 ? launch_seq_t<32>(Vh_p, U, a, s) : launch_seq_t<64>(Vh_p, U, a, s);
+cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U64, const TcSeqArgs& a, int ns, int mt, cudaStream_t s) {
+  if (mt == 2) return launch_seq_t<32, 2>(Vh_p, U64, a, s);
+  return ns == 32 ? launch_seq_t<32, 1>(Vh_p, U64, a, s) : launch_seq_t<64, 1>(Vh_p, U64, a, s);
 }
 
 }  // namespace lstm_approx_impl

@@ -308,7 +308,8 @@ int ensure_factor_maps(lstm_approx_t* h, int l) {
   const uint64_t rows = 4ull * h->Ks;
   if (!tc_make_map(&s.map_vx, s.Vx, s.D, rows, (uint64_t)s.ldx * 2, 128) ||
       !tc_make_map(&s.map_vh, s.Vh, h->H, rows, (uint64_t)h->ldh * 2, 128) ||
-      !tc_make_map(&s.map_u, s.U, h->Ks, 4ull * h->H, (uint64_t)h->Ks * 2, 128))
+      !tc_make_map(&s.map_u, s.U, h->Ks, 4ull * h->H, (uint64_t)h->Ks * 2, 128) ||
+      !tc_make_map(&s.map_u64, s.U, h->Ks, 4ull * h->H, (uint64_t)h->Ks * 2, 128, 64))
     return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for layer %d factors", l);
   for (int i = 0; i < 3; ++i)
     if (!tc_make_map(&s.map_vx_p[i], s.Vx, s.D, rows, (uint64_t)s.ldx * 2, 8u << i) ||
@@ -374,9 +375,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   __nv_bfloat16* hb = static_cast<__nv_bfloat16*>(h->h_bf16);
   __nv_bfloat16* tau = static_cast<__nv_bfloat16*>(h->tau);
   float* cs = h->c_state + (size_t)l * h->max_batch * H;
-  int ns = 0;
+  int ns = 0, utiles = 0;
   if (h->opt_tensor_seq == 0 && h->opt_tau_layout == 0 && (long long)B * ldp < (1LL << 31) &&
-      tc_seq_fits(H, B, K, ck, &ns, nullptr)) {
+      tc_seq_fits(H, B, K, ck, &ns, &utiles, nullptr)) {
     // one launch per tile of streams for all T timesteps
     TcSeqArgs qa{};
     qa.H = H;
@@ -385,7 +386,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     qa.B = B;
     qa.T = T;
     qa.rpg = rpg;
-    qa.cs = H / 128;
+    qa.cs = H / (128 * utiles);
     qa.P = h->Px;
     qa.ldp = (int)ldp;
     qa.sigma = s.sigma;
@@ -405,7 +406,7 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     qa.limit_ns = limit_ns;
     qa.test_stall = h->opt_test_stall;
     h->opt_test_stall = 0;
-    LA_CUDA(h, launch_tc_seq(s.map_vh_p[pi], s.map_u, qa, ns, h->stream), "recurrence launch");
+    LA_CUDA(h, launch_tc_seq(s.map_vh_p[pi], s.map_u64, qa, ns, utiles, h->stream), "recurrence launch");
     h->launches += 1;
     h->last_tensor_seq = 1;
     return LSTM_APPROX_OK;
@@ -1197,10 +1198,10 @@ int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int* chec
       v[LSTM_APPROX_PLAN_TMEM_COLUMNS] = pc.ag.tcols;
     }
   } else if (path == LSTM_APPROX_PATH_TENSOR) {
-    int ns = 0;
-    if (tc_seq_fits(hidden, B, K, ck, &ns, nullptr)) {
+    int ns = 0, mt = 0;
+    if (tc_seq_fits(hidden, B, K, ck, &ns, &mt, nullptr)) {
       v[LSTM_APPROX_PLAN_TENSOR_SEQ] = 1;
-      v[LSTM_APPROX_PLAN_CLUSTER] = hidden / 128;
+      v[LSTM_APPROX_PLAN_CLUSTER] = hidden / (128 * mt);
       v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = ns;
       v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = ns;
       v[LSTM_APPROX_PLAN_GATE_SPLITS] = 1;

@@ -445,6 +445,28 @@ __host__ __device__ __forceinline__ uint32_t sw128_offset(int r, int k) {
   return static_cast<uint32_t>((r & 7) * 128 + ((((k >> 3) ^ r) & 7) << 4) + (k & 7) * 2);
 }
 
+// Shared-memory matrix descriptor of a K-major bf16 tile with 64-byte
+// swizzling: rows of 32 elements (64 B), 8-row groups `sbo` bytes apart
+// (512 when dense).  The tile starts on a 512-byte boundary; advancing by 16
+// elements inside the row adds 32 B to the start address.
+__device__ __forceinline__ uint64_t umma_desc_sw64(uint32_t saddr, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;  // 64-byte swizzle
+  return d;
+}
+
+// Byte offset of bf16 element k (< 32) of row r in a K-major tile of 64-byte
+// rows with 64-byte swizzling, relative to the 512-byte aligned group of 8
+// rows: the 16-byte chunk index (2 bits) is XORed with address bits 7-8,
+// which within the group are (r mod 8) / 2.
+__host__ __device__ __forceinline__ uint32_t sw64_offset(int r, int k) {
+  return static_cast<uint32_t>((r & 7) * 64 + ((((k >> 3) ^ ((r & 7) >> 1)) & 3) << 4) + (k & 7) * 2);
+}
+
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 D, both
 // operands K-major, M x N.
 __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {

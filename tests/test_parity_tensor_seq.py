@@ -41,8 +41,9 @@ def _sample(got, streams):
     (48, 256, 4, 37, 8, 60, [8]),            # ragged second tile; K = 8 (8 packed rows per gate), depth = K
     (96, 512, 3, 100, 32, 150, [16, 32]),    # 4 CTAs x 8 streams, ragged fourth tile, depths on the slices
     (40, 512, 2, 5, 17, 70, [16, 17]),       # 32 packed rows per gate, K and a depth off the slices
-    (64, 1024, 3, 70, 32, 200, [16]),        # 8 CTAs x 8 streams (64 per tile), ragged second tile
+    (64, 1024, 3, 70, 32, 200, [16]),        # 4 CTAs x 256 units x 8 streams, ragged third tile
     (72, 1024, 2, 64, 1, 30, []),            # one term
+    (56, 1024, 2, 40, 8, 50, [8]),           # 256 units per CTA with 8 packed rows per gate
 ])
 def test_seq_kernel_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     gates = _gates(H, D + H, K, nz, 7100 + H + K)
@@ -59,16 +60,19 @@ def test_seq_kernel_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     assert_parity(got, step, BF16_TOL)
 
 
-def test_seq_kernel_wide_tiles_at_h512(cuda_device):
-    """H = 512 with more streams than one wave of 32-stream tiles holds:
-    64 streams per tile, 16 per CTA; sampled streams."""
-    D, H, T, B, K = 32, 512, 2, 1300, 32
-    assert plan(BF16, H, T, B, K)["tau_tile_streams"] == 64
+@pytest.mark.parametrize("H,B,cs", [(512, 1300, 4), (1024, 1200, 8)])
+def test_seq_kernel_wide_tiles(cuda_device, H, B, cs):
+    """More streams than one wave of 32-stream tiles holds: 64 streams per
+    tile (H = 512: 16 per CTA of 128 units; H = 1024: 8 per CTA, on clusters
+    of 8 CTAs of 128 units instead of 4 of 256); sampled streams."""
+    D, T, K = 32, 2, 32
+    p = plan(BF16, H, T, B, K)
+    assert (p["tau_tile_streams"], p["cluster"]) == (64, cs)
     gates = _gates(H, D + H, K, 100, 7300)
     x = draw_inputs(T, B, D, "uniform", 73)
     got, m = run_gpu([gates], x, K, dtype="bf16", checkpoints=[16])
     assert m.query(Q_TENSOR_SEQ) == 1
-    streams = [0, 15, 16, 700, 1299]
+    streams = [0, 15, 16, 700, B - 1]
     ref = oracle_run([gates], x[:, streams], K, dtype="bf16", checkpoints=[16])
     assert_parity(_sample(got, streams), ref, BF16_TOL)
 

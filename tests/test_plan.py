@@ -163,13 +163,14 @@ def test_tensor_tiles(H, B, K):
 @pytest.mark.parametrize("H,B", [(256, 1), (256, 3000), (512, 256), (512, 1300), (1024, 1024), (1024, 5)])
 @pytest.mark.parametrize("K", [1, 8, 16, 17, 32])
 def test_tensor_seq_plan(H, B, K):
-    """One launch per tile of streams for all timesteps: a cluster of H / 128
-    CTAs per tile; 32 streams per tile at H = 256, and at H = 512 while the
-    clusters fit in one wave of 148 CTAs, else 64 (each CTA owns 8 or 16
-    streams)."""
+    """One launch per tile of streams for all timesteps: tiles of 32 streams
+    on clusters of 4 CTAs (H = 512: 128 units each; H = 1024: 256) while the
+    clusters fit in one wave (36 clusters of 4 on the GPU), else 64 streams
+    (H = 1024: on clusters of 8 CTAs of 128 units); H = 256: 2 CTAs, 32
+    streams.  Each CTA owns 8 or 16 streams of a tile."""
     p = plan(BF16, H, 2, B, K)
-    cs = H // 128
-    ns = 32 if cs == 2 or (cs == 4 and -(-B // 32) * cs <= 148) else 64
+    one_wave = -(-B // 32) <= 36
+    cs, ns = {256: (2, 32), 512: (4, 32 if one_wave else 64), 1024: (4, 32) if one_wave else (8, 64)}[H]
     assert (p["tensor_seq"], p["cluster"], p["tau_tile_streams"], p["gate_tile_streams"], p["gate_splits"]) == \
         (1, cs, ns, ns, 1)
     assert ns // cs in (8, 16)
