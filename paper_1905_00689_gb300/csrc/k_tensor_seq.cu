@@ -51,7 +51,7 @@ using namespace lstm_approx_dev;
 
 constexpr int kSeqEpw = 4;                 // epilogue warps per 32-lane quarter of tensor memory
 constexpr int kSeqEpi = 4 * kSeqEpw * 32;  // epilogue threads
-constexpr int kSeqThreads = 128 + kSeqEpi; // warp 0: TMA and MMA issue, warp 1: tensor memory, 2-3 idle
+constexpr int kSeqThreads = 64 + kSeqEpi;  // warp 0: TMA and MMA issue, warp 1: tensor memory, 2..17 epilogue
 constexpr int kSeqMaxRed = 4;              // owner elements (tau' values) per epilogue thread at most
 constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident at once on a GB300 (152 SMs)
 
@@ -59,10 +59,15 @@ constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident a
 // tiles per CTA, NS streams, 4 rpg packed rows):
 //   Atau  [2 MT unit blocks of 64][128 rows][128 B]        128-byte swizzle
 //   Agate [4 gates][MT][128 units][64 B] (terms 0..31)     64-byte swizzle
-//   Bh    [2 planes][2 MT unit blocks of 64][NS streams][128 B]
-//   Btau  [NS/8 stream groups][4 gates][2 planes][8 streams][64 B]   64-byte swizzle
+//   Bh    [2 MT unit blocks of 64][NS/8 stream groups][2 planes][8 streams][128 B]
+//   Btau  [NS/8 stream groups][2 planes][4 gates][8 streams][64 B]   64-byte swizzle
 //   RS    [CS sources][4 rpg rows][SP streams] fp32 partial tau'
 //   barriers, tensor-memory slot
+// The activation operands interleave the two planes of the pair by groups of
+// 8 streams, so that one MMA of N = 2 NS rows (hi, lo, hi, lo, ... groups at
+// a uniform stride) multiplies a factor tile by both planes: the factor tile
+// is read once, and the accumulator holds the hi and lo products of stream
+// group G in columns [16 G, 16 G + 8) and [16 G + 8, 16 G + 16).
 struct SeqLayout {
   uint32_t agate, bh, btau, rs, bar, total;
 };
@@ -98,10 +103,10 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
   constexpr int SPW = NS / kSeqEpw;  // streams per epilogue warp
   constexpr int UC = 128 * MT;       // hidden units per CTA
   constexpr int NU = UC / 64;        // 64-unit blocks (K-dim tiles of the tau' product)
-  // tensor memory: the gate accumulators (gate g, unit tile m at column (g MT + m) NS); the
-  // tau' accumulator shares the first NS columns (it is read before the gate MMAs start,
-  // and they are read before the next tau' MMAs start)
-  constexpr uint32_t kUsed = 4u * MT * NS;
+  // tensor memory: the gate accumulators (gate g, unit tile m: 2 NS columns at (g MT + m) 2 NS);
+  // the tau' accumulator shares the first 2 NS columns (it is read before the gate MMAs
+  // start, and they are read before the next tau' MMAs start)
+  constexpr uint32_t kUsed = 8u * MT * NS;
   constexpr uint32_t kCols = kUsed <= 256 ? 256 : 512;
   constexpr uint32_t tAcc = 0, tGate = 0;
   const int CS = a.cs, SP = NS / CS, rpg = a.rpg, R4 = 4 * rpg;
@@ -178,20 +183,17 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
         for (int m = 0; m < MT; ++m)
           tma_load_2d(sAgate + (g * MT + m) * 8192u, &tmu, fac_full, 0, g * H + j0 + 128 * m);
       bool ok = seq_wait(fac_full, 0, limit, err);
-      constexpr uint32_t idesc = umma_idesc_bf16(128, NS);
+      constexpr uint32_t idesc = umma_idesc_bf16(128, 2 * NS);  // both planes of the activation
       for (int t = 0; t < T && ok; ++t) {
-        // (a2) partial tau' of this CTA's units: UC / 16 slices x both planes of h_{t-1}
+        // (a2) partial tau' of this CTA's units: UC / 16 slices, both planes of h_{t-1} at once
         if (!(ok = seq_wait(h_ready, t & 1, limit, err))) break;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < UC / 16; ++kk) {
           const uint32_t cb = kk >> 2, w = kk & 3;
           const uint64_t da = umma_desc_sw128(sAtau + cb * 16384u) + 2ull * w;
-#pragma unroll
-          for (int p = 0; p < 2; ++p) {
-            const uint64_t db = umma_desc_sw128(sBh + p * (NU * NS * 128u) + cb * (NS * 128u)) + 2ull * w;
-            umma_bf16(tmem + tAcc, da, db, idesc, (kk | p) != 0 ? 1u : 0u);
-          }
+          const uint64_t db = umma_desc_sw128(sBh + cb * (2u * NS * 128u)) + 2ull * w;
+          umma_bf16(tmem + tAcc, da, db, idesc, kk != 0 ? 1u : 0u);
         }
         umma_commit(tacc_full);
         // (a3) the four gate sums once every CTA's tau' block has landed
@@ -202,16 +204,14 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
           const int s_end = c < ncut ? cut_sl[c] : nsl;
           for (; s < s_end; ++s)
 #pragma unroll
-            for (int g = 0; g < 4; ++g)
+            for (int g = 0; g < 4; ++g) {
+              const uint64_t db = umma_desc_sw64(sBtau + g * 512u, 2048u) + 2ull * s;
 #pragma unroll
               for (int m = 0; m < MT; ++m) {
                 const uint64_t da = umma_desc_sw64(sAgate + (g * MT + m) * 8192u, 512u) + 2ull * s;
-#pragma unroll
-                for (int p = 0; p < 2; ++p) {
-                  const uint64_t db = umma_desc_sw64(sBtau + (2 * g + p) * 512u, 4096u) + 2ull * s;
-                  umma_bf16(tmem + tGate + (g * MT + m) * NS, da, db, idesc, (s | p) != 0 ? 1u : 0u);
-                }
+                umma_bf16(tmem + tGate + (g * MT + m) * 2 * NS, da, db, idesc, s != 0 ? 1u : 0u);
               }
+            }
           if (c < ncut) {  // partial sums at depth k_c: the epilogue runs the checkpoint cells
             umma_commit(ckpt_bar);
             ok = seq_wait(ckpt_done, (uint32_t)(t * ncut + c) & 1u, limit, err);
@@ -224,8 +224,9 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
       umma_commit(drain_bar);  // every MMA issued has completed before tensor memory is freed
       seq_wait(drain_bar, 0, limit, err);
     }
-  } else if (warp >= 4) {  // ---- epilogue: exchanges, tau', cells ----
-    const int e = threadIdx.x - 128, ew = warp - 4, q = ew & 3, part = ew >> 2;
+  } else if (warp >= 2) {  // ---- epilogue: exchanges, tau', cells ----
+    // warp w reads tensor-memory lanes [32 (w mod 4), +32); four warps per quarter
+    const int e = threadIdx.x - 64, q = warp & 3, part = (warp - 2) >> 2;
     const uint32_t trow = tmem + ((32u * q) << 16);
     // this thread's hidden units jl = 128 m + 32 q + lane (tensor-memory lane 32 q + lane of unit tile m)
     float bias[MT][4];
@@ -234,34 +235,32 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 #pragma unroll
       for (int g = 0; g < 4; ++g) bias[m][g] = a.bias[g * H + j0 + 128 * m + 32 * q + lane];
     // owner elements: tau' of row (g, k) for stream rank*SP + sp, element
-    // idx = row*SP + sp, taken by threads e, e + kSeqEpi, ...
+    // idx = row*SP + sp, taken by threads e, e + kSeqEpi, ... (recomputed
+    // each step: SP and rpg are powers of two)
     const int E = R4 * SP;
-    int r_at[kSeqMaxRed];  // byte offset in the tau' operand (hi plane) << 12 | idx
-    int r_p[kSeqMaxRed];   // offset of the element in P_t, or -1 (k >= K, or a stream past B)
-    float r_sig[kSeqMaxRed];
-#pragma unroll
-    for (int i = 0; i < kSeqMaxRed; ++i) {
-      const int idx = e + i * kSeqEpi;
-      r_at[i] = 0;
-      r_p[i] = -1;
-      r_sig[i] = 0.f;
-      if (idx < E) {
-        const int row = idx / SP, sp = idx - row * SP, g = row / rpg, k = row - g * rpg;
-        const int nl = rank * SP + sp;
-        r_at[i] = (int)(((nl >> 3) * 4096u + (2u * g) * 512u + sw64_offset(nl, k)) << 12) | idx;
-        if (k < a.K) {
-          r_sig[i] = a.sigma[g * a.Ks + k];
-          if (n0 + nl < B) r_p[i] = (n0 + nl) * a.ldp + g * a.Ks + k;
-        }
-      }
-    }
+    const int sp_sh = SP == 8 ? 3 : 4, rpg_sh = rpg == 8 ? 3 : (rpg == 16 ? 4 : 5);
+    struct Owned {
+      int bt;   // byte offset in the tau' operand (hi plane)
+      int pc;   // offset in P_t, or -1 (k >= K, or a stream past B)
+      int sc;   // column of sigma
+    };
+    auto owned = [&](int idx) {
+      const int row = idx >> sp_sh, sp = idx & (SP - 1), g = row >> rpg_sh, k = row & (rpg - 1);
+      const int nl = rank * SP + sp;
+      Owned o;
+      o.bt = (int)((nl >> 3) * 4096u + g * 512u + sw64_offset(nl, k));
+      o.sc = k < a.K ? g * a.Ks + k : -1;
+      o.pc = (k < a.K && n0 + nl < B) ? (n0 + nl) * a.ldp + g * a.Ks + k : -1;
+      return o;
+    };
     // h pair of (local stream nl, local unit jl) in the tau' product's operand
     auto put_h = [&](int nl, int jl, float v) {
       __nv_bfloat16 hi, lo;
       seq_pair(v, hi, lo);
-      const uint32_t o = (uint32_t)(jl >> 6) * (NS * 128u) + (uint32_t)(nl >> 3) * 1024u + sw128_offset(nl, jl & 63);
+      const uint32_t o =
+          (uint32_t)(jl >> 6) * (2u * NS * 128u) + (uint32_t)(nl >> 3) * 2048u + sw128_offset(nl, jl & 63);
       *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o) = hi;
-      *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + NU * NS * 128u + o) = lo;
+      *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o + 1024u) = lo;
     };
     griddep_wait();  // P, h0 and c0 may come from the kernels before this one
     float c[MT][SPW];
@@ -283,7 +282,10 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     for (int t = 0; t < T && ok; ++t) {
       float pv[kSeqMaxRed];
 #pragma unroll
-      for (int i = 0; i < kSeqMaxRed; ++i) pv[i] = r_p[i] >= 0 ? __ldg(a.P + (long long)t * B * a.ldp + r_p[i]) : 0.f;
+      for (int i = 0; i < kSeqMaxRed; ++i) {
+        const int idx = e + i * kSeqEpi, pc = idx < E ? owned(idx).pc : -1;
+        pv[i] = pc >= 0 ? __ldg(a.P + (long long)t * B * a.ldp + pc) : 0.f;
+      }
       if (e == 0) mbar_arrive_expect_tx(rs_full, (uint32_t)(CS * srcs * 4));
       // exchange 1: this CTA's partial tau' of each stream -> the stream's owner
       ok = __all_sync(0xffffffffu, seq_wait(tacc_full, t & 1, limit, err));
@@ -295,8 +297,10 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 #pragma unroll
         for (int i8 = 0; i8 < SPW / 8; ++i8) {
           const int c8 = part * SPW + 8 * i8;
-          float v[8];
-          tmem_ld8_sync(trow + tAcc + c8, v);
+          float hl[16], v[8];  // the group's hi products, then its lo products
+          tmem_ld16_sync(trow + tAcc + 2 * c8, hl);
+#pragma unroll
+          for (int k8 = 0; k8 < 8; ++k8) v[k8] = hl[k8] + hl[8 + k8];
 #pragma unroll
           for (int h4 = 0; h4 < 2; ++h4) {
             const int col = c8 + 4 * h4, d = col / SP, sp = col - d * SP;
@@ -311,14 +315,15 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
       if (!ok) break;
 #pragma unroll
       for (int i = 0; i < kSeqMaxRed; ++i) {
-        if (e + i * kSeqEpi >= E) break;
+        const int idx = e + i * kSeqEpi;
+        if (idx >= E) break;
+        const Owned o = owned(idx);
         float sum = 0.f;
-        const int at = r_at[i];
-        for (int src = 0; src < CS; ++src) sum += rsb[src * srcs + (at & 4095)];
+        for (int src = 0; src < CS; ++src) sum += rsb[src * srcs + idx];
         __nv_bfloat16 hi, lo;
-        seq_pair(r_sig[i] != 0.f ? r_sig[i] * (sum + pv[i]) : 0.f, hi, lo);
-        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + (at >> 12)) = hi;
-        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + (at >> 12) + 512) = lo;
+        seq_pair(o.sc >= 0 ? __ldg(a.sigma + o.sc) * (sum + pv[i]) : 0.f, hi, lo);
+        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + o.bt) = hi;
+        *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + o.bt + 2048) = lo;
       }
       fence_proxy_async_shared();
       tc_fence_before();  // this thread's tensor-memory reads are done before the gate MMAs overwrite them
@@ -347,9 +352,24 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 #pragma unroll
           for (int i8 = 0; i8 < SPW / 8; ++i8) {
             const int nl0 = part * SPW + 8 * i8;
-            const uint32_t tc0 = trow + tGate + m * NS + nl0;
+            // gate g's sums of this group: hi products at tc0 + g 2 MT NS, lo products 8 columns on
+            const uint32_t tc0 = trow + tGate + m * 2 * NS + 2 * nl0;
             float y[4][8];
-            tmem_ld8x4_sync(tc0, tc0 + MT * NS, tc0 + 2 * MT * NS, tc0 + 3 * MT * NS, y);
+            {
+              float a0[16], a1[16];
+              tmem_ld16x2_sync(tc0, tc0 + 2 * MT * NS, a0, a1);
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8) {
+                y[0][k8] = a0[k8] + a0[8 + k8];
+                y[1][k8] = a1[k8] + a1[8 + k8];
+              }
+              tmem_ld16x2_sync(tc0 + 4 * MT * NS, tc0 + 6 * MT * NS, a0, a1);
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8) {
+                y[2][k8] = a0[k8] + a0[8 + k8];
+                y[3][k8] = a1[k8] + a1[8 + k8];
+              }
+            }
             float hv[8], cv[8];
 #pragma unroll
             for (int k8 = 0; k8 < 8; ++k8)
