@@ -266,6 +266,13 @@ struct TcRowsArgs {
 };
 // `bn` (64, 128 or 256) must match the box rows of Bm's map.
 cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s);
+// The projection (mode 0) with packed gates from fp32 activations: Xf maps
+// the fp32 [N][Kdim] input in boxes of 32 columns x 64 rows (tc_make_map_f32),
+// and the kernel forms the bf16 pair itself (64 columns per tile).
+cudaError_t launch_tc_rows_xf32(const TcMap& A, const TcMap& Xf, const TcRowsArgs& a, int n_cols, cudaStream_t s);
+// 2-D fp32 tensor [rows][inner] as unswizzled TMA boxes of 32 inner elements x box_rows rows.
+bool tc_make_map_f32(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
+                     uint32_t box_rows);
 
 struct TcGatesArgs {
   int H, K, Ks, B;

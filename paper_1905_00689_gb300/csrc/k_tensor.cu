@@ -112,19 +112,28 @@ __device__ __forceinline__ float remainder_terms(const TcGatesArgs& a, int g, in
 // ---------------------------------------------------------------------------
 // tile of tau' / P: rows of the packed factor matrix x columns (streams)
 // ---------------------------------------------------------------------------
-template <int BN, int S>
+// XF (the projection, packed gates only): the activation comes as fp32
+// tiles (tmb is an fp32 map with boxes of 32 columns), and the epilogue
+// warps, idle until the accumulator is complete, convert each stage's tile
+// into its bf16 pair before the MMAs read it: x is read once from memory as
+// fp32 instead of being converted by a separate pass (which reads it and
+// writes its pair, the same bytes again).
+template <int BN, int S, bool XF>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_rows_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, TcRowsArgs a) {
   extern __shared__ uint8_t smem_raw[];
   static_assert(BN <= 128, "the epilogue holds P_t of its columns in registers");
   constexpr uint32_t kBBytes = BN * kTileK * 2;        // one plane of the activation tile
-  constexpr uint32_t kStage = kABytes + 2 * kBBytes;   // factor tile, hi plane, lo plane
+  constexpr uint32_t kRaw = XF ? BN * kTileK * 4 : 0;  // the fp32 activation tile: two boxes of 32 columns
+  constexpr uint32_t kStage = kABytes + 2 * kBBytes + kRaw;  // factor tile, hi plane, lo plane (fp32 tile)
   constexpr uint32_t kCols = BN < 32 ? 32 : BN;
+  constexpr int kNb = XF ? 3 * S : 2 * S;  // full[S] | empty[S] (| converted[S])
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t bar0 = base + S * kStage;  // full[S] | empty[S] | accum | drain | tmem slot
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (2 * S + 2));
-  const uint32_t accum_bar = bar0 + 8u * (2 * S), drain_bar = accum_bar + 8u;
+  const uint32_t bar0 = base + S * kStage;  // the stage barriers, accum | drain | tmem slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (kNb + 2));
+  const uint32_t accum_bar = bar0 + 8u * kNb, drain_bar = accum_bar + 8u;
+  const uint32_t conv0 = bar0 + 8u * (2 * S);  // converted[s] (XF)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = blockIdx.x / a.kt_per_gate, kt = blockIdx.x % a.kt_per_gate;
@@ -145,6 +154,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int i = 0; i < S; ++i) {
       mbar_init(bar0 + 8u * i, 1);
       mbar_init(bar0 + 8u * (S + i), 1);
+      if (XF) mbar_init(conv0 + 8u * i, 8 * 32);
     }
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
@@ -184,8 +194,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // the factor tiles of the first S stages do not depend on the kernel
     // before this one: issue them before waiting for it
     const int npre = nkb < S ? nkb : S;
+    constexpr uint32_t b_bytes = XF ? kRaw : 2 * kBBytes;
     for (int kb = 0; kb < npre; ++kb) {
-      mbar_arrive_expect_tx(bar0 + 8u * kb, a_bytes + 2 * kBBytes);
+      mbar_arrive_expect_tx(bar0 + 8u * kb, a_bytes + b_bytes);
       load_a(base + kb * kStage, bar0 + 8u * kb, kb);
     }
     griddep_wait();
@@ -194,11 +205,16 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
       const uint32_t st = base + s * kStage;
       if (kb >= npre) {
-        mbar_arrive_expect_tx(bar0 + 8u * s, a_bytes + 2 * kBBytes);
+        mbar_arrive_expect_tx(bar0 + 8u * s, a_bytes + b_bytes);
         load_a(st, bar0 + 8u * s, kb);
       }
-      tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);                      // hi plane
-      tma_load_2d(st + kABytes + kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, a.b_plane + col0);  // lo plane
+      if constexpr (XF) {  // the fp32 tile, columns [64 kb, 64 kb + 32) and [64 kb + 32, 64 kb + 64)
+        tma_load_2d(st + kABytes + 2 * kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
+        tma_load_2d(st + kABytes + 2 * kBBytes + BN * 128u, &tmb, bar0 + 8u * s, kb * kTileK + 32, col0);
+      } else {
+        tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);                      // hi plane
+        tma_load_2d(st + kABytes + kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, a.b_plane + col0);  // lo plane
+      }
       ++issued;
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
@@ -212,7 +228,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     bool ok = true;
     for (int kb = 0; kb < nkb && ok; ++kb) {
       const int s = kb % S;
-      if (!(ok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
+      // the stage's copies have landed (XF: and its activation has been converted)
+      if (!(ok = wait_cta((XF ? conv0 : bar0) + 8u * s, (kb / S) & 1, limit, err))) break;
       tc_fence_after();
       const uint32_t st = base + s * kStage;
       const uint64_t da = umma_desc_sw128(st);
@@ -231,6 +248,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp >= 4) {  // ---- epilogue: warps 4..11, two per lane quarter ----
     const int ep = warp - 4, q = ep & 3;
     constexpr int kHalf = BN / 2;
+    if constexpr (XF) {  // each stage's fp32 activation tile -> its bf16 pair, in the stage's B planes
+      const int ce = threadIdx.x - 128;
+      uint8_t* gbase = smem_raw + (base - raw);
+      bool cok = true;
+      for (int kb = 0; kb < nkb && cok; ++kb) {
+        const int s = kb % S;
+        if (!(cok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
+        uint8_t* st = gbase + s * kStage;
+        // 16 chunks of four columns per row: chunk c = row n, columns [4 (c mod 16), +4)
+        for (int c = ce; c < BN * 16; c += 256) {
+          const int n = c >> 4, k4 = (c & 15) * 4;
+          const float4 v = *reinterpret_cast<const float4*>(st + kABytes + 2 * kBBytes + (k4 >> 5) * (BN * 128) +
+                                                             n * 128 + (k4 & 31) * 4);
+          __nv_bfloat16 h[4], l[4];
+          bf16_pair(v.x, h[0], l[0]);
+          bf16_pair(v.y, h[1], l[1]);
+          bf16_pair(v.z, h[2], l[2]);
+          bf16_pair(v.w, h[3], l[3]);
+          const uint32_t o = sw128_offset(n, k4) + (uint32_t)(n >> 3) * 1024u;
+          *reinterpret_cast<uint2*>(st + kABytes + o) =
+              make_uint2((uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16),
+                         (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16));
+          *reinterpret_cast<uint2*>(st + kABytes + kBBytes + o) =
+              make_uint2((uint32_t)__bfloat16_as_ushort(l[0]) | ((uint32_t)__bfloat16_as_ushort(l[1]) << 16),
+                         (uint32_t)__bfloat16_as_ushort(l[2]) | ((uint32_t)__bfloat16_as_ushort(l[3]) << 16));
+        }
+        fence_proxy_async_shared();
+        mbar_arrive(conv0 + 8u * s);
+      }
+      if (!cok) atomicCAS(a.err, 0, kErrTcTimeout);
+    }
     const int cbeg = (ep >> 2) * kHalf;
     const int lrow = 32 * q + lane;
     const int k = rpg > 0 ? lrow % rpg : kt * kTileM + lrow;
@@ -707,20 +755,20 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args..
   return launch_pdl_block(kern, grid, dim3(kTcThreads), smem, s, args...);
 }
 
-template <int BN, int S>
+template <int BN, int S, bool XF>
 size_t rows_smem() {
-  return 1024 + S * (kABytes + 2 * BN * kTileK * 2) + 8 * (2 * S + 2) + 16;
+  return 1024 + S * (kABytes + 2 * BN * kTileK * 2 + (XF ? BN * kTileK * 4 : 0)) + 8 * ((XF ? 3 : 2) * S + 2) + 16;
 }
 template <int NT, int S>
 size_t gates_smem() {
   return 1024 + S * (kABytes + 2 * NT * kTileK * 2) + 8 * (2 * S + 4) + 16;
 }
 
-template <int BN, int S>
+template <int BN, int S, bool XF = false>
 cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
-  auto kern = tc_rows_kernel<BN, S>;
+  auto kern = tc_rows_kernel<BN, S, XF>;
   static thread_local bool attr = false;
-  const size_t smem = rows_smem<BN, S>();
+  const size_t smem = rows_smem<BN, S, XF>();
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -796,6 +844,26 @@ int tc_gates_tile_n(int H, int B) {
   for (int nt : {32, 64, 128})
     if ((long long)unit_tiles * ((B + nt - 1) / nt) <= 148) return nt;
   return 128;
+}
+
+cudaError_t launch_tc_rows_xf32(const TcMap& A, const TcMap& Xf, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
+  return launch_rows_t<64, 4, true>(A, Xf, a, n_cols, s);
+}
+
+bool tc_make_map_f32(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
+                     uint32_t box_rows) {
+  EncodeTiled enc = encoder();
+  if (!enc) return false;
+  std::memset(m->bytes, 0, sizeof(m->bytes));
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {pitch_bytes};
+  const cuuint32_t box[2] = {32u, box_rows};  // 128-byte rows, unswizzled
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(reinterpret_cast<CUtensorMap*>(m->bytes), CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+                         const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
 
 cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s) {

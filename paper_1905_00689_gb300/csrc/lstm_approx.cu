@@ -335,15 +335,18 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   // up to 32 terms the products take one tile of all four gates' rows
   const int rpg = tensor_rows_per_gate(K);
   const int pi = rpg == 8 ? 0 : (rpg == 16 ? 1 : 2);
-  __nv_bfloat16* in_bf16;
-  int ld_in;
-  if (l == 0) {  // operand conversion (outside the timed projection phase)
+  __nv_bfloat16* in_bf16 = nullptr;
+  int ld_in = 0;
+  // packed gates at layer 0: the projection reads x in fp32 and forms its
+  // bf16 pair itself (one tile of rows, so x is read once either way)
+  const bool x_f32 = l == 0 && rpg > 0 && D % 4 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  if (l == 0 && !x_f32) {  // operand conversion (outside the timed projection phase)
     LA_CUDA(h, launch_to_bf16(x, TB, D, static_cast<__nv_bfloat16*>(h->x_bf16), s.ldx, h->stream),
             "input conversion launch");
     in_bf16 = static_cast<__nv_bfloat16*>(h->x_bf16);
     ld_in = s.ldx;
     h->launches += 1;
-  } else {
+  } else if (l > 0) {
     in_bf16 = static_cast<__nv_bfloat16*>(h->seq_bf16);
     ld_in = h->ldh;
   }
@@ -352,8 +355,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     const int kt = (K + 127) / 128;
     const int bnx = tc_rows_tile_n(TB, rpg > 0 ? 1 : 4 * kt);
     TcMap mx;
-    if (!tc_make_map(&mx, in_bf16, D, 2ull * TB, (uint64_t)ld_in * 2, bnx))
-      return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
+    const bool mapped = x_f32 ? tc_make_map_f32(&mx, x, D, TB, (uint64_t)D * 4, 64)
+                              : tc_make_map(&mx, in_bf16, D, 2ull * TB, (uint64_t)ld_in * 2, bnx);
+    if (!mapped) return fail(h, LSTM_APPROX_ECUDA, "tensor map encoding failed for the layer input");
     TcRowsArgs ra{};
     ra.Kdim = D;
     ra.K = K;
@@ -367,8 +371,11 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.ldp = (int)ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
-    LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vx_p[pi] : s.map_vx, mx, ra, TB, bnx, h->stream),
-            "input projection launch");
+    if (x_f32)
+      LA_CUDA(h, launch_tc_rows_xf32(s.map_vx_p[pi], mx, ra, TB, h->stream), "input projection launch");
+    else
+      LA_CUDA(h, launch_tc_rows(rpg > 0 ? s.map_vx_p[pi] : s.map_vx, mx, ra, TB, bnx, h->stream),
+              "input projection launch");
     h->launches += 1;
   }
   PhaseTimer pt(h, 1);

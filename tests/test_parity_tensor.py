@@ -242,3 +242,26 @@ def test_compressed_tau_layout_refused_where_it_does_not_apply(cuda_device):
     with pytest.raises(LSTMApproxError):
         m.set_option(OPT_TAU_LAYOUT, 1)
     m.close()
+
+
+@pytest.mark.parametrize("D,offset", [(64, 0), (42, 0), (64, 1)])
+def test_projection_input_forms(cuda_device, D, offset):
+    """Up to K = 32 at layer 0 the projection reads x in fp32 and forms its
+    bf16 pair itself when D is a multiple of 4 and x is 16-byte aligned;
+    otherwise x goes through the separate conversion pass.  Both agree with
+    the oracle (offset = 1: x starts one float into its buffer)."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox
+    H, T, B, K = 256, 3, 20, 16
+    gates = [draw_factor_set(H, D + H, K, 70, 6600 + D + g) for g in range(4)]
+    x = draw_inputs(T, B, D, "uniform", 9)
+    m = LSTMApprox(1, [D], H, K, B, "bf16")
+    m.set_layer(0, gates)
+    buf = torch.zeros(T * B * D + 4, device="cuda")
+    xt = buf[offset:offset + T * B * D].view(T, B, D)
+    xt.copy_(torch.from_numpy(x.astype(np.float32)))
+    out = torch.empty((T, B, H), device="cuda")
+    m.run(xt, K, out)
+    m.sync()
+    ref = oracle_run([gates], x, K, dtype="bf16")
+    assert_parity({"h": out.double().cpu().numpy()}, ref, BF16_TOL, keys=("h",))
