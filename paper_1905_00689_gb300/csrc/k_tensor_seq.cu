@@ -49,9 +49,12 @@ namespace {
 
 using namespace lstm_approx_dev;
 
-constexpr int kSeqEpw = 4;                 // epilogue warps per 32-lane quarter of tensor memory
-constexpr int kSeqEpi = 4 * kSeqEpw * 32;  // epilogue threads
-constexpr int kSeqThreads = 64 + kSeqEpi;  // warp 0: TMA and MMA issue, warp 1: tensor memory, 2..17 epilogue
+// Threads: warp 0 issues the TMA copies and the MMAs, warp 1 owns tensor
+// memory, and 4 EPW epilogue warps follow (EPW per 32-lane quarter of tensor
+// memory, each taking 8 of the tile's streams per 128 units: 4 at NS >= 32,
+// 2 at NS = 16).
+__host__ __device__ constexpr int seq_epw(int ns) { return ns >= 32 ? 4 : 2; }
+__host__ __device__ constexpr int seq_threads(int ns) { return 64 + 4 * seq_epw(ns) * 32; }
 constexpr int kSeqMaxRed = 4;              // owner elements (tau' values) per epilogue thread at most
 constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident at once on a GB300 (152 SMs)
 
@@ -97,9 +100,11 @@ __device__ __forceinline__ void seq_pair(float v, __nv_bfloat16& hi, __nv_bfloat
 }
 
 template <int NS, int MT>
-__global__ void __launch_bounds__(kSeqThreads, 1)
+__global__ void __launch_bounds__(seq_threads(NS), 1)
     tc_seq_kernel(const __grid_constant__ CUtensorMap tmv, const __grid_constant__ CUtensorMap tmu, TcSeqArgs a) {
   extern __shared__ uint8_t smem_raw[];
+  constexpr int kSeqEpw = seq_epw(NS);
+  constexpr int kSeqEpi = 4 * kSeqEpw * 32;  // epilogue threads
   constexpr int SPW = NS / kSeqEpw;  // streams per epilogue warp
   constexpr int UC = 128 * MT;       // hidden units per CTA
   constexpr int NU = UC / 64;        // 64-unit blocks (K-dim tiles of the tau' product)
@@ -238,7 +243,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     // idx = row*SP + sp, taken by threads e, e + kSeqEpi, ... (recomputed
     // each step: SP and rpg are powers of two)
     const int E = R4 * SP;
-    const int sp_sh = SP == 8 ? 3 : 4, rpg_sh = rpg == 8 ? 3 : (rpg == 16 ? 4 : 5);
+    const int sp_sh = SP == 4 ? 2 : (SP == 8 ? 3 : 4), rpg_sh = rpg == 8 ? 3 : (rpg == 16 ? 4 : 5);
     struct Owned {
       int bt;   // byte offset in the tau' operand (hi plane)
       int pc;   // offset in P_t, or -1 (k >= K, or a stream past B)
@@ -328,15 +333,24 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
       fence_proxy_async_shared();
       tc_fence_before();  // this thread's tensor-memory reads are done before the gate MMAs overwrite them
       mbar_arrive(red_done);
-      // exchange 2: this CTA's block of tau' (its SP streams, all terms) -> every other CTA
-      if (e < CS - 1) {
+      // exchange 2: this CTA's block of tau' (its SP streams, all terms) -> every other CTA:
+      // one copy per peer of SP / 8 whole stream groups, or (SP = 4, half a group) eight
+      // 256-byte pieces per peer, one per (plane, gate)
+      const int ncopy = SP >= 8 ? CS - 1 : 8 * (CS - 1);
+      if (e < ncopy) {
         if (!seq_wait(red_done, t & 1, limit, err)) {
           atomicCAS(a.err, 0, kErrTcTimeout);
         } else {
           if (e == 0) mbar_arrive_expect_tx(tau_full, (uint32_t)((CS - 1) * SP * 512));
-          const int d = (rank + 1 + e) % CS;
-          const uint32_t src = sBtau + (uint32_t)rank * SP * 512u;
-          bulk_copy_s2cluster(mapa_shared(src, d), src, (uint32_t)SP * 512u, mapa_shared(tau_full, d));
+          if (SP >= 8) {
+            const int d = (rank + 1 + e) % CS;
+            const uint32_t src = sBtau + (uint32_t)rank * SP * 512u;
+            bulk_copy_s2cluster(mapa_shared(src, d), src, (uint32_t)SP * 512u, mapa_shared(tau_full, d));
+          } else {
+            const int d = (rank + 1 + (e >> 3)) % CS, piece = e & 7;  // piece = plane * 4 + gate
+            const uint32_t src = sBtau + (uint32_t)(rank >> 1) * 4096u + (uint32_t)piece * 512u + (rank & 1) * 256u;
+            bulk_copy_s2cluster(mapa_shared(src, d), src, 256u, mapa_shared(tau_full, d));
+          }
         }
       }
       // (a4, a6) cells: at each intermediate depth from the partial sums, then at full depth
@@ -439,7 +453,7 @@ cudaError_t launch_seq_t(const TcMap& Vh_p, const TcMap& U64, const TcSeqArgs& a
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.cs, (a.B + NS - 1) / NS);
-  cfg.blockDim = dim3(kSeqThreads);
+  cfg.blockDim = dim3(seq_threads(NS));
   cfg.dynamicSmemBytes = seq_layout(NS, MT, 4 * a.rpg).total;
   cfg.stream = s;
   cudaLaunchAttribute attrs[2];
@@ -465,21 +479,27 @@ bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, int* mt, s
   if (K > 32) return no("K above 32 (the factors of a CTA's units would not fit in shared memory)");
   for (int j = 0; j < ck.n; ++j)
     if (ck.k[j] % 16 != 0 && ck.k[j] < K) return no("an intermediate depth off the 16-term slices");
-  // tiles of 32 streams over clusters of 4 (or 2) CTAs where they fit in one
-  // wave; each CTA owns 8 or 16 streams of a tile, so its tau' block (at
-  // most 128 rows x 16 streams) takes kSeqMaxRed elements per epilogue
-  // thread at most
-  const long long tiles32 = (B + 31) / 32;
+  // the narrowest tiles (16, 32 streams) whose clusters of 4 (or 2) CTAs fit
+  // in one wave; each CTA owns 4, 8 or 16 streams of a tile, so its tau'
+  // block (at most 128 rows x 16 streams) takes kSeqMaxRed elements per
+  // epilogue thread at most
+  const long long tiles16 = (B + 15) / 16, tiles32 = (B + 31) / 32;
   switch (H) {
-    case 256: *ns = 32; *mt = 1; return true;                      // 2 CTAs x 128 units
-    case 512: *ns = tiles32 <= kSeqMaxClusters4 ? 32 : 64; *mt = 1; return true;  // 4 x 128
-    case 1024:
-      if (tiles32 <= kSeqMaxClusters4) {
+    case 256: *ns = tiles16 <= 2 * kSeqMaxClusters4 ? 16 : 32; *mt = 1; return true;  // 2 CTAs x 128 units
+    case 512:                                                                          // 4 x 128
+      *ns = tiles16 <= kSeqMaxClusters4 ? 16 : (tiles32 <= kSeqMaxClusters4 ? 32 : 64);
+      *mt = 1;
+      return true;
+    case 1024:  // 4 CTAs x 256 units (16 or 32 streams), else 8 x 128 (64 streams)
+      if (tiles16 <= kSeqMaxClusters4) {
+        *ns = 16;
+        *mt = 2;
+      } else if (tiles32 <= kSeqMaxClusters4) {
         *ns = 32;
-        *mt = 2;  // 4 CTAs x 256 units
+        *mt = 2;
       } else {
         *ns = 64;
-        *mt = 1;  // 8 CTAs x 128 units
+        *mt = 1;
       }
       return true;
     default: return no("H not 256, 512 or 1024");
@@ -487,8 +507,12 @@ bool tc_seq_fits(int H, int B, int K, const Checkpoints& ck, int* ns, int* mt, s
 }
 
 cudaError_t launch_tc_seq(const TcMap& Vh_p, const TcMap& U64, const TcSeqArgs& a, int ns, int mt, cudaStream_t s) {
-  if (mt == 2) return launch_seq_t<32, 2>(Vh_p, U64, a, s);
-  return ns == 32 ? launch_seq_t<32, 1>(Vh_p, U64, a, s) : launch_seq_t<64, 1>(Vh_p, U64, a, s);
+  if (mt == 2) return ns == 16 ? launch_seq_t<16, 2>(Vh_p, U64, a, s) : launch_seq_t<32, 2>(Vh_p, U64, a, s);
+  switch (ns) {
+    case 16: return launch_seq_t<16, 1>(Vh_p, U64, a, s);
+    case 32: return launch_seq_t<32, 1>(Vh_p, U64, a, s);
+    default: return launch_seq_t<64, 1>(Vh_p, U64, a, s);
+  }
 }
 
 }  // namespace lstm_approx_impl

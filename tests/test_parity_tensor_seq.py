@@ -37,11 +37,11 @@ def _sample(got, streams):
 
 
 @pytest.mark.parametrize("D,H,T,B,K,nz,cps", [
-    (64, 256, 3, 32, 16, 90, []),            # one tile: 2 CTAs x 16 streams
-    (48, 256, 4, 37, 8, 60, [8]),            # ragged second tile; K = 8 (8 packed rows per gate), depth = K
-    (96, 512, 3, 100, 32, 150, [16, 32]),    # 4 CTAs x 8 streams, ragged fourth tile, depths on the slices
+    (64, 256, 3, 32, 16, 90, []),            # two tiles of 2 CTAs x 8 streams
+    (48, 256, 4, 37, 8, 60, [8]),            # ragged third tile; K = 8 (8 packed rows per gate), depth = K
+    (96, 512, 3, 100, 32, 150, [16, 32]),    # 4 CTAs x 4 streams (half an 8-stream group), ragged tile, depths
     (40, 512, 2, 5, 17, 70, [16, 17]),       # 32 packed rows per gate, K and a depth off the slices
-    (64, 1024, 3, 70, 32, 200, [16]),        # 4 CTAs x 256 units x 8 streams, ragged third tile
+    (64, 1024, 3, 70, 32, 200, [16]),        # 4 CTAs x 256 units x 4 streams, ragged fifth tile
     (72, 1024, 2, 64, 1, 30, []),            # one term
     (56, 1024, 2, 40, 8, 50, [8]),           # 256 units per CTA with 8 packed rows per gate
 ])
@@ -60,19 +60,21 @@ def test_seq_kernel_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     assert_parity(got, step, BF16_TOL)
 
 
-@pytest.mark.parametrize("H,B,cs", [(512, 1300, 4), (1024, 1200, 8)])
-def test_seq_kernel_wide_tiles(cuda_device, H, B, cs):
-    """More streams than one wave of 32-stream tiles holds: 64 streams per
-    tile (H = 512: 16 per CTA of 128 units; H = 1024: 8 per CTA, on clusters
-    of 8 CTAs of 128 units instead of 4 of 256); sampled streams."""
+@pytest.mark.parametrize("H,B,cs,ns", [(512, 700, 4, 32), (512, 1300, 4, 64), (1024, 700, 4, 32),
+                                        (1024, 1200, 8, 64)])
+def test_seq_kernel_wide_tiles(cuda_device, H, B, cs, ns):
+    """More streams than one wave of narrower tiles holds: 32 streams per
+    tile (8 per CTA), then 64 (H = 512: 16 per CTA of 128 units; H = 1024:
+    8 per CTA, on clusters of 8 CTAs of 128 units instead of 4 of 256);
+    sampled streams."""
     D, T, K = 32, 2, 32
     p = plan(BF16, H, T, B, K)
-    assert (p["tau_tile_streams"], p["cluster"]) == (64, cs)
+    assert (p["tau_tile_streams"], p["cluster"]) == (ns, cs)
     gates = _gates(H, D + H, K, 100, 7300)
     x = draw_inputs(T, B, D, "uniform", 73)
     got, m = run_gpu([gates], x, K, dtype="bf16", checkpoints=[16])
     assert m.query(Q_TENSOR_SEQ) == 1
-    streams = [0, 15, 16, 700, B - 1]
+    streams = [0, 15, 16, B // 2 + 3, B - 1]
     ref = oracle_run([gates], x[:, streams], K, dtype="bf16", checkpoints=[16])
     assert_parity(_sample(got, streams), ref, BF16_TOL)
 

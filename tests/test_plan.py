@@ -160,20 +160,26 @@ def test_tensor_tiles(H, B, K):
         assert p["gate_splits"] == -(-chunks // per)  # no empty split
 
 
-@pytest.mark.parametrize("H,B", [(256, 1), (256, 3000), (512, 256), (512, 1300), (1024, 1024), (1024, 5)])
+@pytest.mark.parametrize("H,B", [(256, 1), (256, 3000), (512, 256), (512, 700), (512, 1300), (1024, 1024), (1024, 5),
+                                 (1024, 600)])
 @pytest.mark.parametrize("K", [1, 8, 16, 17, 32])
 def test_tensor_seq_plan(H, B, K):
-    """One launch per tile of streams for all timesteps: tiles of 32 streams
-    on clusters of 4 CTAs (H = 512: 128 units each; H = 1024: 256) while the
-    clusters fit in one wave (36 clusters of 4 on the GPU), else 64 streams
-    (H = 1024: on clusters of 8 CTAs of 128 units); H = 256: 2 CTAs, 32
-    streams.  Each CTA owns 8 or 16 streams of a tile."""
+    """One launch per tile of streams for all timesteps: the narrowest tiles
+    (16, then 32 streams) whose clusters fit in one wave (36 clusters of 4
+    CTAs, 72 of 2), else 64 streams.  H = 256: clusters of 2 CTAs of 128
+    units; H = 512: 4 of 128; H = 1024: 4 of 256 with 16 or 32 streams, or 8
+    of 128 with 64.  Each CTA owns 4, 8 or 16 streams of a tile."""
     p = plan(BF16, H, 2, B, K)
-    one_wave = -(-B // 32) <= 36
-    cs, ns = {256: (2, 32), 512: (4, 32 if one_wave else 64), 1024: (4, 32) if one_wave else (8, 64)}[H]
+    t16, t32 = -(-B // 16), -(-B // 32)
+    if H == 256:
+        cs, ns = 2, (16 if t16 <= 72 else 32)
+    elif H == 512:
+        cs, ns = 4, (16 if t16 <= 36 else 32 if t32 <= 36 else 64)
+    else:
+        cs, ns = (4, 16) if t16 <= 36 else (4, 32) if t32 <= 36 else (8, 64)
     assert (p["tensor_seq"], p["cluster"], p["tau_tile_streams"], p["gate_tile_streams"], p["gate_splits"]) == \
         (1, cs, ns, ns, 1)
-    assert ns // cs in (8, 16)
+    assert ns // cs in (4, 8, 16)
 
 
 @pytest.mark.parametrize("H,K,ck,seq", [
