@@ -49,14 +49,16 @@ namespace {
 
 using namespace lstm_approx_dev;
 
+
+constexpr int kSeqMaxRed = 4;              // owner elements (tau' values) per epilogue thread at most
+constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident at once on a GB300 (152 SMs)
+
 // Threads: warp 0 issues the TMA copies and the MMAs, warp 1 owns tensor
 // memory, and 4 EPW epilogue warps follow (EPW per 32-lane quarter of tensor
 // memory, each taking 8 of the tile's streams per 128 units: 4 at NS >= 32,
 // 2 at NS = 16).
 __host__ __device__ constexpr int seq_epw(int ns) { return ns >= 32 ? 4 : 2; }
 __host__ __device__ constexpr int seq_threads(int ns) { return 64 + 4 * seq_epw(ns) * 32; }
-constexpr int kSeqMaxRed = 4;              // owner elements (tau' values) per epilogue thread at most
-constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident at once on a GB300 (152 SMs)
 
 // Shared-memory layout, offsets from the 1024-byte aligned base (MT 128-unit
 // tiles per CTA, NS streams, 4 rpg packed rows):
@@ -65,6 +67,7 @@ constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident a
 //   Bh    [2 MT unit blocks of 64][NS/8 stream groups][2 planes][8 streams][128 B]
 //   Btau  [NS/8 stream groups][2 planes][4 gates][8 streams][64 B]   64-byte swizzle
 //   RS    [CS sources][4 rpg rows][SP streams] fp32 partial tau'
+//   Cst   [MT 8 streams-per-warp blocks][epilogue threads] fp32 c_{t-1} of each thread's cells
 //   barriers, tensor-memory slot
 // The activation operands interleave the two planes of the pair by groups of
 // 8 streams, so that one MMA of N = 2 NS rows (hi, lo, hi, lo, ... groups at
@@ -72,7 +75,7 @@ constexpr int kSeqMaxClusters4 = 36;       // clusters of 4 such CTAs resident a
 // is read once, and the accumulator holds the hi and lo products of stream
 // group G in columns [16 G, 16 G + 8) and [16 G + 8, 16 G + 16).
 struct SeqLayout {
-  uint32_t agate, bh, btau, rs, bar, total;
+  uint32_t agate, bh, btau, rs, cst, bar, total;
 };
 __host__ __device__ inline SeqLayout seq_layout(int ns, int mt, int r4) {
   SeqLayout l;
@@ -80,7 +83,9 @@ __host__ __device__ inline SeqLayout seq_layout(int ns, int mt, int r4) {
   l.bh = l.agate + 32768u * mt;
   l.btau = l.bh + (uint32_t)ns * 512u * mt;
   l.rs = l.btau + (uint32_t)ns * 512u;
-  l.bar = l.rs + (uint32_t)r4 * ns * 4u;
+  l.cst = l.rs + (uint32_t)r4 * ns * 4u;
+  // each epilogue thread's c: MT x (NS / EPW) values, EPW warps per quarter
+  l.bar = l.cst + (uint32_t)mt * (uint32_t)(ns / seq_epw(ns)) * (uint32_t)(4 * seq_epw(ns) * 32) * 4u;
   l.total = l.bar + 128u + 1024u;  // barriers and slot, alignment slack
   return l;
 }
@@ -106,6 +111,9 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
   constexpr int kSeqEpw = seq_epw(NS);
   constexpr int kSeqEpi = 4 * kSeqEpw * 32;  // epilogue threads
   constexpr int SPW = NS / kSeqEpw;  // streams per epilogue warp
+  // owner elements per epilogue thread at most: 4 rpg rows x SP streams over the
+  // epilogue threads; with 256 units per CTA the cluster has 4 CTAs and SP = NS / 4
+  constexpr int kMaxRed = MT == 2 ? (128 * (NS / 4) + kSeqEpi - 1) / kSeqEpi : kSeqMaxRed;
   constexpr int UC = 128 * MT;       // hidden units per CTA
   constexpr int NU = UC / 64;        // 64-unit blocks (K-dim tiles of the tau' product)
   // tensor memory: the gate accumulators (gate g, unit tile m: 2 NS columns at (g MT + m) 2 NS);
@@ -268,14 +276,15 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
       *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o + 1024u) = lo;
     };
     griddep_wait();  // P, h0 and c0 may come from the kernels before this one
-    float c[MT][SPW];
-#pragma unroll
+    // c_{t-1} of this thread's cell (m, stream s of its SPW): word (m SPW + s) kSeqEpi + e
+    float* cst = reinterpret_cast<float*>(gb + L.cst) + e;
+#pragma unroll 1
     for (int m = 0; m < MT; ++m)
-#pragma unroll
+#pragma unroll 1
       for (int s = 0; s < SPW; ++s) {
         const int nl = part * SPW + s, n = n0 + nl, jl = 128 * m + 32 * q + lane;
         const long long o = (long long)n * H + j0 + jl;
-        c[m][s] = (a.c0 != nullptr && n < B) ? a.c0[o] : 0.f;
+        cst[(m * SPW + s) * kSeqEpi] = (a.c0 != nullptr && n < B) ? a.c0[o] : 0.f;
         put_h(nl, jl, (a.h0 != nullptr && n < B) ? a.h0[o] : 0.f);
       }
     fence_proxy_async_shared();
@@ -285,9 +294,9 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
     const int srcs = R4 * SP;  // floats per source in the RS buffer
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
-      float pv[kSeqMaxRed];
+      float pv[kMaxRed];
 #pragma unroll
-      for (int i = 0; i < kSeqMaxRed; ++i) {
+      for (int i = 0; i < kMaxRed; ++i) {
         const int idx = e + i * kSeqEpi, pc = idx < E ? owned(idx).pc : -1;
         pv[i] = pc >= 0 ? __ldg(a.P + (long long)t * B * a.ldp + pc) : 0.f;
       }
@@ -319,7 +328,7 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
       ok = __all_sync(0xffffffffu, seq_wait_cluster(rs_full, t & 1, limit, err));
       if (!ok) break;
 #pragma unroll
-      for (int i = 0; i < kSeqMaxRed; ++i) {
+      for (int i = 0; i < kMaxRed; ++i) {
         const int idx = e + i * kSeqEpi;
         if (idx >= E) break;
         const Owned o = owned(idx);
@@ -369,50 +378,86 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
             // gate g's sums of this group: hi products at tc0 + g 2 MT NS, lo products 8 columns on
             const uint32_t tc0 = trow + tGate + m * 2 * NS + 2 * nl0;
             float y[4][8];
-            {
-              float a0[16], a1[16];
-              tmem_ld16x2_sync(tc0, tc0 + 2 * MT * NS, a0, a1);
+            if constexpr (MT * NS >= 64) {  // one gate at a time: 16 registers in flight (the wide tiles need them)
 #pragma unroll
-              for (int k8 = 0; k8 < 8; ++k8) {
-                y[0][k8] = a0[k8] + a0[8 + k8];
-                y[1][k8] = a1[k8] + a1[8 + k8];
+              for (int g = 0; g < 4; ++g) {
+                float a0[16];
+                tmem_ld16_sync(tc0 + g * 2 * MT * NS, a0);
+#pragma unroll
+                for (int k8 = 0; k8 < 8; ++k8) y[g][k8] = a0[k8] + a0[8 + k8];
               }
-              tmem_ld16x2_sync(tc0 + 4 * MT * NS, tc0 + 6 * MT * NS, a0, a1);
+            } else {  // two gates per wait
 #pragma unroll
-              for (int k8 = 0; k8 < 8; ++k8) {
-                y[2][k8] = a0[k8] + a0[8 + k8];
-                y[3][k8] = a1[k8] + a1[8 + k8];
+              for (int g = 0; g < 4; g += 2) {
+                float a0[16], a1[16];
+                tmem_ld16x2_sync(tc0 + g * 2 * MT * NS, tc0 + (g + 1) * 2 * MT * NS, a0, a1);
+#pragma unroll
+                for (int k8 = 0; k8 < 8; ++k8) {
+                  y[g][k8] = a0[k8] + a0[8 + k8];
+                  y[g + 1][k8] = a1[k8] + a1[8 + k8];
+                }
               }
             }
             float hv[8], cv[8];
+            float* cs8 = cst + (m * SPW + 8 * i8) * kSeqEpi;
 #pragma unroll
             for (int k8 = 0; k8 < 8; ++k8)
               lstm_cell_s(y[0][k8] + bias[m][0], y[1][k8] + bias[m][1], y[2][k8] + bias[m][2],
-                          y[3][k8] + bias[m][3], c[m][8 * i8 + k8], hv[k8], cv[k8]);
+                          y[3][k8] + bias[m][3], cs8[k8 * kSeqEpi], hv[k8], cv[k8]);
+            // outputs of streams n0 + nl0 + k8 (k8 < nv) of unit j: element (t, n, j) at (t B + n) H + j
+            const int nv = min(8, B - (n0 + nl0));
+            const long long o0 = ((long long)t * B + n0 + nl0) * H + j;
+            if (!fin) {
+              if (a.ckpt_h) {
+                float* p = a.ckpt_h + (long long)cj * a.ck_stride + o0;
 #pragma unroll
-            for (int k8 = 0; k8 < 8; ++k8) {
-              const int nl = nl0 + k8, n = n0 + nl;
-              const long long o = ((long long)t * B + n) * H + j;
-              if (!fin) {
-                if (n < B) {
-                  if (a.ckpt_h) a.ckpt_h[(long long)cj * a.ck_stride + o] = hv[k8];
-                  if (a.ckpt_c) a.ckpt_c[(long long)cj * a.ck_stride + o] = cv[k8];
-                }
-                continue;
+                for (int k8 = 0; k8 < 8; ++k8)
+                  if (k8 < nv) p[(long long)k8 * H] = hv[k8];
               }
-              c[m][8 * i8 + k8] = cv[k8];
-              put_h(nl, jl, hv[k8]);
-              if (n < B) {
-                if (a.out_h) a.out_h[o] = hv[k8];
-                if (a.seq_bf16) {
+              if (a.ckpt_c) {
+                float* p = a.ckpt_c + (long long)cj * a.ck_stride + o0;
+#pragma unroll
+                for (int k8 = 0; k8 < 8; ++k8)
+                  if (k8 < nv) p[(long long)k8 * H] = cv[k8];
+              }
+              continue;
+            }
+            {  // h_t as the pair into the next step's operand (streams nl0 .. nl0 + 7 of unit jl)
+              const uint32_t hb = L.bh + (uint32_t)(jl >> 6) * (2u * NS * 128u) + (uint32_t)(nl0 >> 3) * 2048u +
+                                  (uint32_t)(jl & 7) * 2u;
+              const uint32_t cjl = (uint32_t)(jl & 63) >> 3;
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8) {
+                cs8[k8 * kSeqEpi] = cv[k8];
+                __nv_bfloat16 hi, lo;
+                seq_pair(hv[k8], hi, lo);
+                const uint32_t off = hb + k8 * 128u + ((cjl ^ (uint32_t)k8) << 4);
+                *reinterpret_cast<__nv_bfloat16*>(gb + off) = hi;
+                *reinterpret_cast<__nv_bfloat16*>(gb + off + 1024u) = lo;
+              }
+            }
+            if (a.out_h) {
+              float* p = a.out_h + o0;
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8)
+                if (k8 < nv) p[(long long)k8 * H] = hv[k8];
+            }
+            if (a.seq_bf16) {
+              __nv_bfloat16* p = a.seq_bf16 + ((long long)t * B + n0 + nl0) * a.ldh + j;
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8)
+                if (k8 < nv) {
                   __nv_bfloat16 hi, lo;
                   seq_pair(hv[k8], hi, lo);
-                  const long long so = ((long long)t * B + n) * a.ldh + j;
-                  a.seq_bf16[so] = hi;
-                  a.seq_bf16[a.seq_plane + so] = lo;
+                  p[(long long)k8 * a.ldh] = hi;
+                  p[a.seq_plane + (long long)k8 * a.ldh] = lo;
                 }
-                if (a.c_last && t == T - 1) a.c_last[(long long)n * H + j] = cv[k8];
-              }
+            }
+            if (a.c_last && t == T - 1) {
+              float* p = a.c_last + (long long)(n0 + nl0) * H + j;
+#pragma unroll
+              for (int k8 = 0; k8 < 8; ++k8)
+                if (k8 < nv) p[(long long)k8 * H] = cv[k8];
             }
           }
         }
