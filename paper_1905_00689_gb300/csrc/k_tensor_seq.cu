@@ -151,14 +151,14 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
   griddep_launch_dependents();
   if (threadIdx.x == 0) {
     mbar_init(fac_full, 1);
-    mbar_init(h_ready, kSeqEpi);
+    mbar_init(h_ready, kSeqEpi / 32);  // one arrival per epilogue warp
     mbar_init(tacc_full, 1);
     mbar_init(rs_full, 1);
     mbar_init(tau_full, 1);
     mbar_init(acc_full, 1);
     mbar_init(ckpt_bar, 1);
-    mbar_init(ckpt_done, kSeqEpi);
-    mbar_init(red_done, kSeqEpi);
+    mbar_init(ckpt_done, kSeqEpi / 32);
+    mbar_init(red_done, kSeqEpi / 32);
     mbar_init(drain_bar, 1);
     fence_mbarrier_init_cluster();
   }
@@ -255,14 +255,12 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
     struct Owned {
       int bt;   // byte offset in the tau' operand (hi plane)
       int pc;   // offset in P_t, or -1 (k >= K, or a stream past B)
-      int sc;   // column of sigma
     };
     auto owned = [&](int idx) {
       const int row = idx >> sp_sh, sp = idx & (SP - 1), g = row >> rpg_sh, k = row & (rpg - 1);
       const int nl = rank * SP + sp;
       Owned o;
       o.bt = (int)((nl >> 3) * 4096u + g * 512u + sw64_offset(nl, k));
-      o.sc = k < a.K ? g * a.Ks + k : -1;
       o.pc = (k < a.K && n0 + nl < B) ? (n0 + nl) * a.ldp + g * a.Ks + k : -1;
       return o;
     };
@@ -275,6 +273,23 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
       *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o) = hi;
       *reinterpret_cast<__nv_bfloat16*>(gb + L.bh + o + 1024u) = lo;
     };
+    // one arrival per warp on an mbarrier counting epilogue warps, once every
+    // lane of the warp has finished (its writes ordered by the warp barrier)
+    auto warp_arrive = [&](uint32_t mb) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(mb);
+    };
+    // sigma of this thread's owner elements (0 for k >= K)
+    float r_sig[kMaxRed];
+#pragma unroll
+    for (int i = 0; i < kMaxRed; ++i) {
+      const int idx = e + i * kSeqEpi;
+      r_sig[i] = 0.f;
+      if (idx < E) {
+        const int row = idx >> sp_sh, g = row >> rpg_sh, k = row & (rpg - 1);
+        if (k < a.K) r_sig[i] = a.sigma[g * a.Ks + k];
+      }
+    }
     griddep_wait();  // P, h0 and c0 may come from the kernels before this one
     // c_{t-1} of this thread's cell (m, stream s of its SPW): word (m SPW + s) kSeqEpi + e
     float* cst = reinterpret_cast<float*>(gb + L.cst) + e;
@@ -289,7 +304,7 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
       }
     fence_proxy_async_shared();
     tc_fence_before();
-    mbar_arrive(h_ready);
+    warp_arrive(h_ready);
     const float* rsb = reinterpret_cast<const float*>(gb + L.rs);
     const int srcs = R4 * SP;  // floats per source in the RS buffer
     bool ok = true;
@@ -335,13 +350,13 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
         float sum = 0.f;
         for (int src = 0; src < CS; ++src) sum += rsb[src * srcs + idx];
         __nv_bfloat16 hi, lo;
-        seq_pair(o.sc >= 0 ? __ldg(a.sigma + o.sc) * (sum + pv[i]) : 0.f, hi, lo);
+        seq_pair(r_sig[i] * (sum + pv[i]), hi, lo);
         *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + o.bt) = hi;
         *reinterpret_cast<__nv_bfloat16*>(gb + L.btau + o.bt + 2048) = lo;
       }
       fence_proxy_async_shared();
       tc_fence_before();  // this thread's tensor-memory reads are done before the gate MMAs overwrite them
-      mbar_arrive(red_done);
+      warp_arrive(red_done);
       // exchange 2: this CTA's block of tau' (its SP streams, all terms) -> every other CTA:
       // one copy per peer of SP / 8 whole stream groups, or (SP = 4, half a group) eight
       // 256-byte pieces per peer, one per (plane, gate)
@@ -463,13 +478,13 @@ __global__ void __launch_bounds__(seq_threads(NS), 1)
         }
         if (!fin) {
           tc_fence_before();
-          mbar_arrive(ckpt_done);
+          warp_arrive(ckpt_done);
         }
       }
       if (!ok) break;
       fence_proxy_async_shared();  // h_t in the operand, before the next step's MMAs read it
       tc_fence_before();
-      mbar_arrive(h_ready);
+      warp_arrive(h_ready);
     }
     if (!ok) atomicCAS(a.err, 0, kErrTcTimeout);
   }
