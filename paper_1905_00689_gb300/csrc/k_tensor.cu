@@ -64,6 +64,22 @@ constexpr int kTcThreads = 384;  // warps 0..3: TMA, MMA, TMEM, spare; warps 4..
 constexpr int kTileM = 128;
 constexpr int kTileK = 64;  // bf16 elements in one 128-byte swizzled row
 constexpr uint32_t kABytes = kTileM * kTileK * 2;
+constexpr int kConvGroups = 2;  // groups of epilogue warps converting alternate stages of fp32 activations
+
+// Named barrier `id` of `count` threads; returns whether any of them passed `pred`.
+__device__ __forceinline__ bool block_or(int id, int count, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+      "barrier.cta.red.or.pred q, %2, %3, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(pred ? 1u : 0u), "r"(id), "r"(count)
+      : "memory");
+  return r != 0u;
+}
+__device__ __forceinline__ void named_barrier(int id, int count) {
+  asm volatile("barrier.cta.sync.aligned %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
 
 __device__ __forceinline__ bool wait_cta(uint32_t mb, uint32_t parity, uint64_t limit, const volatile int* err) {
   return mbar_wait_bounded<false>(mb, parity, limit, err);
@@ -117,15 +133,17 @@ __device__ __forceinline__ float remainder_terms(const TcGatesArgs& a, int g, in
 // warps, idle until the accumulator is complete, convert each stage's tile
 // into its bf16 pair before the MMAs read it: x is read once from memory as
 // fp32 instead of being converted by a separate pass (which reads it and
-// writes its pair, the same bytes again).
+// writes its pair, the same bytes again).  The fp32 tile (BN rows x 64
+// columns) lands where the pair goes (both planes: the same bytes); the
+// converting threads read all of it into registers, meet at a named
+// barrier, and write the pair over it.
 template <int BN, int S, bool XF>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_rows_kernel(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, TcRowsArgs a) {
   extern __shared__ uint8_t smem_raw[];
   static_assert(BN <= 128, "the epilogue holds P_t of its columns in registers");
   constexpr uint32_t kBBytes = BN * kTileK * 2;        // one plane of the activation tile
-  constexpr uint32_t kRaw = XF ? BN * kTileK * 4 : 0;  // the fp32 activation tile: two boxes of 32 columns
-  constexpr uint32_t kStage = kABytes + 2 * kBBytes + kRaw;  // factor tile, hi plane, lo plane (fp32 tile)
+  constexpr uint32_t kStage = kABytes + 2 * kBBytes;   // factor tile, hi plane, lo plane (XF: first the fp32 tile)
   constexpr uint32_t kCols = BN < 32 ? 32 : BN;
   constexpr int kNb = XF ? 3 * S : 2 * S;  // full[S] | empty[S] (| converted[S])
   const uint32_t raw = smem_u32(smem_raw);
@@ -154,7 +172,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int i = 0; i < S; ++i) {
       mbar_init(bar0 + 8u * i, 1);
       mbar_init(bar0 + 8u * (S + i), 1);
-      if (XF) mbar_init(conv0 + 8u * i, 8 * 32);
+      if (XF) mbar_init(conv0 + 8u * i, 8 / kConvGroups);  // one arrival per warp of the stage's converting group
     }
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
@@ -194,7 +212,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // the factor tiles of the first S stages do not depend on the kernel
     // before this one: issue them before waiting for it
     const int npre = nkb < S ? nkb : S;
-    constexpr uint32_t b_bytes = XF ? kRaw : 2 * kBBytes;
+    constexpr uint32_t b_bytes = 2 * kBBytes;  // the pair, or (XF) the fp32 tile: the same bytes
     for (int kb = 0; kb < npre; ++kb) {
       mbar_arrive_expect_tx(bar0 + 8u * kb, a_bytes + b_bytes);
       load_a(base + kb * kStage, bar0 + 8u * kb, kb);
@@ -209,8 +227,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         load_a(st, bar0 + 8u * s, kb);
       }
       if constexpr (XF) {  // the fp32 tile, columns [64 kb, 64 kb + 32) and [64 kb + 32, 64 kb + 64)
-        tma_load_2d(st + kABytes + 2 * kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
-        tma_load_2d(st + kABytes + 2 * kBBytes + BN * 128u, &tmb, bar0 + 8u * s, kb * kTileK + 32, col0);
+        tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);
+        tma_load_2d(st + kABytes + BN * 128u, &tmb, bar0 + 8u * s, kb * kTileK + 32, col0);
       } else {
         tma_load_2d(st + kABytes, &tmb, bar0 + 8u * s, kb * kTileK, col0);                      // hi plane
         tma_load_2d(st + kABytes + kBBytes, &tmb, bar0 + 8u * s, kb * kTileK, a.b_plane + col0);  // lo plane
@@ -248,34 +266,52 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp >= 4) {  // ---- epilogue: warps 4..11, two per lane quarter ----
     const int ep = warp - 4, q = ep & 3;
     constexpr int kHalf = BN / 2;
-    if constexpr (XF) {  // each stage's fp32 activation tile -> its bf16 pair, in the stage's B planes
-      const int ce = threadIdx.x - 128;
+    if constexpr (XF) {  // each stage's fp32 activation tile -> its bf16 pair, in place
+      // kConvGroups groups of warps take the stages in turn (group g: stages kb = g mod kConvGroups),
+      // so that several stages are converted at once
+      constexpr int kGt = 256 / kConvGroups;  // threads per group
+      static_assert(BN * 16 % kGt == 0, "whole chunks per thread");
+      constexpr int kChunks = BN * 16 / kGt;  // 16-byte chunks of four columns per thread
+      const int grp = ep / (8 / kConvGroups), ce = (threadIdx.x - 128) % kGt;
       uint8_t* gbase = smem_raw + (base - raw);
       bool cok = true;
-      for (int kb = 0; kb < nkb && cok; ++kb) {
+      for (int kb = grp; kb < nkb; kb += kConvGroups) {
         const int s = kb % S;
-        if (!(cok = wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err))) break;
-        uint8_t* st = gbase + s * kStage;
-        // 16 chunks of four columns per row: chunk c = row n, columns [4 (c mod 16), +4)
-        for (int c = ce; c < BN * 16; c += 256) {
-          const int n = c >> 4, k4 = (c & 15) * 4;
-          const float4 v = *reinterpret_cast<const float4*>(st + kABytes + 2 * kBBytes + (k4 >> 5) * (BN * 128) +
-                                                             n * 128 + (k4 & 31) * 4);
+        // every thread of the group takes the same decision (reduction barrier), so that
+        // none of them waits at the group's second barrier for one that left
+        const bool failed = !wait_cta(bar0 + 8u * s, (kb / S) & 1, limit, err);
+        if (block_or(1 + 2 * grp, kGt, failed)) {
+          cok = false;
+          break;
+        }
+        uint8_t* st = gbase + s * kStage + kABytes;
+        // chunk c = row n, columns [4 (c mod 16), +4): box (k4 / 32) of the fp32 tile
+        float4 v[kChunks];
+#pragma unroll
+        for (int i = 0; i < kChunks; ++i) {
+          const int c = ce + kGt * i, n = c >> 4, k4 = (c & 15) * 4;
+          v[i] = *reinterpret_cast<const float4*>(st + (k4 >> 5) * (BN * 128) + n * 128 + (k4 & 31) * 4);
+        }
+        named_barrier(2 + 2 * grp, kGt);  // the whole fp32 tile is read before the pair overwrites it
+#pragma unroll
+        for (int i = 0; i < kChunks; ++i) {
+          const int c = ce + kGt * i, n = c >> 4, k4 = (c & 15) * 4;
           __nv_bfloat16 h[4], l[4];
-          bf16_pair(v.x, h[0], l[0]);
-          bf16_pair(v.y, h[1], l[1]);
-          bf16_pair(v.z, h[2], l[2]);
-          bf16_pair(v.w, h[3], l[3]);
+          bf16_pair(v[i].x, h[0], l[0]);
+          bf16_pair(v[i].y, h[1], l[1]);
+          bf16_pair(v[i].z, h[2], l[2]);
+          bf16_pair(v[i].w, h[3], l[3]);
           const uint32_t o = sw128_offset(n, k4) + (uint32_t)(n >> 3) * 1024u;
-          *reinterpret_cast<uint2*>(st + kABytes + o) =
+          *reinterpret_cast<uint2*>(st + o) =
               make_uint2((uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16),
                          (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16));
-          *reinterpret_cast<uint2*>(st + kABytes + kBBytes + o) =
+          *reinterpret_cast<uint2*>(st + kBBytes + o) =
               make_uint2((uint32_t)__bfloat16_as_ushort(l[0]) | ((uint32_t)__bfloat16_as_ushort(l[1]) << 16),
                          (uint32_t)__bfloat16_as_ushort(l[2]) | ((uint32_t)__bfloat16_as_ushort(l[3]) << 16));
         }
         fence_proxy_async_shared();
-        mbar_arrive(conv0 + 8u * s);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(conv0 + 8u * s);
       }
       if (!cok) atomicCAS(a.err, 0, kErrTcTimeout);
     }
@@ -757,7 +793,7 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args..
 
 template <int BN, int S, bool XF>
 size_t rows_smem() {
-  return 1024 + S * (kABytes + 2 * BN * kTileK * 2 + (XF ? BN * kTileK * 4 : 0)) + 8 * ((XF ? 3 : 2) * S + 2) + 16;
+  return 1024 + S * (kABytes + 2 * BN * kTileK * 2) + 8 * ((XF ? 3 : 2) * S + 2) + 16;
 }
 template <int NT, int S>
 size_t gates_smem() {
@@ -847,7 +883,7 @@ int tc_gates_tile_n(int H, int B) {
 }
 
 cudaError_t launch_tc_rows_xf32(const TcMap& A, const TcMap& Xf, const TcRowsArgs& a, int n_cols, cudaStream_t s) {
-  return launch_rows_t<64, 4, true>(A, Xf, a, n_cols, s);
+  return launch_rows_t<64, 6, true>(A, Xf, a, n_cols, s);
 }
 
 bool tc_make_map_f32(TcMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t pitch_bytes,
