@@ -128,7 +128,7 @@ __device__ __forceinline__ float remainder_terms(const TcGatesArgs& a, int g, in
 // ---------------------------------------------------------------------------
 // tile of tau' / P: rows of the packed factor matrix x columns (streams)
 // ---------------------------------------------------------------------------
-// XF (the projection, packed gates only): the activation comes as fp32
+// XF (the projection with packed gates): the activation comes as fp32
 // tiles (tmb is an fp32 map with boxes of 32 columns), and the epilogue
 // warps, idle until the accumulator is complete, convert each stage's tile
 // into its bf16 pair before the MMAs read it: x is read once from memory as

@@ -338,7 +338,9 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
   __nv_bfloat16* in_bf16 = nullptr;
   int ld_in = 0;
   // packed gates at layer 0: the projection reads x in fp32 and forms its
-  // bf16 pair itself (one tile of rows, so x is read once either way)
+  // bf16 pair itself (one tile of rows, so x is converted once either way;
+  // with several row tiles each would convert it again: at K = 512 the
+  // projection took twice as long), where TMA can map x
   const bool x_f32 = l == 0 && rpg > 0 && D % 4 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
   if (l == 0 && !x_f32) {  // operand conversion (outside the timed projection phase)
     LA_CUDA(h, launch_to_bf16(x, TB, D, static_cast<__nv_bfloat16*>(h->x_bf16), s.ldx, h->stream),

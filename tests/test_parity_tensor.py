@@ -244,16 +244,18 @@ def test_compressed_tau_layout_refused_where_it_does_not_apply(cuda_device):
     m.close()
 
 
+@pytest.mark.parametrize("K", [16, 200])
 @pytest.mark.parametrize("D,offset", [(64, 0), (42, 0), (64, 1)])
-def test_projection_input_forms(cuda_device, D, offset):
+def test_projection_input_forms(cuda_device, D, offset, K):
     """Up to K = 32 at layer 0 the projection reads x in fp32 and forms its
     bf16 pair itself when D is a multiple of 4 and x is 16-byte aligned;
-    otherwise x goes through the separate conversion pass.  Both agree with
-    the oracle (offset = 1: x starts one float into its buffer)."""
+    otherwise (and at K = 200, two 128-row tiles per gate) x goes through
+    the separate conversion pass.  All agree with the oracle (offset = 1: x
+    starts one float into its buffer)."""
     import torch
     from paper_1905_00689_gb300 import LSTMApprox
-    H, T, B, K = 256, 3, 20, 16
-    gates = [draw_factor_set(H, D + H, K, 70, 6600 + D + g) for g in range(4)]
+    H, T, B = 256, 3, 20
+    gates = [draw_factor_set(H, D + H, K, 70, 6600 + D + K + g) for g in range(4)]
     x = draw_inputs(T, B, D, "uniform", 9)
     m = LSTMApprox(1, [D], H, K, B, "bf16")
     m.set_layer(0, gates)
