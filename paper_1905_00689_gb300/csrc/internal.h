@@ -91,6 +91,8 @@ struct lstm_approx {
   void* h_bf16 = nullptr;     // [2][B][ldh] bf16 pair of the h operand (tensor path)
   int* err = nullptr;         // device status word (0 = ok)
   int* err_host = nullptr;    // pinned host copy of it, read after the stream synchronises
+  unsigned* proj_flags = nullptr;  // [kProjFlags] completion flags of a projection launched after the recurrence
+  unsigned proj_epoch = 0;         // the value the last such launch wrote
 
   // staging for lstm_approx_run_host
   size_t stage_bytes = 0;
@@ -142,9 +144,26 @@ struct SparseXRows {
 // The same product from the compressed rows, for T*B <= 32 columns.
 cudaError_t launch_xproj_sparse(const SparseXRows& sr, int K, int Ks, const float* X, int ldxin, int N, float* out,
                                 int ldo, cudaStream_t s);
+// Launched after the recurrence kernel that reads its output (see
+// run_device): the projection then starts as a programmatic dependent of
+// that kernel, may take every SM the recurrence leaves free, and each of its
+// CTAs writes `epoch` to flags[its linear index] (release, GPU scope) once
+// its outputs are stored; the recurrence waits for all of them before its
+// first read of P.
+struct XprojSignal {
+  unsigned* flags = nullptr;
+  unsigned epoch = 0;
+};
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
                                  int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s,
-                                 int max_split);
+                                 int max_split, const XprojSignal* sig = nullptr);
+// CTAs of that launch (one flag each when it signals).
+int xproj_cluster_ctas(int K, int N, int D, int max_split);
+// Loads the kernel that launch_xproj_cluster would launch for N columns
+// (lazy module loading would otherwise delay a launch made while the
+// recurrence runs until that recurrence has finished).
+cudaError_t xproj_cluster_prepare(bool a_bf16, int N);
+constexpr int kProjFlags = 2048;  // flags of one signalling projection launch
 
 // One timestep of the refinement sums over u (a3), the intermediate outputs
 // (a6) and the cell update (a4) for B streams.
@@ -200,6 +219,12 @@ struct PersistentArgs {
   Checkpoints ck;
   long long wait_limit_ns;
   int test_stall;
+  // Non-null when the projection that writes P is launched after this kernel
+  // (XprojSignal): the kernel then waits until proj_flags[0, proj_nflags)
+  // all hold proj_epoch instead of waiting for the grid before it.
+  const unsigned* proj_flags;
+  int proj_nflags;
+  unsigned proj_epoch;
 };
 cudaError_t launch_persistent(const PersistentPlan& plan, const PersistentArgs& a, cudaStream_t s);
 

@@ -235,7 +235,6 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(DenseArgs a) {
         lstm_cell_f(ys[lane], ys[UB + lane], ys[2 * UB + lane], ys[3 * UB + lane], c_reg, hh, cc);
         c_reg = cc;
         h_new = hh;
-        a.out_h[((long long)t * a.B + b) * H + cj] = hh;
       }
       if (t + 1 < a.T) {
         // message m = (piece m / CS, CTA m % CS): the 4 units of the piece
@@ -254,6 +253,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(DenseArgs a) {
           }
         }
       }
+      // the output store after the sends: it is not on the path to the next timestep
+      if (cell_lane) a.out_h[((long long)t * a.B + b) * H + cj] = h_new;
     }
     p_cur = p_next;
   }

@@ -320,6 +320,8 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
   const int b = blockIdx.x / p.CS;  // one cluster per stream
+  // a projection launched after this kernel may start now (it waits for nothing)
+  if (a.proj_flags != nullptr) griddep_launch_dependents();
   const int H = a.H, K = a.K, J = a.ck.n;
   const int tau_len = 4 * tau_gate_len(p.Kp) + kTauSlack;
   const int h_len = h_buffer_len(p, HC);
@@ -543,10 +545,12 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     }
     if (!placed) masked |= 1u << n;
   }
-  // everything above only read the factors; P is written by the projection
-  // launched just before this kernel, which may still be running
-  griddep_wait();
-  float p_cur = p_off >= 0 ? __ldg(a.P + (long long)b * p_stride + p_off) : 0.f;
+  // everything above only read the factors; P is written by the projection,
+  // launched either just before this kernel (which may still be running) or
+  // just after it (whose CTAs each raise a flag once their part is stored)
+  bool setup_ok = true;
+  if (a.proj_flags == nullptr) griddep_wait();
+  else if (warp == 0) setup_ok = wait_flags_epoch(a.proj_flags, a.proj_nflags, a.proj_epoch, limit_ns, err);
 
   // remote addresses of the exchange buffers in CTA (lane mod CS)
   const uint32_t peer = static_cast<uint32_t>(lane) & static_cast<uint32_t>(p.CS - 1);
@@ -558,9 +562,10 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
   const uint32_t r_bar_h = mapa_shared(bar_h0, peer);
   const int lcs = ilog2(p.CS);
 
-  bool setup_ok = true;
-  if constexpr (!kTmem) setup_ok = mbar_wait_bounded<false>(bar_setup, 0, limit_ns, err);
+  if constexpr (!kTmem) setup_ok = mbar_wait_bounded<false>(bar_setup, 0, limit_ns, err) && setup_ok;
   if (!__syncthreads_and(setup_ok) && tid == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
+  // P through L2 (it may have been written while this kernel ran)
+  float p_cur = p_off >= 0 ? __ldcg(a.P + (long long)b * p_stride + p_off) : 0.f;
   cluster_sync_all();  // every CTA's barriers are armed before any st.async
 
   const int t_end = *err == 0 ? a.T : 0;  // nothing to do after a failed set-up
@@ -570,7 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
     int fail = 0;  // error code of a wait of this warp that ran out
     // prefetch the next step's projection for this lane's row
     const float p_next = (p_off >= 0 && t + 1 < a.T)
-                             ? __ldg(a.P + ((long long)(t + 1) * a.B + b) * p_stride + p_off)
+                             ? __ldcg(a.P + ((long long)(t + 1) * a.B + b) * p_stride + p_off)
                              : 0.f;
     // ---- wait for h_{t-1} (t = 0 uses h0, loaded locally) ----------------
     if (t > 0) {
@@ -727,22 +732,18 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
       const long long tbo = ((long long)t * a.B + b) * H;
       const float cp = __shfl_sync(0xffffffffu, c_reg, ci);  // c_{t-1} of unit ci
       float h_new = 0.f;
-      for (int n0 = 0; n0 < p.nset; n0 += 32 / UW) {
-        const int n = n0 + lane / UW;
-        if (n < p.nset && unit_ok) {
-          const float* src = pb + n * 4 * S4 + c_slot;
-          float hh, cc;
-          lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3], cp,
-                      hh, cc);
-          if (n == 0) {
-            c_reg = cc;
-            h_new = hh;
-            a.out_h[tbo + cj] = hh;
-          } else {
-            const long long o = (long long)(n - 1) * a.T * a.B * H + tbo + cj;
-            if (a.ckpt_h) a.ckpt_h[o] = hh;
-            if (a.ckpt_c) a.ckpt_c[o] = cc;
-          }
+      // the cells of the first round (the full depth and the first depth
+      // sets) are computed before h_t is sent and stored after it, so that
+      // the output stores are not on the path to the next timestep
+      const int n_first = lane / UW;
+      float hh0 = 0.f, cc0 = 0.f;
+      if (n_first < p.nset && unit_ok) {
+        const float* src = pb + n_first * 4 * S4 + c_slot;
+        lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3], cp,
+                    hh0, cc0);
+        if (n_first == 0) {
+          c_reg = cc0;
+          h_new = hh0;
         }
       }
       if (t + 1 < a.T) {
@@ -761,6 +762,27 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_kernel(PersistentArgs 
             const uint32_t off = 4u * (nb * h_len + rank * p.UBv + slot);
             st_async_piece(r_h + off, hv, PIECE, r_bar_h + 8u * nb);
           }
+        }
+      }
+      if (n_first < p.nset && unit_ok) {
+        if (n_first == 0) {
+          a.out_h[tbo + cj] = hh0;
+        } else {
+          const long long o = (long long)(n_first - 1) * a.T * a.B * H + tbo + cj;
+          if (a.ckpt_h) a.ckpt_h[o] = hh0;
+          if (a.ckpt_c) a.ckpt_c[o] = cc0;
+        }
+      }
+      for (int n0 = 32 / UW; n0 < p.nset; n0 += 32 / UW) {
+        const int n = n0 + lane / UW;
+        if (n < p.nset && unit_ok) {
+          const float* src = pb + n * 4 * S4 + c_slot;
+          float hh, cc;
+          lstm_cell_f(src[0] + bias_r[0], src[S4] + bias_r[1], src[2 * S4] + bias_r[2], src[3 * S4] + bias_r[3], cp,
+                      hh, cc);
+          const long long o = (long long)(n - 1) * a.T * a.B * H + tbo + cj;
+          if (a.ckpt_h) a.ckpt_h[o] = hh;
+          if (a.ckpt_c) a.ckpt_c[o] = cc;
         }
       }
     }
@@ -796,9 +818,10 @@ cudaError_t launch_t(const DevPlan& dp, size_t smem, const PersistentArgs& a, cu
   attr[0].val.clusterDim.x = dp.CS;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  // may start while the projection before it finishes (set-up overlaps it)
+  // may start while the projection before it finishes (set-up overlaps it);
+  // with the projection launched after it, an ordinary launch
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].val.programmaticStreamSerializationAllowed = a.proj_flags == nullptr ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   // function attributes once per instantiation (the largest shared memory any

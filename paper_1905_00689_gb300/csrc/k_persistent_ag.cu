@@ -119,6 +119,8 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_ag_kernel(PersistentAr
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
   const int b = blockIdx.x / p.CS;  // one cluster per stream
+  // a projection launched after this kernel may start now (it waits for nothing)
+  if (a.proj_flags != nullptr) griddep_launch_dependents();
   const int per_gate = p.CS / 4;    // CTAs sharing one gate's terms
   const int gate = (int)rank / per_gate, part = (int)rank % per_gate;
   const int k0 = part * p.RA;       // first own term
@@ -253,8 +255,14 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_ag_kernel(PersistentAr
     for (int g = 0; g < 4; ++g) bias_r[g] = a.bias[g * H + tid];
     if (a.c0 != nullptr) c_reg = a.c0[(long long)b * H + tid];
   }
-  griddep_wait();  // P is written by the projection launched just before
-  float p_cur = p_off >= 0 ? __ldg(a.P + (long long)b * p_stride + p_off) : 0.f;
+  // P is written by the projection launched just before this kernel, or just
+  // after it (its CTAs then each raise a flag once their part is stored)
+  bool setup_ok = true;
+  if (a.proj_flags == nullptr) griddep_wait();
+  else if (warp == 0) setup_ok = wait_flags_epoch(a.proj_flags, a.proj_nflags, a.proj_epoch, limit_ns, err);
+  if (!__syncthreads_and(setup_ok) && tid == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
+  // P through L2 (it may have been written while this kernel ran)
+  float p_cur = p_off >= 0 ? __ldcg(a.P + (long long)b * p_stride + p_off) : 0.f;
   const uint32_t bar0 = smem_u32(&bars[0]);
   const bool writer = tid >= ub0 && tid < ub0 + my_ub;
   const bool warp_units = warp * 32 < H;  // tensor-memory loads are warp-wide
@@ -262,12 +270,13 @@ __global__ void __launch_bounds__(kThreads, 1) persistent_ag_kernel(PersistentAr
   __syncthreads();
   cluster_sync_all();  // every CTA's barriers are armed before any copy reaches them
 
+  const int t_end = *err == 0 ? a.T : 0;  // nothing to do after a failed set-up
   bool failed = false;
-  for (int t = 0; t < a.T; ++t) {
+  for (int t = 0; t < t_end; ++t) {
     const int hb = t & 1;
     int fail = 0;
     const float p_next = (p_off >= 0 && t + 1 < a.T)
-                             ? __ldg(a.P + ((long long)(t + 1) * a.B + b) * p_stride + p_off)
+                             ? __ldcg(a.P + ((long long)(t + 1) * a.B + b) * p_stride + p_off)
                              : 0.f;
     // ---- phase A: tau' = sigma (V_h h_{t-1} + P_t), own rows, kept locally --
     if (warp < ngroups) {
@@ -507,9 +516,10 @@ cudaError_t launch_ag_t(const AgPlan& p, size_t smem, const PersistentArgs& a, c
   attr[0].val.clusterDim.x = p.CS;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  // may start while the projection before it finishes (set-up overlaps it)
+  // may start while the projection before it finishes (set-up overlaps it);
+  // with the projection launched after it, an ordinary launch
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].val.programmaticStreamSerializationAllowed = a.proj_flags == nullptr ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   static thread_local bool attrs_set = false;

@@ -148,7 +148,8 @@ template <typename TF, int NC>
 __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ A, int lda, int K, int Ks,
                                                          const float* __restrict__ X, int ldxin, int N, int D,
                                                          int dchunk, float* __restrict__ out, int ldo, int S,
-                                                         int* err, long long limit_ns) {
+                                                         int* err, long long limit_ns, unsigned* done_flags,
+                                                         unsigned epoch) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw);  // [0]: incoming chunk sums
   // ring slot s: V_x rows [32][v_stride] then x columns [4 NC][kXStride]
@@ -300,6 +301,16 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
       if (n < N && r < nrows) out[(long long)n * ldo + (long long)(r / K) * Ks + r % K] = red[o];
     }
   }
+  if (done_flags != nullptr) {
+    // the recurrence kernel launched before this one waits for every CTA's flag
+    __syncthreads();  // this CTA's outputs are stored
+    if (tid == 0 && ok)
+      flag_release(done_flags + ((long long)blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x, epoch);
+    // CTA 0 then stays until that recurrence has finished, so that this grid
+    // completes after it: work later in the stream that starts as this grid's
+    // programmatic dependent and waits for it sees the recurrence's outputs
+    if (blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0) griddep_wait();
+  }
   if (!ok) {
     // a wait ran out: copies or pushes issued before it may still be in
     // flight towards this CTA; let them land before it exits
@@ -308,51 +319,91 @@ __global__ void __launch_bounds__(kThreads) xproj_kernel(const TF* __restrict__ 
   }
 }
 
+// Chunks of D per cluster: about half a CTA per SM in total, at least 128
+// values of D each, and at most max_split.  (Beside a resident recurrence,
+// twice as many CTAs made the whole call slower: D = 1024, 4K = 1024,
+// T*B = 20: 68.7 against 60.0 us.)
+int xproj_split(int row_tiles, int col_chunks, int D, int max_split) {
+  int S = 1;
+  while (S < kMaxSplit && S < max_split && row_tiles * col_chunks * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
+  return S;
+}
+
+// Sets the kernel's shared-memory limit once per thread; this also loads the
+// kernel's code if the module is loaded lazily, which a launch that must
+// start while another kernel runs (XprojSignal) cannot wait for.
 template <typename TF, int NC>
-cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
-                      int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split) {
-  auto kern = xproj_kernel<TF, NC>;
-  constexpr size_t smem = smem_bytes<TF, NC>();
+cudaError_t prepare_nc() {
   static thread_local bool attr_set = false;
   if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = cudaFuncSetAttribute(xproj_kernel<TF, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem_bytes<TF, NC>());
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  return cudaSuccess;
+}
+
+template <typename TF>
+cudaError_t prepare_typed(int N) {
+  switch ((min(N, kCols) + 3) / 4) {
+    case 1: return prepare_nc<TF, 1>();
+    case 2: return prepare_nc<TF, 2>();
+    case 3: return prepare_nc<TF, 3>();
+    case 4: return prepare_nc<TF, 4>();
+    case 5: return prepare_nc<TF, 5>();
+    case 6: return prepare_nc<TF, 6>();
+    case 7: return prepare_nc<TF, 7>();
+    case 8: return prepare_nc<TF, 8>();
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <typename TF, int NC>
+cudaError_t launch_nc(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
+                      int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split, const XprojSignal* sig) {
+  auto kern = xproj_kernel<TF, NC>;
+  constexpr size_t smem = smem_bytes<TF, NC>();
+  const cudaError_t pe = prepare_nc<TF, NC>();
+  if (pe != cudaSuccess) return pe;
   const int row_tiles = (4 * K + kRows - 1) / kRows;
   const int col_chunks = (N + kCols - 1) / kCols;
-  // chunks of D: about one CTA per SM in total, at least 128 values of D
-  // each, and at most max_split (the caller's choice: see run_device)
-  int S = 1;
-  while (S < kMaxSplit && S < max_split && row_tiles * col_chunks * S * 2 <= 148 && D >= 2 * S * 128) S *= 2;
+  const bool signals = sig != nullptr && sig->flags != nullptr;
+  const int S = xproj_split(row_tiles, col_chunks, D, max_split);
   const int dchunk = (((D + S - 1) / S) + 7) & ~7;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(row_tiles, S, col_chunks);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = S;
   attr[0].val.clusterDim.z = 1;
+  // after a recurrence kernel that waits for this one's flags: start as its
+  // programmatic dependent (it signals at its start), never wait for it
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, A, lda, K, Ks, X, ldxin, N, D, dchunk, out, ldo, S, err, limit_ns);
+  cfg.numAttrs = signals ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kern, A, lda, K, Ks, X, ldxin, N, D, dchunk, out, ldo, S, err, limit_ns,
+                            signals ? sig->flags : nullptr, signals ? sig->epoch : 0u);
 }
 
 template <typename TF>
 cudaError_t launch_typed(const TF* A, int lda, int K, int Ks, const float* X, int ldxin, int N, int D, float* out,
-                         int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split) {
+                         int ldo, int* err, long long limit_ns, cudaStream_t s, int max_split,
+                         const XprojSignal* sig) {
   switch ((min(N, kCols) + 3) / 4) {  // columns per lane (more than 32: chunks of 32)
-    case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 4: return launch_nc<TF, 4>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 5: return launch_nc<TF, 5>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 6: return launch_nc<TF, 6>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 7: return launch_nc<TF, 7>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
-    case 8: return launch_nc<TF, 8>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+    case 1: return launch_nc<TF, 1>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 2: return launch_nc<TF, 2>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 3: return launch_nc<TF, 3>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 4: return launch_nc<TF, 4>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 5: return launch_nc<TF, 5>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 6: return launch_nc<TF, 6>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 7: return launch_nc<TF, 7>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
+    case 8: return launch_nc<TF, 8>(A, lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split, sig);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -438,11 +489,22 @@ bool xproj_cluster_fits(int N, int D, const void* A, int lda, const float* X, in
 
 cudaError_t launch_xproj_cluster(const void* A, bool a_bf16, int lda, int K, int Ks, const float* X, int ldxin,
                                  int N, int D, float* out, int ldo, int* err, long long limit_ns, cudaStream_t s,
-                                 int max_split) {
+                                 int max_split, const XprojSignal* sig) {
   if (a_bf16)
     return launch_typed(static_cast<const __nv_bfloat16*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns,
-                        s, max_split);
-  return launch_typed(static_cast<const float*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split);
+                        s, max_split, sig);
+  return launch_typed(static_cast<const float*>(A), lda, K, Ks, X, ldxin, N, D, out, ldo, err, limit_ns, s, max_split,
+                      sig);
+}
+
+cudaError_t xproj_cluster_prepare(bool a_bf16, int N) {
+  return a_bf16 ? prepare_typed<__nv_bfloat16>(N) : prepare_typed<float>(N);
+}
+
+int xproj_cluster_ctas(int K, int N, int D, int max_split) {
+  const int row_tiles = (4 * K + kRows - 1) / kRows;
+  const int col_chunks = (N + kCols - 1) / kCols;
+  return row_tiles * col_chunks * xproj_split(row_tiles, col_chunks, D, max_split);
 }
 
 }  // namespace lstm_approx_impl

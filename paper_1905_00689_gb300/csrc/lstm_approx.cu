@@ -575,18 +575,44 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
       continue;
     }
     // (a1) hoisted input projection P[t][b][(g,k)] = prune(v_{g,k})[0:D]^T x_t,b
-    // Before the per-unit-block kernel at K > 128 (a cluster of 16 CTAs
-    // whose set-up fills about 256 KB of tensor memory each), the projection
-    // runs unsplit along D: its smaller grid leaves a GPC free, so that the
-    // recurrence's set-up overlaps it (D = 1024, H = 512, T = 20: the run
-    // 2% faster although the projection takes 15.8 instead of 10.5 us).
-    // Shorter set-ups gain less than the slower projection costs (K = 64:
-    // 4% slower, the one-exchange kernel at K = 16: 11%).
+    //
+    // Order of the two launches.  Ahead of the per-unit-block persistent
+    // kernel for one stream, when the few-column projection kernel serves and
+    // no phase is being timed, the recurrence is launched first: its cluster
+    // takes its SMs at once, the projection follows as its programmatic
+    // dependent on the SMs left free and raises one flag per CTA, and the
+    // recurrence loads its factors meanwhile and waits for the flags before
+    // its first read of P (D = 1024, H = 512, T = 20, whole call: K = 256
+    // with two intermediate depths 64.1 -> 60.0 us, K = 64 46.8 -> 45.0 us;
+    // with the projection split four ways along D, 128 CTAs, 68.7 us).  The
+    // one-exchange kernel's short set-up gains nothing from it (K = 16:
+    // 41.4 -> 43.0 us), and several streams' clusters need not all be
+    // resident at once, which the flags would require.  Otherwise the
+    // projection comes first and the recurrence starts as its programmatic
+    // dependent; there, before the per-unit-block kernel at K > 128 (a
+    // cluster of 16 CTAs whose set-up fills about 256 KB of tensor memory
+    // each), the projection runs unsplit along D: its smaller grid leaves a
+    // GPC free, so that the recurrence's set-up overlaps it (the run 2%
+    // faster although the projection takes 15.8 instead of 10.5 us).
+    // Shorter set-ups gain less than the slower projection costs (K = 64: 4%
+    // slower, the one-exchange kernel at K = 16: 11%).
+    const bool sparse_x = sparse_x_projection(h, s, K, T * B);
+    const bool cluster_x = !sparse_x && xproj_cluster_fits(T * B, s.D, s.Vx, s.ldx, in, s.D, bf16);
+    bool rec_first = path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && B == 1 && cluster_x &&
+                     !h->timing.on && h->proj_flags != nullptr;
+    const int proj_ctas = rec_first ? xproj_cluster_ctas(K, T * B, s.D, 8) : 0;
+    rec_first = rec_first && proj_ctas <= kProjFlags && xproj_cluster_prepare(bf16, T * B) == cudaSuccess;
     const int xproj_max_split =
-        (path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && K > 128) ? 1 : 8;
-    {
+        rec_first ? 8 : (path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && K > 128) ? 1 : 8;
+    XprojSignal sig;
+    if (rec_first) {
+      if (++h->proj_epoch == 0) ++h->proj_epoch;  // the flags start at zero
+      sig.flags = h->proj_flags;
+      sig.epoch = h->proj_epoch;
+    }
+    auto launch_projection = [&]() -> int {
       PhaseTimer pt(h, 0);
-      if (sparse_x_projection(h, s, K, T * B)) {
+      if (sparse_x) {
         SparseXRows sr;
         for (int g = 0; g < 4; ++g) {
           sr.off[g] = s.xoff[g];
@@ -595,10 +621,11 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
         }
         LA_CUDA(h, launch_xproj_sparse(sr, K, h->Ks, in, s.D, T * B, h->Px, (int)ldp, h->stream),
                 "input projection launch");
-      } else if (xproj_cluster_fits(T * B, s.D, s.Vx, s.ldx, in, s.D, bf16))
+      } else if (cluster_x)
         LA_CUDA(h,
                 launch_xproj_cluster(s.Vx, bf16, s.ldx, K, h->Ks, in, s.D, T * B, s.D, h->Px, (int)ldp, h->err,
-                                     h->opt_wait_limit_us * 1000LL, h->stream, xproj_max_split),
+                                     h->opt_wait_limit_us * 1000LL, h->stream, xproj_max_split,
+                                     rec_first ? &sig : nullptr),
                 "input projection launch");
       else
         LA_CUDA(h,
@@ -606,9 +633,14 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
                                  nullptr, 0, h->stream),
                 "input projection launch");
       h->launches += 1;
+      return LSTM_APPROX_OK;
+    };
+    if (!rec_first) {
+      rc = launch_projection();
+      if (rc) return rc;
     }
-    PhaseTimer pt(h, 1);
     if (path == LSTM_APPROX_PATH_PERSISTENT) {
+      PhaseTimer pt(h, 1);
       PersistentArgs a{};
       a.Vh = static_cast<const float*>(s.Vh);
       a.U = static_cast<const float*>(s.U);
@@ -631,12 +663,22 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
       a.ck = lck;
       a.wait_limit_ns = h->opt_wait_limit_us * 1000LL;
       a.test_stall = h->opt_test_stall;
+      if (rec_first) {
+        a.proj_flags = h->proj_flags;
+        a.proj_nflags = proj_ctas;
+        a.proj_epoch = sig.epoch;
+      }
       h->opt_test_stall = 0;
       LA_CUDA(h, launch_persistent_choice(plan, a, h->stream), "persistent kernel launch");
       h->launches += 1;
       h->last_cluster = plan.CS;
       h->last_variant = plan.variant;
+      if (rec_first) {
+        rc = launch_projection();
+        if (rc) return rc;
+      }
     } else {
+      PhaseTimer pt(h, 1);
       float* hs = h->h_state + (size_t)l * h->max_batch * H;
       float* cs = h->c_state + (size_t)l * h->max_batch * H;
       const size_t sb = (size_t)B * H * sizeof(float);
@@ -750,6 +792,8 @@ int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dim
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->c_state), state, "state");
   if (!rc) rc = dmalloc(h, &h->tau, (size_t)max_batch * 4 * h->Ks * sizeof(float), "scratch tau");
   if (!rc) rc = dmalloc(h, reinterpret_cast<void**>(&h->err), sizeof(int), "status word");
+  if (!rc)
+    rc = dmalloc(h, reinterpret_cast<void**>(&h->proj_flags), kProjFlags * sizeof(unsigned), "projection flags");
   if (!rc && cudaHostAlloc(reinterpret_cast<void**>(&h->err_host), sizeof(int), cudaHostAllocDefault) != cudaSuccess)
     rc = fail(h, LSTM_APPROX_ENOMEM, "pinned status word");
   if (!rc && dtype == LSTM_APPROX_BF16)
@@ -1077,6 +1121,7 @@ void lstm_approx_destroy(lstm_approx_t* h) {
   cudaFree(h->seq);
   cudaFree(h->tau);
   cudaFree(h->err);
+  cudaFree(h->proj_flags);
   if (h->err_host) cudaFreeHost(h->err_host);
   cudaFree(h->stage);
   cudaFree(h->gpart);

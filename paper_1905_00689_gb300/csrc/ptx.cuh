@@ -143,6 +143,43 @@ __device__ __forceinline__ void griddep_launch_dependents() {
 }
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// Completion flag of a CTA of another grid: its stores before the call are
+// visible to a thread that reads `epoch` from the flag with acquire
+// semantics.  The caller orders the CTA's stores before it (a CTA barrier).
+__device__ __forceinline__ void flag_release(unsigned* flag, unsigned epoch) {
+  __threadfence();
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(flag), "r"(epoch) : "memory");
+}
+
+// Bounded wait of the calling warp until flags[0, n) all hold `epoch`;
+// gives up after limit_ns of wall time or once *err is set.  Each pass
+// reads every flag with relaxed loads (they overlap, where acquire loads
+// would each wait for the one before), and one acquire fence after the
+// pass that saw them all orders the caller's later reads after the writes
+// the flags release.  Warp-uniform result.
+__device__ __forceinline__ bool wait_flags_epoch(const unsigned* flags, int n, unsigned epoch, uint64_t limit_ns,
+                                                 const volatile int* err) {
+  const int lane = threadIdx.x & 31;
+  uint64_t t0 = 0;
+  for (;;) {
+    bool mine = true;
+    for (int i = lane; i < n; i += 32) {
+      unsigned v;
+      asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(flags + i) : "memory");
+      mine = mine && v == epoch;
+    }
+    if (__all_sync(0xffffffffu, mine)) {
+      asm volatile("fence.acq_rel.gpu;" ::: "memory");
+      return true;
+    }
+    if (__any_sync(0xffffffffu, *err != 0)) return false;
+    const uint64_t now = global_timer_ns();
+    if (t0 == 0) t0 = now;
+    else if (now - t0 > limit_ns) return false;
+    __nanosleep(32);
+  }
+}
+
 // Makes a value opaque to the compiler, so that it stays in its register for
 // the rest of a persistent kernel instead of being loaded again from memory
 // where it is used.

@@ -13,7 +13,8 @@ import pytest
 
 from parity_util import (FP32_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run,
                          persistent_layout_cases, run_gpu, synthetic_layer, workload_inputs)
-from paper_1905_00689_gb300 import FP32, PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_PERSISTENT_VARIANT, plan
+from paper_1905_00689_gb300 import (FP32, OPT_TIMING, PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_LAUNCHES,
+                                    Q_PERSISTENT_VARIANT, plan)
 from workloads import draw_factor_set, draw_inputs
 
 pytestmark = pytest.mark.gpu
@@ -156,3 +157,51 @@ def test_one_exchange_kernel_every_layout(cuda_device, H, cs, K):
     layers = [[draw_factor_set(H, D + H, K, 30, 5300 + H + K + g) for g in range(4)]]
     x = draw_inputs(T, 1, D, "relu", H + K)
     _check(layers, x, K, 2, cluster=cs, checkpoints=[K // 3, K - 7])
+
+
+def _run_again(m, x, K, H, checkpoints):
+    import torch
+    T, B, _ = x.shape
+    xt = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).cuda()
+    out = torch.full((T, B, H), float("nan"), device="cuda")
+    ck = torch.full((len(checkpoints), T, B, H), float("nan"), device="cuda")
+    m.run(xt, K, out, checkpoints=list(checkpoints), ckpt_h=ck)
+    m.sync()
+    return {"h": out.double().cpu().numpy(), "ckpt_h": ck.double().cpu().numpy()}
+
+
+def test_launch_orders_agree(cuda_device):
+    """Batch 1, per-unit-block kernel: by default the recurrence is launched
+    before its input projection and waits for the projection's per-CTA flags;
+    with phase timing on, the projection comes first.  Both orders, several
+    calls in a row (each call raises its flags with a new value), on the
+    benchmark workload, against the oracle."""
+    K, cps = 256, [16, 64]
+    layers = [list(synthetic_layer("c2", 0, 256, 0.25))]
+    x = workload_inputs(WORKLOADS["c2"])
+    ref = oracle_run(layers, x, K, checkpoints=cps)
+    got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=1, checkpoints=cps, max_rank=256)
+    assert_parity(got, ref, FP32_TOL)
+    n0 = m.query(Q_LAUNCHES)
+    for timing in (0, 1, 0, 1, 0):
+        m.set_option(OPT_TIMING, timing)
+        again = _run_again(m, x, K, 512, cps)
+        assert_parity(again, ref, FP32_TOL, keys=("h", "ckpt_h"))
+    assert m.query(Q_LAUNCHES) - n0 == 5 * 2  # projection and recurrence in either order
+
+
+def test_launch_orders_two_layer_stack(cuda_device):
+    """Two fp32 layers of one stream: the second layer's recurrence (launched
+    first) and projection read the first layer's outputs."""
+    D, H, T, K = 64, 128, 6, 32
+    layers = [[draw_factor_set(H, (D if l == 0 else H) + H, K, 60, 1700 + 10 * l + g) for g in range(4)]
+              for l in range(2)]
+    x = draw_inputs(T, 1, D, "uniform", 17)
+    ref = oracle_run(layers, x, K, checkpoints=[8, 32])
+    for timing in (0, 1):
+        got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=1, checkpoints=[8, 32])
+        if timing:
+            m.set_option(OPT_TIMING, 1)
+            got = _run_again(m, x, K, H, [8, 32])
+        assert m.query(Q_PERSISTENT_VARIANT) == 1
+        assert_parity(got, ref, FP32_TOL, keys=("h", "ckpt_h"))
