@@ -269,7 +269,8 @@ enum lstm_approx_option_key {
   LSTM_APPROX_OPT_FORCE_PATH = 0,   /* 0 = automatic, else an lstm_approx_path */
   LSTM_APPROX_OPT_CLUSTER = 1,      /* 0 = automatic, else 1, 2, 4, 8 or 16 */
   LSTM_APPROX_OPT_TIMING = 2,       /* 1 = record CUDA events around each phase */
-  LSTM_APPROX_OPT_WAIT_LIMIT = 3,   /* bounded-wait limit in polls (default 2^26) */
+  LSTM_APPROX_OPT_WAIT_LIMIT = 3,   /* wall-time limit of every bounded in-kernel
+                                       wait, in microseconds (default 2000000) */
   LSTM_APPROX_OPT_TEST_STALL = 4,   /* 1 = next persistent run waits on a signal
                                        nobody sends (exercises ETIMEOUT) */
   LSTM_APPROX_OPT_PERSISTENT_VARIANT = 5, /* persistent kernel: 0 = automatic (the
@@ -289,12 +290,24 @@ enum lstm_approx_option_key {
                                tensor cores (default: faster at every shape
                                measured), 1 = v's kept h entries (compressed
                                rows) on the CUDA cores, H <= 1280 */
-  LSTM_APPROX_OPT_TENSOR_SEQ = 8 /* tensor path: 0 = automatic (one launch per
+  LSTM_APPROX_OPT_TENSOR_SEQ = 8, /* tensor path: 0 = automatic (one launch per
                                tile of streams for all T timesteps where the
                                layer fits: K <= 32, H = 256, 512 or 1024,
                                intermediate depths multiples of 16 or >= K,
                                masked-dense tau'), 1 = two launches per
                                timestep */
+  LSTM_APPROX_OPT_LAUNCH_ORDER = 9 /* batch-1 fp32 path with the per-unit-block
+                               kernel: 0 = automatic (the recurrence is
+                               launched before its input projection and
+                               waits, bounded, for flags the projection
+                               raises: the two kernels must be able to run
+                               at the same time), 1 = projection first,
+                               recurrence as its programmatic dependent.
+                               Tools that run kernels one at a time (kernel
+                               profilers, memory checkers) need 1; with 0
+                               under such a tool each run ends in
+                               LSTM_APPROX_ETIMEOUT after the wait limit.
+                               Phase timing (LSTM_APPROX_OPT_TIMING) uses 1. */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 

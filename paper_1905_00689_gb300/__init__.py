@@ -9,7 +9,7 @@ been built.
 from ._binding import (  # noqa: F401
     BF16, FP32, LSTMApprox, LSTMApproxError, dense_run, dense_workspace_bytes, load, plan, run_static, PLAN_KEYS,
     PATH_NONE, PATH_PERSISTENT, PATH_SIMT, PATH_TENSOR,
-    OPT_CLUSTER, OPT_FORCE_PATH, OPT_PERSISTENT_VARIANT, OPT_TAU_LAYOUT, OPT_TENSOR_SEQ, OPT_TEST_STALL, OPT_TIMING,
-    OPT_WAIT_LIMIT, OPT_XPROJ,
+    OPT_CLUSTER, OPT_FORCE_PATH, OPT_LAUNCH_ORDER, OPT_PERSISTENT_VARIANT, OPT_TAU_LAYOUT, OPT_TENSOR_SEQ,
+    OPT_TEST_STALL, OPT_TIMING, OPT_WAIT_LIMIT, OPT_XPROJ,
     Q_CLUSTER, Q_DEVICE_BYTES, Q_LAST_PATH, Q_LAUNCHES, Q_PERSISTENT_VARIANT, Q_TENSOR_SEQ,
 )

@@ -22,7 +22,7 @@ FP32, BF16 = 0, 1
 Q_LAUNCHES, Q_LAST_PATH, Q_CLUSTER, Q_DEVICE_BYTES, Q_PERSISTENT_VARIANT, Q_TENSOR_SEQ = range(6)
 PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
 (OPT_FORCE_PATH, OPT_CLUSTER, OPT_TIMING, OPT_WAIT_LIMIT, OPT_TEST_STALL, OPT_PERSISTENT_VARIANT, OPT_XPROJ,
- OPT_TAU_LAYOUT, OPT_TENSOR_SEQ) = range(9)
+ OPT_TAU_LAYOUT, OPT_TENSOR_SEQ, OPT_LAUNCH_ORDER) = range(10)
 (PLAN_PATH, PLAN_PERSISTENT_VARIANT, PLAN_CLUSTER, PLAN_TERMS_PER_CTA, PLAN_UNITS_PER_WARP, PLAN_TERMS_PER_LANE,
  PLAN_VH_LAYOUT, PLAN_H_QUADS, PLAN_SMEM_BYTES, PLAN_TMEM_COLUMNS, PLAN_TAU_TILE_STREAMS, PLAN_GATE_TILE_STREAMS,
  PLAN_GATE_SPLITS, PLAN_TENSOR_SEQ, PLAN_ITEMS) = range(15)

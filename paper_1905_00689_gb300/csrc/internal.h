@@ -105,6 +105,7 @@ struct lstm_approx {
   int opt_xproj = 0;  // 0 automatic, 1 masked-dense, 2 compressed (fp32, T*B <= 32)
   int opt_tau_layout = 0;  // tensor path's tau': 0 masked-dense (tensor cores), 1 compressed (CUDA cores)
   int opt_tensor_seq = 0;  // tensor path: 0 one launch for all timesteps where the layer fits, 1 per-step launches
+  int opt_launch_order = 0;  // batch-1 persistent path: 0 recurrence before its projection where it applies, 1 after
   long long opt_wait_limit_us = 2000000;
   int opt_test_stall = 0;
   long long launches = 0;

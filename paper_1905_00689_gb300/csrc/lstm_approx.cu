@@ -599,7 +599,7 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     const bool sparse_x = sparse_x_projection(h, s, K, T * B);
     const bool cluster_x = !sparse_x && xproj_cluster_fits(T * B, s.D, s.Vx, s.ldx, in, s.D, bf16);
     bool rec_first = path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && B == 1 && cluster_x &&
-                     !h->timing.on && h->proj_flags != nullptr;
+                     !h->timing.on && h->opt_launch_order == 0 && h->proj_flags != nullptr;
     const int proj_ctas = rec_first ? xproj_cluster_ctas(K, T * B, s.D, 8) : 0;
     rec_first = rec_first && proj_ctas <= kProjFlags && xproj_cluster_prepare(bf16, T * B) == cudaSuccess;
     const int xproj_max_split =
@@ -1181,6 +1181,10 @@ int lstm_approx_set_option(lstm_approx_t* h, int key, long long value) {
     case LSTM_APPROX_OPT_TENSOR_SEQ:
       if (value < 0 || value > 1) return fail(h, LSTM_APPROX_EINVAL, "bad tensor launch choice %lld", value);
       h->opt_tensor_seq = (int)value;
+      return LSTM_APPROX_OK;
+    case LSTM_APPROX_OPT_LAUNCH_ORDER:
+      if (value < 0 || value > 1) return fail(h, LSTM_APPROX_EINVAL, "bad launch order %lld", value);
+      h->opt_launch_order = (int)value;
       return LSTM_APPROX_OK;
     case LSTM_APPROX_OPT_PERSISTENT_VARIANT:
       if (value < 0 || value > 2) return fail(h, LSTM_APPROX_EINVAL, "bad persistent variant %lld", value);

@@ -13,8 +13,8 @@ import pytest
 
 from parity_util import (FP32_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run,
                          persistent_layout_cases, run_gpu, synthetic_layer, workload_inputs)
-from paper_1905_00689_gb300 import (FP32, OPT_TIMING, PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH, Q_LAUNCHES,
-                                    Q_PERSISTENT_VARIANT, plan)
+from paper_1905_00689_gb300 import (FP32, OPT_LAUNCH_ORDER, OPT_TIMING, PATH_PERSISTENT, Q_CLUSTER, Q_LAST_PATH,
+                                    Q_LAUNCHES, Q_PERSISTENT_VARIANT, plan)
 from workloads import draw_factor_set, draw_inputs
 
 pytestmark = pytest.mark.gpu
@@ -183,8 +183,9 @@ def test_launch_orders_agree(cuda_device):
     got, m = run_gpu(layers, x, K, force_path=PATH_PERSISTENT, variant=1, checkpoints=cps, max_rank=256)
     assert_parity(got, ref, FP32_TOL)
     n0 = m.query(Q_LAUNCHES)
-    for timing in (0, 1, 0, 1, 0):
+    for timing, order in ((0, 0), (1, 0), (0, 0), (0, 1), (0, 0)):
         m.set_option(OPT_TIMING, timing)
+        m.set_option(OPT_LAUNCH_ORDER, order)
         again = _run_again(m, x, K, 512, cps)
         assert_parity(again, ref, FP32_TOL, keys=("h", "ckpt_h"))
     assert m.query(Q_LAUNCHES) - n0 == 5 * 2  # projection and recurrence in either order
