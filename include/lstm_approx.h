@@ -191,8 +191,14 @@ int lstm_approx_run_static(const float *Vx, const float *Vh, const float *U, con
  *   x, h0, c0, out_h, out_c: as lstm_approx_run with L = 1 (DEVICE, fp32)
  *   workspace  DEVICE buffer of at least
  *              lstm_approx_dense_workspace_bytes(H, T, B) bytes, 256-byte
- *              aligned, owned by the caller (the hoisted Wx x_t and a status
- *              word); it must not be used by another call in flight
+ *              aligned, owned by the caller (the hoisted Wx x_t, a status
+ *              word and the projection's completion flags); it must not be
+ *              used by another call in flight
+ *
+ * For one stream the recurrence is launched before the input projection and
+ * waits (bounded) for flags the projection raises, as lstm_approx_run does
+ * (LSTM_APPROX_OPT_LAUNCH_ORDER): the two kernels must be able to run at the
+ * same time, which tools that run one kernel at a time do not allow.
  *   cuda_stream  cudaStream_t (NULL = legacy default stream)
  *   msg   optional host buffer of msg_len bytes for an error text
  *

@@ -40,6 +40,9 @@ using namespace lstm_approx_dev;
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
+// workspace of lstm_approx_dense_run: status word, projection flags, P
+constexpr size_t kDenseFlagsOffset = 256;
+constexpr size_t kDensePOffset = kDenseFlagsOffset + kProjFlags * sizeof(unsigned);
 
 struct DenseArgs {
   const float* Wh;    // [4H][H], row g*H + j = the recurrent part of row j of W_g
@@ -52,6 +55,11 @@ struct DenseArgs {
   int* err;
   int H, T, B, CS, UB;
   long long limit_ns;
+  // non-null when the projection that writes P is launched after this kernel
+  // (the approximate path's launch order, XprojSignal)
+  const unsigned* proj_flags;
+  int proj_nflags;
+  unsigned proj_epoch;
 };
 
 // Sum of NV values over the 32 lanes, transposed (high lane bits first):
@@ -91,6 +99,8 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(DenseArgs a) {
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
+  // a projection launched after this kernel may start now (it waits for nothing)
+  if (a.proj_flags != nullptr) griddep_launch_dependents();
   const int b = blockIdx.x / CS;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
   const volatile int* err = a.err;
@@ -172,16 +182,23 @@ __global__ void __launch_bounds__(kThreads, 1) dense_kernel(DenseArgs a) {
   const bool cell_lane = warp == 0 && lane < UB && cj < H;
   float c_reg = (cell_lane && a.c0 != nullptr) ? a.c0[(long long)b * H + cj] : 0.f;
 
-  griddep_wait();  // P is written by the projection launched just before this kernel
-  float p_cur = (writer && my_j < H) ? __ldg(a.P + (long long)b * 4 * H + p_off) : 0.f;
+  // P is written by the projection launched just before this kernel, or just
+  // after it (its CTAs then each raise a flag once their part is stored)
+  bool setup_ok = true;
+  if (a.proj_flags == nullptr) griddep_wait();
+  else if (warp == 0) setup_ok = wait_flags_epoch(a.proj_flags, a.proj_nflags, a.proj_epoch, limit, err);
+  if (!__syncthreads_and(setup_ok) && tid == 0) atomicCAS(a.err, 0, kErrWaitTimeoutA);
+  // P through L2 (it may have been written while this kernel ran)
+  float p_cur = (writer && my_j < H) ? __ldcg(a.P + (long long)b * 4 * H + p_off) : 0.f;
   const uint32_t bar_h0 = smem_u32(&bars[0]);
   cluster_sync_all();  // every CTA's barriers are armed before any st.async
+  const int t_end = *err == 0 ? a.T : 0;  // nothing to do after a failed set-up
 
   bool failed = false;
-  for (int t = 0; t < a.T && !failed; ++t) {
+  for (int t = 0; t < t_end && !failed; ++t) {
     const int hb = t & 1;
     const float p_next = (writer && my_j < H && t + 1 < a.T)
-                             ? __ldg(a.P + ((long long)(t + 1) * a.B + b) * 4 * H + p_off)
+                             ? __ldcg(a.P + ((long long)(t + 1) * a.B + b) * 4 * H + p_off)
                              : 0.f;
     bool fail = false;
     if (t > 0) {
@@ -298,8 +315,9 @@ cudaError_t launch_dense_t(const DenseArgs& a, cudaStream_t s) {
   attr[0].val.clusterDim.x = a.CS;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // after the projection: its programmatic dependent; before it: an ordinary launch
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].val.programmaticStreamSerializationAllowed = a.proj_flags == nullptr ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, a);
@@ -329,8 +347,11 @@ bool plan_dense(int H, int* CS, int* UB, int* HQ) {
 
 cudaError_t launch_dense(const float* Wh, const float* bias, const float* P, const float* h0, const float* c0,
                          float* out_h, float* c_last, int* err, int H, int T, int B, long long limit_ns,
-                         cudaStream_t s) {
+                         cudaStream_t s, const unsigned* proj_flags, int proj_nflags, unsigned proj_epoch) {
   DenseArgs a{};
+  a.proj_flags = proj_flags;
+  a.proj_nflags = proj_nflags;
+  a.proj_epoch = proj_epoch;
   int HQ = 0;
   if (!plan_dense(H, &a.CS, &a.UB, &HQ)) return cudaErrorInvalidValue;
   a.Wh = Wh;
@@ -375,18 +396,37 @@ extern "C" int lstm_approx_dense_run(const float* Wx, const float* Wh, const flo
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (major != 10 || minor != 3) return report(msg, msg_len, LSTM_APPROX_ECUDA, "needs an sm_103 device");
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  // workspace: the status word, the projection's completion flags, then P
   int* status = static_cast<int*>(workspace);
-  float* P = reinterpret_cast<float*>(static_cast<char*>(workspace) + 256);
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), s);
+  unsigned* flags = reinterpret_cast<unsigned*>(static_cast<char*>(workspace) + kDenseFlagsOffset);
+  float* P = reinterpret_cast<float*>(static_cast<char*>(workspace) + kDensePOffset);
   // Wx x_t for all t: the approximate path's projection with the 4H gate rows
-  // of Wx in place of the pruned v rows (K = Ks = H)
-  if (e == cudaSuccess)
-    e = xproj_cluster_fits(T * B, D, Wx, D, x, D, false)
-            ? launch_xproj_cluster(Wx, false, D, H, H, x, D, T * B, D, P, 4 * H, status, 2000000000LL, s, 8)
-            : launch_rows_gemm(Wx, false, D, H, H, x, D, T * B, D, P, 4 * H, 0, nullptr, nullptr, 0, s);
+  // of Wx in place of the pruned v rows (K = Ks = H).  For one stream it is
+  // launched after the recurrence, as the approximate path does (the flags
+  // are cleared first, every call, so that epoch 1 always marks this call).
+  const bool cluster_x = xproj_cluster_fits(T * B, D, Wx, D, x, D, false);
+  const int proj_ctas = cluster_x ? xproj_cluster_ctas(H, T * B, D, 8) : 0;
+  const bool rec_first = B == 1 && cluster_x && proj_ctas <= kProjFlags &&
+                         xproj_cluster_prepare(false, T * B) == cudaSuccess;
+  cudaError_t e = cudaMemsetAsync(workspace, 0, kDensePOffset, s);
+  XprojSignal sig;
+  sig.flags = flags;
+  sig.epoch = 1u;
+  auto projection = [&]() {
+    return cluster_x ? launch_xproj_cluster(Wx, false, D, H, H, x, D, T * B, D, P, 4 * H, status, 2000000000LL, s,
+                                            8, rec_first ? &sig : nullptr)
+                     : launch_rows_gemm(Wx, false, D, H, H, x, D, T * B, D, P, 4 * H, 0, nullptr, nullptr, 0, s);
+  };
+  if (e == cudaSuccess && !rec_first) e = projection();
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "projection launch: %s", cudaGetErrorString(e));
-  e = launch_dense(Wh, bias, P, h0, c0, out_h, out_c, status, H, T, B, 2000000000LL, s);
+  e = launch_dense(Wh, bias, P, h0, c0, out_h, out_c, status, H, T, B, 2000000000LL, s, rec_first ? flags : nullptr,
+                   proj_ctas, 1u);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "recurrence launch: %s", cudaGetErrorString(e));
+  if (rec_first) {
+    e = projection();
+    if (e != cudaSuccess)
+      return report(msg, msg_len, LSTM_APPROX_ECUDA, "projection launch: %s", cudaGetErrorString(e));
+  }
   e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return report(msg, msg_len, LSTM_APPROX_ECUDA, "synchronise: %s", cudaGetErrorString(e));
   int code = 0;
@@ -398,5 +438,5 @@ extern "C" int lstm_approx_dense_run(const float* Wx, const float* Wh, const flo
 
 extern "C" size_t lstm_approx_dense_workspace_bytes(int H, int T, int B) {
   if (H < 1 || T < 1 || B < 1) return 0;
-  return 256 + (size_t)T * B * 4 * H * sizeof(float);
+  return kDensePOffset + (size_t)T * B * 4 * H * sizeof(float);
 }
