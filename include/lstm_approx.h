@@ -370,7 +370,9 @@ enum lstm_approx_plan_item {
                                               all T (then CLUSTER = H / 128 CTAs per tile and both
                                               tile items = the streams per tile), 0 = two launches
                                               per timestep */
-  LSTM_APPROX_PLAN_ITEMS = 14
+  LSTM_APPROX_PLAN_TAU_SPLITS = 14,        /* tensor path: CTAs of a cluster over which the tau'
+                                              GEMM splits its reduction axis (H), 1 = none */
+  LSTM_APPROX_PLAN_ITEMS = 15
 };
 int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int *checkpoints, int J,
                      int force_path, int cluster, int persistent_variant, int *out, int n_out,

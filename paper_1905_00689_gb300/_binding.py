@@ -25,10 +25,10 @@ PATH_NONE, PATH_SIMT, PATH_PERSISTENT, PATH_TENSOR = range(4)
  OPT_TAU_LAYOUT, OPT_TENSOR_SEQ, OPT_LAUNCH_ORDER) = range(10)
 (PLAN_PATH, PLAN_PERSISTENT_VARIANT, PLAN_CLUSTER, PLAN_TERMS_PER_CTA, PLAN_UNITS_PER_WARP, PLAN_TERMS_PER_LANE,
  PLAN_VH_LAYOUT, PLAN_H_QUADS, PLAN_SMEM_BYTES, PLAN_TMEM_COLUMNS, PLAN_TAU_TILE_STREAMS, PLAN_GATE_TILE_STREAMS,
- PLAN_GATE_SPLITS, PLAN_TENSOR_SEQ, PLAN_ITEMS) = range(15)
+ PLAN_GATE_SPLITS, PLAN_TENSOR_SEQ, PLAN_TAU_SPLITS, PLAN_ITEMS) = range(16)
 PLAN_KEYS = ("path", "persistent_variant", "cluster", "terms_per_cta", "units_per_warp", "terms_per_lane",
              "vh_layout", "h_quads", "smem_bytes", "tmem_columns", "tau_tile_streams", "gate_tile_streams",
-             "gate_splits", "tensor_seq")
+             "gate_splits", "tensor_seq", "tau_splits")
 STATUS_NAMES = {OK: "OK", EINVAL: "EINVAL", ENOMEM: "ENOMEM", ECUDA: "ECUDA", ETIMEOUT: "ETIMEOUT",
                 ESTATE: "ESTATE"}
 

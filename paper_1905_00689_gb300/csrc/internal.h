@@ -289,6 +289,11 @@ struct TcRowsArgs {
   long long tau_plane;
   int* err;
   long long limit_ns;
+  // mode 1 only: the reduction axis split over the sk CTAs of a cluster
+  // (grid z), nkb_per 64-element chunks each; each CTA then finishes
+  // 128 / sk rows of the tile from all sk partial sums (1: no split)
+  int sk;
+  int nkb_per;
 };
 // `bn` (64, 128 or 256) must match the box rows of Bm's map.
 cudaError_t launch_tc_rows(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, int n_cols, int bn, cudaStream_t s);

@@ -148,9 +148,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   constexpr int kNb = XF ? 3 * S : 2 * S;  // full[S] | empty[S] (| converted[S])
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t bar0 = base + S * kStage;  // the stage barriers, accum | drain | tmem slot
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (kNb + 2));
-  const uint32_t accum_bar = bar0 + 8u * kNb, drain_bar = accum_bar + 8u;
+  const uint32_t bar0 = base + S * kStage;  // the stage barriers, accum | drain | split | tmem slot
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (bar0 - raw) + 8 * (kNb + 3));
+  const uint32_t accum_bar = bar0 + 8u * kNb, drain_bar = accum_bar + 8u, split_bar = accum_bar + 16u;
   const uint32_t conv0 = bar0 + 8u * (2 * S);  // converted[s] (XF)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -163,9 +163,19 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const uint32_t a_bytes = rpg > 0 ? 4u * rpg * kTileK * 2 : kABytes;
   const int col0 = blockIdx.y * BN;
   const int nkb = (a.Kdim + kTileK - 1) / kTileK;
+  // reduction axis split over the sk CTAs of a cluster (grid z, mode 1):
+  // this CTA's 64-element chunks [kb0, kb0 + nloc)
+  const int sk = (!XF && BN <= 64 && a.sk > 1) ? a.sk : 1;
+  const int kb0 = sk > 1 ? (int)blockIdx.z * a.nkb_per : 0;
+  const int nloc = sk > 1 ? max(0, min(nkb, kb0 + a.nkb_per) - kb0) : nkb;
   const volatile int* err = a.err;
   const uint64_t limit = static_cast<uint64_t>(a.limit_ns);
   const bool add_p = a.mode == 1;  // tau' = sigma * (accumulator + P_t)
+  // split (sk > 1, tiles of at most 64 columns): an epilogue thread's row and
+  // columns of this CTA's partial sums, and that row's sigma and P_t
+  constexpr int kSplitCols = BN <= 64 ? BN / 2 : 1;
+  float sp_val[kSplitCols], sp_p[kSplitCols];
+  float sp_sig = 0.f;
 
   griddep_launch_dependents();  // the next kernel may start its own set-up
   if (threadIdx.x == 0) {
@@ -176,7 +186,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     mbar_init(accum_bar, 1);
     mbar_init(drain_bar, 1);
+    // split: the partial sums of this CTA's rows pushed by the sk - 1 peers
+    if (sk > 1) mbar_init(split_bar, 1);
     fence_mbarrier_init_cluster();
+    if (sk > 1) mbar_arrive_expect_tx(split_bar, (uint32_t)((sk - 1) * (kTileM / sk) * BN * 4));
   }
   if (rpg > 0) {  // the factor tile's rows no copy writes: zero in every stage, before the MMAs read them
     const uint32_t zbytes = kABytes - a_bytes;
@@ -211,18 +224,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     bool ok = true;
     // the factor tiles of the first S stages do not depend on the kernel
     // before this one: issue them before waiting for it
-    const int npre = nkb < S ? nkb : S;
+    const int npre = nloc < S ? nloc : S;
     constexpr uint32_t b_bytes = 2 * kBBytes;  // the pair, or (XF) the fp32 tile: the same bytes
-    for (int kb = 0; kb < npre; ++kb) {
-      mbar_arrive_expect_tx(bar0 + 8u * kb, a_bytes + b_bytes);
-      load_a(base + kb * kStage, bar0 + 8u * kb, kb);
+    for (int i = 0; i < npre; ++i) {
+      mbar_arrive_expect_tx(bar0 + 8u * i, a_bytes + b_bytes);
+      load_a(base + i * kStage, bar0 + 8u * i, kb0 + i);
     }
     griddep_wait();
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % S;
-      if (kb >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((kb / S) - 1) & 1, limit, err))) break;
+    for (int i = 0; i < nloc; ++i) {
+      const int s = i % S, kb = kb0 + i;
+      if (i >= S && !(ok = wait_cta(bar0 + 8u * (S + s), ((i / S) - 1) & 1, limit, err))) break;
       const uint32_t st = base + s * kStage;
-      if (kb >= npre) {
+      if (i >= npre) {
         mbar_arrive_expect_tx(bar0 + 8u * s, a_bytes + b_bytes);
         load_a(st, bar0 + 8u * s, kb);
       }
@@ -244,17 +257,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1 && lane == 0) {  // ---- MMA issuer ----
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, BN);
     bool ok = true;
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-      const int s = kb % S;
+    for (int i = 0; i < nloc && ok; ++i) {
+      const int s = i % S;
       // the stage's copies have landed (XF: and its activation has been converted)
-      if (!(ok = wait_cta((XF ? conv0 : bar0) + 8u * s, (kb / S) & 1, limit, err))) break;
+      if (!(ok = wait_cta((XF ? conv0 : bar0) + 8u * s, (i / S) & 1, limit, err))) break;
       tc_fence_after();
       const uint32_t st = base + s * kStage;
       const uint64_t da = umma_desc_sw128(st);
       const uint64_t dhi = umma_desc_sw128(st + kABytes), dlo = umma_desc_sw128(st + kABytes + kBBytes);
 #pragma unroll
       for (int kk = 0; kk < kTileK / 16; ++kk) {
-        umma_bf16(tmem, da + 2ull * kk, dhi + 2ull * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+        umma_bf16(tmem, da + 2ull * kk, dhi + 2ull * kk, idesc, (i | kk) != 0 ? 1u : 0u);
         umma_bf16(tmem, da + 2ull * kk, dlo + 2ull * kk, idesc, 1u);
       }
       umma_commit(bar0 + 8u * (S + s));  // frees the stage once these MMAs are done
@@ -321,6 +334,29 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int row = rpg > 0 ? (lrow / rpg) * a.Ks + k : row0 + lrow;
     const bool row_ok = k < a.K && (rpg == 0 || lrow < 4 * rpg);
     const uint32_t trow = tmem + ((32u * q) << 16);
+    if (sk > 1) {
+      // split: this thread's row and columns of the CTA's partial sums, and
+      // (for the row's owner, below) its sigma and P_t, loaded while the
+      // mainloop runs
+      if constexpr (BN <= 64) {
+#pragma unroll
+        for (int c = 0; c < kHalf; ++c) {
+          const int n = col0 + cbeg + c;
+          sp_p[c] = (row_ok && n < a.N) ? __ldg(a.P + (long long)n * a.ldp + row) : 0.f;
+        }
+        sp_sig = row_ok ? a.sigma[row] : 0.f;
+        const bool ok = wait_cta(accum_bar, 0, limit, err);
+        tc_fence_after();
+#pragma unroll
+        for (int cc = 0; cc < kHalf; cc += 16) {
+          float v[16];
+          tmem_ld16(trow + cbeg + cc, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) sp_val[cc + j] = (ok && nloc > 0) ? v[j] : 0.f;
+        }
+      }
+    } else {
     float preg[kHalf];  // P_t of this thread's row and columns, loaded while the mainloop runs
     if (add_p) {
 #pragma unroll
@@ -354,6 +390,57 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           a.tau[a.tau_plane + (long long)n * a.ldt + row] = lo;
         }
       }
+    }
+    }
+  }
+  if constexpr (BN <= 64) {
+    if (sk > 1) {
+      // Every CTA of the cluster holds its partial sums of the whole tile (in
+      // its epilogue threads' registers); CTA z finishes rows
+      // [z RS, (z + 1) RS).  The threads of other rows push their values
+      // into the owner's receive buffer (over its stage ring, free once the
+      // cluster barrier shows every accumulator complete) with st.async,
+      // which completes the owner's split barrier; each owning thread adds
+      // the sk partials of its row in rank order (the result does not depend
+      // on timing), forms tau' = sigma (sum + P_t) and stores its pair.
+      __syncwarp();  // warps 0 and 1 reconverge after their single-lane roles
+      cluster_sync_all();
+      if (warp >= 4) {
+        const int ep = warp - 4, q = ep & 3, lrow = 32 * q + lane, cbeg = (ep >> 2) * (BN / 2);
+        const int z = (int)blockIdx.z, RS = kTileM / sk, owner = lrow / RS;
+        constexpr int RSTR = BN + 4;  // receive-row stride in floats (16-byte rows, banks skewed)
+        // receive buffer [sender][row of the owner's block][RSTR] at the start of the stage ring
+        const uint32_t recv = base;
+        if (owner != z) {
+          const uint32_t dst = mapa_shared(recv, (uint32_t)owner) +
+                               4u * (uint32_t)((z * RS + (lrow - owner * RS)) * RSTR + cbeg);
+          const uint32_t bar = mapa_shared(split_bar, (uint32_t)owner);
+#pragma unroll
+          for (int c = 0; c < BN / 2; c += 4)
+            st_async_v4(dst + 4u * c, sp_val[c], sp_val[c + 1], sp_val[c + 2], sp_val[c + 3], bar);
+        } else {
+          const bool got = mbar_wait_bounded<true>(split_bar, 0, limit, err);  // pushes from other CTAs
+          const float* rb = reinterpret_cast<const float*>(smem_raw + (recv - raw));
+          griddep_wait();  // tau' may still be read by the kernel before this one
+          const bool write = got && *err == 0;
+          const int kr = kt * kTileM + lrow;
+#pragma unroll
+          for (int c = 0; c < BN / 2; ++c) {
+            float sum = 0.f;
+#pragma unroll
+            for (int zz = 0; zz < 4; ++zz)
+              if (zz < sk) sum += zz == z ? sp_val[c] : rb[(zz * RS + (lrow - z * RS)) * RSTR + cbeg + c];
+            const int n = col0 + cbeg + c;
+            if (write && n < a.N) {
+              __nv_bfloat16 hi, lo;
+              bf16_pair(kr < a.K ? sp_sig * (sum + sp_p[c]) : 0.f, hi, lo);
+              a.tau[(long long)n * a.ldt + row0 + lrow] = hi;
+              a.tau[a.tau_plane + (long long)n * a.ldt + row0 + lrow] = lo;
+            }
+          }
+        }
+      }
+      cluster_sync_all();  // no CTA leaves while pushes towards it may still be in flight
     }
   }
   tc_fence_before();
@@ -793,7 +880,7 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, size_t smem, cudaStream_t s, Args..
 
 template <int BN, int S, bool XF>
 size_t rows_smem() {
-  return 1024 + S * (kABytes + 2 * BN * kTileK * 2) + 8 * ((XF ? 3 : 2) * S + 2) + 16;
+  return 1024 + S * (kABytes + 2 * BN * kTileK * 2) + 8 * ((XF ? 3 : 2) * S + 3) + 16;
 }
 template <int NT, int S>
 size_t gates_smem() {
@@ -810,9 +897,30 @@ cudaError_t launch_rows_t(const TcMap& A, const TcMap& Bm, const TcRowsArgs& a, 
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  return launch_pdl(kern, dim3(a.rpg > 0 ? 1 : 4 * a.kt_per_gate, (n_cols + BN - 1) / BN), smem, s,
-                    *reinterpret_cast<const CUtensorMap*>(A.bytes), *reinterpret_cast<const CUtensorMap*>(Bm.bytes),
-                    a);
+  static_assert((size_t)kTileM * (BN + 4) * 4 <= (size_t)S * (kABytes + 2 * BN * kTileK * 2),
+                "a split's receive buffer fits over the stage ring");
+  const int sk = (!XF && a.sk > 1) ? a.sk : 1;
+  const dim3 grid(a.rpg > 0 ? 1 : 4 * a.kt_per_gate, (n_cols + BN - 1) / BN, sk);
+  if (sk == 1)
+    return launch_pdl(kern, grid, smem, s, *reinterpret_cast<const CUtensorMap*>(A.bytes),
+                      *reinterpret_cast<const CUtensorMap*>(Bm.bytes), a);
+  // the sk CTAs of a split tile form one cluster along z
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kTcThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attrs[2];
+  attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attrs[0].val.programmaticStreamSerializationAllowed = 1;
+  attrs[1].id = cudaLaunchAttributeClusterDimension;
+  attrs[1].val.clusterDim.x = 1;
+  attrs[1].val.clusterDim.y = 1;
+  attrs[1].val.clusterDim.z = sk;
+  cfg.attrs = attrs;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, *reinterpret_cast<const CUtensorMap*>(A.bytes),
+                            *reinterpret_cast<const CUtensorMap*>(Bm.bytes), a);
 }
 
 template <int NT, int S, bool SPLIT>

@@ -231,6 +231,7 @@ int select_path(int dtype, int H, int K, int T, const Checkpoints& ck, int force
 
 struct TensorTiles {
   int bnh = 0, nt = 0, ks = 1, nkb_per = 0;
+  int sk = 1, nkb_per_h = 0;  // the tau' GEMM's splits of its reduction axis (H) and 64-chunks per split
   bool raw = false;  // raw gate sums and a reduce kernel (term split, or depths off the 16-term slices)
 };
 
@@ -245,6 +246,23 @@ TensorTiles tensor_tiles(int H, int B, int K, const Checkpoints& ck) {
   TensorTiles t;
   // packed gates: one row tile, so narrower stream tiles keep more SMs busy
   t.bnh = tensor_rows_per_gate(K) > 0 ? 32 : tc_rows_tile_n(B, 4 * ((K + 127) / 128));
+  if (tensor_rows_per_gate(K) == 0) {
+    // few tiles of 64 streams over a long reduction axis (H >= 1024): split
+    // it over a cluster of 4 CTAs instead of narrowing the stream tiles, so
+    // that each CTA streams a quarter of the factor rows.  Measured (whole
+    // recurrence): the two-layer D=4096 H=2048 B=64 K=1024 workload 1207 ->
+    // 1165 us; splitting in two at D=1024 H=512 B=256 K=512 (383 -> 460 us)
+    // and at D=2048 H=1024 B=1024 K=128 (1209 -> 1316 us) cost more in
+    // cluster barriers and pushes than the shorter streams save.
+    const int row_tiles = 4 * ((K + 127) / 128), nkbh = (H + 63) / 64;
+    const long long tiles64 = (long long)row_tiles * ((B + 63) / 64);
+    int sk = tiles64 * 4 <= 148 && nkbh >= 16 ? 4 : 1;
+    if (sk > 1) {
+      t.bnh = 64;
+      t.nkb_per_h = (nkbh + sk - 1) / sk;
+      t.sk = (nkbh + t.nkb_per_h - 1) / t.nkb_per_h;  // no empty split
+    }
+  }
   t.nt = tc_gates_tile_n(H, B);
   const int gate_tiles = ((H + 127) / 128) * ((B + t.nt - 1) / t.nt);
   t.ks = tc_gates_splits(gate_tiles, (K + 63) / 64, &t.nkb_per);
@@ -463,6 +481,8 @@ int run_layer_tensor(lstm_approx_t* h, int l, const float* x, int T, int B, int 
     ra.tau_plane = (long long)B * ldp;
     ra.err = h->err;
     ra.limit_ns = limit_ns;
+    ra.sk = tt.sk;
+    ra.nkb_per = tt.nkb_per_h;
     if (h->opt_tau_layout == 1) {  // compressed rows of v's h part on the CUDA cores
       TauSparseArgs sa{};
       sa.off = s.hoff;
@@ -1263,11 +1283,13 @@ int lstm_approx_plan(int dtype, int hidden, int T, int B, int K, const int* chec
       v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = ns;
       v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = ns;
       v[LSTM_APPROX_PLAN_GATE_SPLITS] = 1;
+      v[LSTM_APPROX_PLAN_TAU_SPLITS] = 1;
     } else {
       const TensorTiles tt = tensor_tiles(hidden, B, K, ck);
       v[LSTM_APPROX_PLAN_TAU_TILE_STREAMS] = tt.bnh;
       v[LSTM_APPROX_PLAN_GATE_TILE_STREAMS] = tt.nt;
       v[LSTM_APPROX_PLAN_GATE_SPLITS] = tt.ks;
+      v[LSTM_APPROX_PLAN_TAU_SPLITS] = tt.sk;
     }
   }
   for (int i = 0; i < n_out; ++i) out[i] = i < LSTM_APPROX_PLAN_ITEMS ? v[i] : 0;

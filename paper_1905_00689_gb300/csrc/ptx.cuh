@@ -119,6 +119,13 @@ __device__ __forceinline__ void bulk_copy_s2cluster(uint32_t dst_cluster, uint32
       : "memory");
 }
 
+// 4-byte load from shared memory of a CTA of the cluster (address from mapa).
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+
 // Orders this thread's generic-proxy shared-memory writes before later
 // async-proxy (bulk copy) reads of them.
 __device__ __forceinline__ void fence_proxy_async_shared() {

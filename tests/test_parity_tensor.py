@@ -11,7 +11,7 @@ import pytest
 
 from parity_util import (BF16_TOL, WORKLOADS, assert_parity, decomposed_layer, oracle_run, run_gpu,
                          synthetic_layer, workload_inputs)
-from paper_1905_00689_gb300 import PATH_SIMT, PATH_TENSOR, Q_LAST_PATH
+from paper_1905_00689_gb300 import BF16, PATH_SIMT, PATH_TENSOR, Q_LAST_PATH, plan
 from workloads import draw_factor_set, draw_inputs
 
 pytestmark = pytest.mark.gpu
@@ -41,6 +41,11 @@ def _sample(got, streams, T=None):
     (40, 200, 4, 3, 80, 70, [5, 21, 79]),
     (48, 128, 3, 8, 256, 100, [5, 67, 130, 200, 256]),
     (64, 136, 2, 40, 45, 80, [1, 17, 45]),
+    # tau' with its reduction axis (H >= 1024) split over clusters of 4 CTAs:
+    # ragged H (the last split shorter), K off the 128-row tiles, two tiles
+    # of 64 streams with a ragged tail
+    (64, 1000, 3, 70, 200, 300, [16, 200]),
+    (32, 1024, 2, 9, 130, 400, [64, 129]),
 ])
 def test_tensor_path_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     gates = [draw_factor_set(H, D + H, K, nz, 5100 + 7 * D + g) for g in range(4)]
@@ -52,6 +57,8 @@ def test_tensor_path_small_shapes(cuda_device, D, H, T, B, K, nz, cps):
     c0 = 0.3 * rng.standard_normal((1, B, H))
     got, m = run_gpu([gates], x, K, dtype="bf16", h0=h0, c0=c0, checkpoints=cps, force_path=PATH_TENSOR)
     assert m.query(Q_LAST_PATH) == PATH_TENSOR
+    if H >= 1000:  # the cases above meant to split tau'
+        assert plan(BF16, H, T, B, K, cps, PATH_TENSOR)["tau_splits"] == 4
     ref = oracle_run([gates], x, K, dtype="bf16", h0=h0, c0=c0, checkpoints=cps)
     assert_parity(got, ref, BF16_TOL)
 

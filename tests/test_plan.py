@@ -49,14 +49,20 @@ def test_large_batch_workloads():
     # D=1024, H=512, B=256, K=512: 4 unit tiles x 8 tiles of 32 streams, the
     # terms split 4 ways to fill the GPU
     p = plan(BF16, 512, 20, 256, 512)
-    assert (p["path"], p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"]) == (PATH_TENSOR, 32, 4, 32)
+    assert (p["path"], p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"], p["tau_splits"]) == \
+        (PATH_TENSOR, 32, 4, 32, 1)
     # D=2048, H=1024, B=1024, K=512: 8 x 16 tiles of 64 streams, no split;
     # the tau' GEMM's 16 row tiles take 128 streams per tile
     p = plan(BF16, 1024, 64, 1024, 512)
-    assert (p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"]) == (64, 1, 128)
-    # second layer of D=4096, H=2048, B=64, K=1024 with four depths
+    assert (p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"], p["tau_splits"]) == (64, 1, 128, 1)
+    # the same at K = 128: 4 row tiles x 32 tiles of 32 streams
+    p = plan(BF16, 1024, 64, 1024, 128)
+    assert (p["tau_tile_streams"], p["tau_splits"]) == (32, 1)
+    # second layer of D=4096, H=2048, B=64, K=1024 with four depths (tau':
+    # 32 row tiles of 64 streams, H split over clusters of 4)
     p = plan(BF16, 2048, 16, 64, 1024, [16, 64, 256, 1024])
-    assert (p["path"], p["gate_tile_streams"], p["gate_splits"]) == (PATH_TENSOR, 32, 4)
+    assert (p["path"], p["gate_tile_streams"], p["gate_splits"], p["tau_tile_streams"], p["tau_splits"]) == \
+        (PATH_TENSOR, 32, 4, 64, 4)
 
 
 # ---- the rules -----------------------------------------------------------------
@@ -137,8 +143,9 @@ def test_tensor_tiles(H, B, K):
     """Stream tiles: the narrowest of 32/64/128 (gates) that keeps the grid
     within one wave of 148 CTAs, else the widest; tau' takes 32 streams up to
     K = 32 (one tile of all four gates' rows), else the narrowest of 32/64
-    that keeps one wave, else 128; the gate GEMM's terms split over
-    min(148 // tiles, 8, chunks of 64) CTAs."""
+    that keeps one wave, else 128, except where few tiles of 64 streams
+    over H >= 1024 split its reduction axis over clusters of 4 CTAs; the gate GEMM's
+    terms split over min(148 // tiles, 8, chunks of 64) CTAs."""
     p = plan(BF16, H, 2, B, K)
     if K <= 32 and H in (256, 512, 1024):  # one launch for all timesteps (test_tensor_seq_plan)
         assert p["tensor_seq"] == 1
@@ -149,7 +156,13 @@ def test_tensor_tiles(H, B, K):
     assert p["gate_tile_streams"] == nt
     rows = 4 * -(-K // 128)
     bn = 32 if K <= 32 else next((n for n in (32, 64) if rows * -(-B // n) <= 148), 128)
-    assert p["tau_tile_streams"] == bn
+    # few tiles of 64 streams over H >= 1024: the reduction axis over clusters of 4
+    tiles64, hchunks = rows * -(-B // 64), -(-H // 64)
+    sk = 1 if K <= 32 else 4 if tiles64 * 4 <= 148 and hchunks >= 16 else 1
+    if sk > 1:
+        bn, per = 64, -(-hchunks // sk)
+        sk = -(-hchunks // per)
+    assert (p["tau_tile_streams"], p["tau_splits"]) == (bn, sk)
     tiles = units * -(-B // nt)
     chunks = -(-K // 64)
     ks = min(148 // tiles, 8, chunks)
