@@ -795,7 +795,8 @@ def run_profile(args):
     from paper_1905_00689_gb300 import LSTMApprox, Q_LAST_PATH
     w = WORKLOADS[args.profile]
     if args.profile_dense:  # the dense comparator kernel on this workload's shape (fp32, one layer)
-        from paper_1905_00689_gb300 import dense_run
+        from paper_1905_00689_gb300 import dense_run, dense_set_launch_order
+        dense_set_launch_order(1)  # a profiler runs kernels one at a time: projection first
         from workloads import draw_weight
         dev = torch.device("cuda", 0)
         W = [draw_weight(w.H, w.D + w.H, 77 + g) for g in range(4)]

@@ -212,6 +212,11 @@ int lstm_approx_dense_run(const float *Wx, const float *Wh, const float *bias, i
                           void *cuda_stream, char *msg, int msg_len);
 /* Workspace bytes lstm_approx_dense_run needs for (H, T, B); 0 for invalid sizes. */
 size_t lstm_approx_dense_workspace_bytes(int H, int T, int B);
+/* Launch order of lstm_approx_dense_run for every later call in the process,
+ * as LSTM_APPROX_OPT_LAUNCH_ORDER: 0 = automatic (recurrence first for one
+ * stream), 1 = projection first (what tools that run one kernel at a time
+ * need).  Returns OK or EINVAL (another value). */
+int lstm_approx_dense_set_launch_order(int order);
 
 /*
  * Wait for the handle's stream and report kernel-side status: OK, or

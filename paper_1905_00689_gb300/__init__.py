@@ -7,7 +7,8 @@ Importing the package does not load the library; constructing
 been built.
 """
 from ._binding import (  # noqa: F401
-    BF16, FP32, LSTMApprox, LSTMApproxError, dense_run, dense_workspace_bytes, load, plan, run_static, PLAN_KEYS,
+    BF16, FP32, LSTMApprox, LSTMApproxError, dense_run, dense_set_launch_order, dense_workspace_bytes, load, plan,
+    run_static, PLAN_KEYS,
     PATH_NONE, PATH_PERSISTENT, PATH_SIMT, PATH_TENSOR,
     OPT_CLUSTER, OPT_FORCE_PATH, OPT_LAUNCH_ORDER, OPT_PERSISTENT_VARIANT, OPT_TAU_LAYOUT, OPT_TENSOR_SEQ,
     OPT_TEST_STALL, OPT_TIMING, OPT_WAIT_LIMIT, OPT_XPROJ,

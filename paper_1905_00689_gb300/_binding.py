@@ -37,6 +37,7 @@ EXPORTS = (
     "lstm_approx_sync", "lstm_approx_get_mask", "lstm_approx_last_error", "lstm_approx_destroy",
     "lstm_approx_query", "lstm_approx_set_option", "lstm_approx_phase_times", "lstm_approx_run_static",
     "lstm_approx_plan", "lstm_approx_get_term", "lstm_approx_dense_run", "lstm_approx_dense_workspace_bytes",
+    "lstm_approx_dense_set_launch_order",
 )
 
 _lib = None
@@ -79,6 +80,7 @@ def load(path: str = LIB_PATH):
     lib.lstm_approx_dense_run.argtypes = [P, P, P, I, I, P, I, I, P, P, P, P, P, ctypes.c_size_t, P,
                                           ctypes.c_char_p, I]
     lib.lstm_approx_dense_workspace_bytes.argtypes = [I, I, I]
+    lib.lstm_approx_dense_set_launch_order.argtypes = [I]
     for name in EXPORTS:
         if name not in ("lstm_approx_last_error", "lstm_approx_destroy", "lstm_approx_dense_workspace_bytes"):
             getattr(lib, name).restype = ctypes.c_int
@@ -148,6 +150,13 @@ def dense_run(Wx, Wh, bias, x, out_h, h0=None, c0=None, out_c=None, workspace=No
 
 def dense_workspace_bytes(H: int, T: int, B: int) -> int:
     return int(load().lstm_approx_dense_workspace_bytes(H, T, B))
+
+
+def dense_set_launch_order(order: int) -> None:
+    """lstm_approx_dense_set_launch_order (process-wide)."""
+    rc = load().lstm_approx_dense_set_launch_order(order)
+    if rc != OK:
+        raise LSTMApproxError(rc, f"bad launch order {order}")
 
 
 def plan(dtype: int, hidden: int, T: int, B: int, K: int, checkpoints: Sequence[int] = (), force_path: int = 0,

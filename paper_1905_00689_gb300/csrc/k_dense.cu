@@ -27,6 +27,7 @@
 // the tau' exchange as well.  Every wait is bounded in wall time; a wait that
 // runs out writes the status word, the CTA leaves the loop, and the cluster
 // meets at a final barrier.
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 
@@ -376,6 +377,16 @@ cudaError_t launch_dense(const float* Wh, const float* bias, const float* P, con
 
 using namespace lstm_approx_impl;
 
+namespace {
+std::atomic<int> g_dense_launch_order{0};
+}  // namespace
+
+extern "C" int lstm_approx_dense_set_launch_order(int order) {
+  if (order < 0 || order > 1) return LSTM_APPROX_EINVAL;
+  g_dense_launch_order.store(order);
+  return LSTM_APPROX_OK;
+}
+
 extern "C" int lstm_approx_dense_run(const float* Wx, const float* Wh, const float* bias, int D, int H,
                                      const float* x, int T, int B, const float* h0, const float* c0, float* out_h,
                                      float* out_c, void* workspace, size_t workspace_bytes, void* cuda_stream,
@@ -406,7 +417,7 @@ extern "C" int lstm_approx_dense_run(const float* Wx, const float* Wh, const flo
   // are cleared first, every call, so that epoch 1 always marks this call).
   const bool cluster_x = xproj_cluster_fits(T * B, D, Wx, D, x, D, false);
   const int proj_ctas = cluster_x ? xproj_cluster_ctas(H, T * B, D, 8) : 0;
-  const bool rec_first = B == 1 && cluster_x && proj_ctas <= kProjFlags &&
+  const bool rec_first = B == 1 && cluster_x && proj_ctas <= kProjFlags && g_dense_launch_order.load() == 0 &&
                          xproj_cluster_prepare(false, T * B) == cudaSuccess;
   cudaError_t e = cudaMemsetAsync(workspace, 0, kDensePOffset, s);
   XprojSignal sig;

@@ -47,10 +47,19 @@ def test_dense_kernel_matches_oracle(cuda_device, D, H, T, B, extras):
     Wh = f32(np.concatenate([w[:, D:] for w in W]))
     out_h = torch.full((T, B, H), float("nan"), device=dev)
     out_c = torch.full((B, H), float("nan"), device=dev)
-    for _ in range(2):  # twice: the workspace and the kernel's barriers start from scratch each call
-        dense_run(Wx, Wh, f32(bias), f32(x), out_h, h0=f32(h0), c0=f32(c0), out_c=out_c)
-        got = {"h": out_h.double().cpu().numpy(), "c_last": out_c.double().cpu().numpy()}
-        assert_parity(got, {"h": ref_h, "c_last": ref_c}, FP32_TOL)
+    from paper_1905_00689_gb300 import dense_set_launch_order
+    # twice in each launch order (one stream: recurrence first by default, then
+    # projection first): the workspace, its flags and the kernel's barriers
+    # start from scratch each call
+    try:
+        for order in (0, 0, 1, 1, 0):
+            dense_set_launch_order(order)
+            out_h.fill_(float("nan"))
+            dense_run(Wx, Wh, f32(bias), f32(x), out_h, h0=f32(h0), c0=f32(c0), out_c=out_c)
+            got = {"h": out_h.double().cpu().numpy(), "c_last": out_c.double().cpu().numpy()}
+            assert_parity(got, {"h": ref_h, "c_last": ref_c}, FP32_TOL)
+    finally:
+        dense_set_launch_order(0)
 
 
 def test_dense_kernel_refuses_what_it_cannot_take(cuda_device):
