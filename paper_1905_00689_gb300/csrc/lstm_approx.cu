@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -791,6 +792,10 @@ int lstm_approx_create(lstm_approx_t** out, int num_layers, const int* input_dim
   h->stream = static_cast<cudaStream_t>(cuda_stream);
   h->device = dev;
   h->sm_count = prop.multiProcessorCount;
+  // with every launch made blocking, the recurrence can never run beside the
+  // projection launched after it: start with the projection first
+  const char* blocking = std::getenv("CUDA_LAUNCH_BLOCKING");
+  if (blocking != nullptr && blocking[0] == '1') h->opt_launch_order = 1;
   h->layers.resize(num_layers);
   int rc = LSTM_APPROX_OK;
   for (int l = 0; l < num_layers && !rc; ++l) {

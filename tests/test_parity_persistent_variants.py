@@ -206,3 +206,27 @@ def test_launch_orders_two_layer_stack(cuda_device):
             got = _run_again(m, x, K, H, [8, 32])
         assert m.query(Q_PERSISTENT_VARIANT) == 1
         assert_parity(got, ref, FP32_TOL, keys=("h", "ckpt_h"))
+
+
+def test_blocking_launches_take_the_projection_first(cuda_device):
+    """With CUDA_LAUNCH_BLOCKING=1 no two kernels run side by side: a handle
+    created then starts with the projection first, and the batch-1 run of
+    the per-unit-block kernel completes and matches the oracle."""
+    import os
+    import subprocess
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    code = (
+        "import sys; sys.path[:0] = [%r, %r]\n"
+        "import numpy as np\n"
+        "from parity_util import FP32_TOL, assert_parity, decomposed_layer, oracle_run, run_gpu, WORKLOADS, "
+        "workload_inputs\n"
+        "from paper_1905_00689_gb300 import PATH_PERSISTENT\n"
+        "layers = [list(decomposed_layer('c1', 0, 16, 0.5))]\n"
+        "x = workload_inputs(WORKLOADS['c1'])\n"
+        "got, m = run_gpu(layers, x, 16, force_path=PATH_PERSISTENT, variant=1, checkpoints=[4])\n"
+        "assert_parity(got, oracle_run(layers, x, 16, checkpoints=[4]), FP32_TOL, keys=('h', 'ckpt_h'))\n"
+        "print('ok')\n") % (here, os.path.dirname(here))
+    env = dict(os.environ, CUDA_LAUNCH_BLOCKING="1")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout[-2000:] + r.stderr[-2000:]
