@@ -318,9 +318,11 @@ enum lstm_approx_option_key {
                                profilers, memory checkers) need 1; with 0
                                under such a tool each run ends in
                                LSTM_APPROX_ETIMEOUT after the wait limit.
-                               Phase timing (LSTM_APPROX_OPT_TIMING) uses 1;
-                               a handle created with CUDA_LAUNCH_BLOCKING=1
-                               in the environment starts at 1. */
+                               Phase timing (LSTM_APPROX_OPT_TIMING) and
+                               runs on a stream being captured into a CUDA
+                               graph use 1; a handle created with
+                               CUDA_LAUNCH_BLOCKING=1 in the environment
+                               starts at 1. */
 };
 int lstm_approx_set_option(lstm_approx_t *h, int key, long long value);
 

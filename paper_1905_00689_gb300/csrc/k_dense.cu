@@ -419,8 +419,10 @@ extern "C" int lstm_approx_dense_run(const float* Wx, const float* Wh, const flo
   const bool cluster_x = xproj_cluster_fits(T * B, D, Wx, D, x, D, false);
   const int proj_ctas = cluster_x ? xproj_cluster_ctas(H, T * B, D, 8) : 0;
   const char* blocking = std::getenv("CUDA_LAUNCH_BLOCKING");  // every launch blocking: never side by side
+  cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;  // (the call synchronises: never captured,
+  if (cudaStreamIsCapturing(s, &capture) != cudaSuccess) capture = cudaStreamCaptureStatusActive;  // but checked)
   const bool rec_first = B == 1 && cluster_x && proj_ctas <= kProjFlags && g_dense_launch_order.load() == 0 &&
-                         !(blocking != nullptr && blocking[0] == '1') &&
+                         !(blocking != nullptr && blocking[0] == '1') && capture == cudaStreamCaptureStatusNone &&
                          xproj_cluster_prepare(false, T * B) == cudaSuccess;
   cudaError_t e = cudaMemsetAsync(workspace, 0, kDensePOffset, s);
   XprojSignal sig;

@@ -603,7 +603,8 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // takes its SMs at once, the projection follows as its programmatic
     // dependent on the SMs left free and raises one flag per CTA, and the
     // recurrence loads its factors meanwhile and waits for the flags before
-    // its first read of P (D = 1024, H = 512, T = 20, whole call: K = 256
+    // its first read of P, unless the stream is being captured into a graph
+    // (D = 1024, H = 512, T = 20, whole call: K = 256
     // with two intermediate depths 64.1 -> 60.0 us, K = 64 46.8 -> 45.0 us;
     // with the projection split four ways along D, 128 CTAs, 68.7 us).  The
     // one-exchange kernel's short set-up gains nothing from it (K = 16:
@@ -619,8 +620,14 @@ int run_device(lstm_approx_t* h, const float* x, int T, int B, int K, const floa
     // slower, the one-exchange kernel at K = 16: 11%).
     const bool sparse_x = sparse_x_projection(h, s, K, T * B);
     const bool cluster_x = !sparse_x && xproj_cluster_fits(T * B, s.D, s.Vx, s.ldx, in, s.D, bf16);
+    // (not while the stream is being captured: a graph would replay the
+    // launches with the epoch value of the capture, and the flags of the
+    // previous replay would already hold it)
+    cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(h->stream, &capture) != cudaSuccess) capture = cudaStreamCaptureStatusActive;
     bool rec_first = path == LSTM_APPROX_PATH_PERSISTENT && plan.variant == 1 && B == 1 && cluster_x &&
-                     !h->timing.on && h->opt_launch_order == 0 && h->proj_flags != nullptr;
+                     !h->timing.on && h->opt_launch_order == 0 && h->proj_flags != nullptr &&
+                     capture == cudaStreamCaptureStatusNone;
     const int proj_ctas = rec_first ? xproj_cluster_ctas(K, T * B, s.D, 8) : 0;
     rec_first = rec_first && proj_ctas <= kProjFlags && xproj_cluster_prepare(bf16, T * B) == cudaSuccess;
     const int xproj_max_split =

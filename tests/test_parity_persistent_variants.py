@@ -230,3 +230,39 @@ def test_blocking_launches_take_the_projection_first(cuda_device):
     env = dict(os.environ, CUDA_LAUNCH_BLOCKING="1")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout[-2000:] + r.stderr[-2000:]
+
+
+def test_graph_replays_with_new_inputs(cuda_device):
+    """A batch-1 run of the per-unit-block kernel captured into a CUDA graph
+    (where the projection comes first) and replayed after the input changed
+    in place matches the oracle on the new input each time."""
+    import torch
+    from paper_1905_00689_gb300 import LSTMApprox
+    D, H, T, K = 96, 256, 5, 48
+    layers = [[draw_factor_set(H, D + H, K, 120, 1800 + g) for g in range(4)]]
+    xs = [draw_inputs(T, 1, D, "uniform", 30 + i) for i in range(3)]
+    stream = torch.cuda.Stream()
+    m = LSTMApprox(1, [D], H, K, 1, "fp32", stream=stream)
+    m.set_layer(0, layers[0])
+    from paper_1905_00689_gb300 import OPT_FORCE_PATH, OPT_PERSISTENT_VARIANT
+    m.set_option(OPT_FORCE_PATH, PATH_PERSISTENT)
+    m.set_option(OPT_PERSISTENT_VARIANT, 1)
+    x = torch.from_numpy(xs[0].astype(np.float32)).cuda()
+    out = torch.zeros((T, 1, H), device="cuda")
+    ck = torch.zeros((1, T, 1, H), device="cuda")
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        m.run(x, K, out, checkpoints=[8], ckpt_h=ck)  # eager, recurrence first
+    m.sync()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        m.run(x, K, out, checkpoints=[8], ckpt_h=ck)
+    for xi in xs[1:] + xs[:1]:
+        with torch.cuda.stream(stream):
+            x.copy_(torch.from_numpy(xi.astype(np.float32)))
+            g.replay()
+        stream.synchronize()
+        ref = oracle_run(layers, xi, K, checkpoints=[8])
+        assert_parity({"h": out.double().cpu().numpy(), "ckpt_h": ck.double().cpu().numpy()}, ref, FP32_TOL,
+                      keys=("h", "ckpt_h"))
+    assert m.query(Q_PERSISTENT_VARIANT) == 1
