@@ -54,7 +54,7 @@ L2_FLUSH_BYTES = 256 << 20
 # holds only for the kernel sources it was taken on: `captured_traffic`
 # returns None once their SHA-256 differs.
 TRAFFIC_SOURCES = ("k_persistent.cu", "ptx.cuh")
-TRAFFIC_CAPTURE = {"sha256": "4e1582bdcb57173f701f21ac68af5e314f2f08d10e7251f5a26b389824dc7535",
+TRAFFIC_CAPTURE = {"sha256": "74b3043aed6800cc4782c7daec6ca4f72bc8c4a7bf4ec800d298c7eadca2fe73",
                    "bytes": 4345600}
 
 
