@@ -61,6 +61,11 @@ def test_invalid_arguments_rejected_before_any_device_work(built_lib):
     assert built_lib.lstm_approx_sync(None) == 1
     built_lib.lstm_approx_destroy(None)
     assert built_lib.lstm_approx_last_error(None) == b"invalid handle (NULL)"
+    # the dense comparator's process-wide launch order: 0 or 1 only
+    assert built_lib.lstm_approx_dense_set_launch_order(2) == 1
+    assert built_lib.lstm_approx_dense_set_launch_order(-1) == 1
+    assert built_lib.lstm_approx_dense_set_launch_order(1) == 0
+    assert built_lib.lstm_approx_dense_set_launch_order(0) == 0
 
 
 def test_no_cpu_fallback_without_a_device(built_lib):
