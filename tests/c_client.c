@@ -23,5 +23,10 @@ int main(void) {
   printf("create %d %s\n", rc, h == NULL ? "null" : "handle");
   printf("error %s\n", lstm_approx_last_error(NULL));
   lstm_approx_destroy(h);
+  rc = lstm_approx_plan(LSTM_APPROX_BF16, 2048, 16, 64, 1024, NULL, 0, 0, 0, 0, out, LSTM_APPROX_PLAN_ITEMS, msg,
+                        (int)sizeof msg);
+  printf("tensor plan %d tau splits %d tau streams %d\n", rc, out[LSTM_APPROX_PLAN_TAU_SPLITS],
+         out[LSTM_APPROX_PLAN_TAU_TILE_STREAMS]);
+  printf("dense order %d %d\n", lstm_approx_dense_set_launch_order(1), lstm_approx_dense_set_launch_order(0));
   return 0;
 }

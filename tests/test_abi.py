@@ -98,6 +98,8 @@ def test_header_is_c_and_a_c_client_links(built_lib, tmp_path):
     if not torch.cuda.is_available():
         assert lines[2] == "create 3 null"  # ECUDA: no CPU fallback
     assert lines[3] == "error invalid handle (NULL)"
+    assert lines[4] == "tensor plan 0 tau splits 4 tau streams 64"
+    assert lines[5] == "dense order 0 0"
 
 
 def test_product_path_does_not_import_the_oracle():
