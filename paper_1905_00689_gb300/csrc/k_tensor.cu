@@ -405,6 +405,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       // on timing), forms tau' = sigma (sum + P_t) and stores its pair.
       __syncwarp();  // warps 0 and 1 reconverge after their single-lane roles
       cluster_sync_all();
+      bool split_failed = false;  // an owning thread's wait for the pushes ran out
       if (warp >= 4) {
         const int ep = warp - 4, q = ep & 3, lrow = 32 * q + lane, cbeg = (ep >> 2) * (BN / 2);
         const int z = (int)blockIdx.z, RS = kTileM / sk, owner = lrow / RS;
@@ -420,6 +421,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             st_async_v4(dst + 4u * c, sp_val[c], sp_val[c + 1], sp_val[c + 2], sp_val[c + 3], bar);
         } else {
           const bool got = mbar_wait_bounded<true>(split_bar, 0, limit, err);  // pushes from other CTAs
+          split_failed = !got;
           const float* rb = reinterpret_cast<const float*>(smem_raw + (recv - raw));
           griddep_wait();  // tau' may still be read by the kernel before this one
           const bool write = got && *err == 0;
@@ -440,7 +442,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
         }
       }
-      cluster_sync_all();  // no CTA leaves while pushes towards it may still be in flight
+      // A CTA may leave once the pushes towards it have landed, which its
+      // owning threads waited for (a CTA that only pushes leaves at once, so
+      // the next kernel's CTAs can take its SM); if such a wait ran out,
+      // pushes may still be in flight: let them land first.
+      if (__syncthreads_or(split_failed)) {
+        const uint64_t t0 = global_timer_ns();
+        while (global_timer_ns() - t0 < 50000ull) __nanosleep(1000);
+      }
     }
   }
   tc_fence_before();
