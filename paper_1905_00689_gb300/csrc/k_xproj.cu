@@ -329,17 +329,22 @@ int xproj_split(int row_tiles, int col_chunks, int D, int max_split) {
   return S;
 }
 
-// Sets the kernel's shared-memory limit once per thread; this also loads the
-// kernel's code if the module is loaded lazily, which a launch that must
-// start while another kernel runs (XprojSignal) cannot wait for.
+// Sets the kernel's shared-memory limit once per thread and device; this
+// also loads the kernel's code on that device if the module is loaded
+// lazily, which a launch that must start while another kernel runs
+// (XprojSignal) cannot wait for.
 template <typename TF, int NC>
 cudaError_t prepare_nc() {
-  static thread_local bool attr_set = false;
-  if (!attr_set) {
-    const cudaError_t e = cudaFuncSetAttribute(xproj_kernel<TF, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)smem_bytes<TF, NC>());
+  static thread_local unsigned long long done = 0;  // bit d: device d prepared
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+  if (bit == 0 || (done & bit) == 0) {
+    e = cudaFuncSetAttribute(xproj_kernel<TF, NC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem_bytes<TF, NC>());
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    done |= bit;
   }
   return cudaSuccess;
 }
